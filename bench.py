@@ -1,0 +1,328 @@
+"""Throughput of fused-tile execution of the YOLOv2 first-16-layer front-end on GB300.
+
+One step = one mafat_run of the whole plan (every fused layer group, every
+tile) over one batch of synthetic input already resident in HBM.  Default
+workload: 608x608x3, batch 1, bf16, two layer groups cut after layer 7, group 1
+tiled 5x5 and group 2 tiled 2x2.  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mafat|reference] [--workload NAME]
+
+--impl reference times the fp64 CPU oracle on the host cores (the only other
+place this script runs oracle code, together with the cpu_baseline leg).
+Under torchrun (N > 1) every rank runs an independent replica on its own GPU
+(the method does not shard a frame across devices); rank 0 reports the frames
+of all ranks over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "frames/s (YOLOv2 first 16 layers, 608x608, bf16, fused tiles)"
+DEFAULT_WORKLOAD = "yolo16_608_5x5_c8_2x2"
+L2_FLUSH_BYTES = 256 << 20
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+KERNEL_SOURCES = ["kernel_tc.cu", "sched.cuh", "device_types.h", "planner.cpp"]
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2107_06960_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            p = json.load(fh)
+        return float(p["bf16_tflops"]), float(p["bf16_tflops_sustained"]), float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def aggregate(units_per_rank, seconds_per_rank):
+    """Whole-job throughput of independent replicas: all units over the slowest rank's time."""
+    return float(sum(units_per_rank)) / float(max(seconds_per_rank))
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.QUERY, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() in ("active", "1"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def cpu_oracle_rate(wl, budget_s=12.0):
+    """The oracle as it stands (fp64, OpenMP over rows) on the host cores: frames/s on whole frames."""
+    import oracle
+    x = wl["input"][0]
+    n, t0 = 0, time.perf_counter()
+    while True:
+        oracle.forward(wl["layers"], wl["params"], x)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or n >= 8:
+            break
+    return n / el, oracle.num_threads(), "%d whole %dx%d frame(s), unfused fp64 forward of all %d layers" % (
+        n, wl["h"], wl["w"], len(wl["layers"]))
+
+
+def run_reference(args, wl):
+    """--impl reference: the CPU oracle timed per step on a bounded sample of the workload."""
+    import oracle
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return
+    layers, params = wl["layers"], wl["params"]
+    full = oracle.conv_flops(layers, oracle.layer_shapes(layers, wl["h"], wl["w"], 3))
+    # size the per-step sample so the whole run stays within about two minutes
+    t0 = time.perf_counter()
+    oracle.forward(layers, params, wl["input"][0][:152, :152])
+    t_small = time.perf_counter() - t0
+    est_full = t_small * (wl["h"] * wl["w"]) / (152 * 152)
+    steps = args.steps + args.warmup
+    side = wl["h"]
+    while side > 64 and est_full * (side * side) / (wl["h"] * wl["w"]) * steps > 120.0:
+        side //= 2
+    side = max(16, side - side % 16)
+    x = wl["input"][0][:side, :side]
+    frac = oracle.conv_flops(layers, oracle.layer_shapes(layers, side, side, 3)) / full
+    for _ in range(args.warmup):
+        oracle.forward(layers, params, x)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.forward(layers, params, x)
+    el = time.perf_counter() - t0
+    value = frac * args.steps / el
+    sample = "%dx%d crop per step (%.4f of a frame's FLOPs), unfused fp64 forward" % (side, side, frac)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "input": "%dx%dx3" % (wl["h"], wl["w"]), "batch": wl["batch"]},
+        "cpu_baseline": {"value": value, "unit": "frames/s", "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "frames/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="mafat", choices=["mafat", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    wl = synth.workload(args.workload)
+
+    if args.impl == "reference":
+        run_reference(args, wl)
+        return
+
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    import paper_2107_06960_gb300 as mf
+
+    ws, rank, local = dist_env()
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        pg = dist
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    B, H, W = wl["batch"], wl["h"], wl["w"]
+    net = mf.Net(wl["layers"], H, W, 3)
+    net.set_params(wl["params"])
+    dt = mf.BF16 if wl["dtype"] == "bf16" else mf.FP32
+    tdt = torch.bfloat16 if dt == mf.BF16 else torch.float32
+    plan = mf.Plan(net, wl["cut"], wl["grids"], batch=B, dtype=dt)
+    st = plan.stats()
+    sh = net.shape(len(wl["layers"]) - 1)
+    xin = torch.from_numpy(mf.to_planar(wl["input"])).to(tdt).to(dev)
+    out = torch.empty((B, sh[3], sh[4], sh[5]), dtype=tdt, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        plan.run(xin, out, stream=stream)
+    plan.sync_status(stream=stream)
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        flush.fill_(i)                       # write 256 MiB: evicts the 129 MB L2 (not timed)
+        starts[i].record(stream)
+        plan.run(xin, out, stream=stream)    # one kernel launch
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    clk = clocks.stop()
+    plan.sync_status(stream=stream)
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    dev_s = sum(step_ms) / 1e3
+
+    # end to end through the C ABI on pinned host buffers (copies inside the timed region)
+    xh = xin.cpu().pin_memory()
+    oh = torch.empty(out.shape, dtype=tdt).pin_memory()
+    for _ in range(2):
+        plan.run_host(xh, oh, stream=stream)
+    torch.cuda.synchronize()
+    e2e_steps = max(5, min(args.steps, 50))
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        plan.run_host(xh, oh, stream=stream)
+    e2e_s = time.perf_counter() - t0
+
+    if pg:
+        t = torch.tensor([dev_s, e2e_s], dtype=torch.float64, device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        dev_s_max, e2e_s_max = float(t[0]), float(t[1])
+    else:
+        dev_s_max, e2e_s_max = dev_s, e2e_s
+    if rank != 0:
+        if pg:
+            pg.destroy_process_group()
+        return
+
+    frames = B * args.steps
+    value = aggregate([frames] * ws, [dev_s_max])
+    e2e_value = aggregate([B * e2e_steps] * ws, [e2e_s_max])
+    peak_burst, peak_sus, hbm, peak_src = measured_peaks()
+    avg_launch_s = dev_s / args.steps
+    achieved_tf = st["useful_flops"] / avg_launch_s / 1e12
+    traffic = None
+    try:
+        with open(TRAFFIC_FILE) as fh:
+            tr = json.load(fh)
+        ent = tr.get(args.workload)
+        if ent and ent.get("kernel_source_hash") == kernel_source_hash():
+            traffic = ent["dram_bytes_per_launch"]
+    except Exception:
+        pass
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        v, cores, sample = cpu_oracle_rate(wl)
+        cpu = {"value": v, "unit": "frames/s", "cores": cores, "kind": "oracle", "sample": sample}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if dt == mf.BF16 else "f32", "data": "synthetic",
+        "config": {
+            "workload": args.workload, "input": "%dx%dx3" % (H, W), "batch": B,
+            "cut": wl["cut"], "grids": "/".join("%dx%d" % tuple(gd) for gd in wl["grids"]),
+            "l2": "flushed before every timed step (256 MiB write, not timed)",
+            "useful_gflop_per_frame": st["useful_flops"] / B / 1e9,
+            "executed_gflop_per_frame": st["executed_flops"] / B / 1e9,
+            "halo_recompute": st["executed_flops"] / st["useful_flops"] - 1.0,
+            "issued_gflop_per_frame": st["issued_flops"] / B / 1e9,
+            "group_io_mb_per_frame": st["group_io_bytes"] / B / 1e6,
+            "weight_mb": st["weight_bytes"] / 1e6,
+            "predicted_mib_alg1": st["predicted_mib"],
+            "ctas": st["max_ctas"], "work_items": st["n_items"],
+            "step_ms_min": min(step_ms), "step_ms_median": statistics.median(step_ms),
+        },
+        "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_burst, "unit": "TFLOP/s",
+                     "frac": achieved_tf / peak_burst, "traffic": traffic,
+                     "kernel": "mafat_tc_kernel", "flops": "useful (unfused network) per launch",
+                     "peak_source": "%s dense bf16 burst" % peak_src},
+        "e2e": {"value": e2e_value, "unit": "frames/s", "h2d_bytes_per_step": int(xh.numel() * xh.element_size()),
+                "d2h_bytes_per_step": int(oh.numel() * oh.element_size())},
+        "gpu_launches": args.steps * plan.launches_per_run(),
+        "clocks": clk,
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    print(json.dumps(line), flush=True)
+    if pg:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,235 @@
+/*
+ * mafat.h -- C ABI of a GB300 (sm_103a) implementation of fused-tile execution
+ * of CNN layer groups, after MAFAT: Memory-Aware Fusing and Tiling of Neural
+ * Networks for Accelerated Edge Inference (Farley & Gerstlauer, arXiv
+ * 2107.06960).
+ *
+ * The method (Sec. 3-4): a stack of n convolution / max-pool layers is cut into
+ * at most two layer groups (group 1 = layers 0..cut-1, group 2 = cut..n-1).
+ * The last-layer output of each group is split into an even N x M grid of
+ * tiles; every tile's input region (with the overlap, or halo, its receptive
+ * field needs) is found by walking the layers of the group backwards, and the
+ * tile runs all layers of its group as one fused unit.  The group-1 tiles are
+ * merged into the full cut tensor, which group 2 re-tiles.  Sec. 4.1-4.2 add a
+ * memory predictor (Algorithm 1) and a configuration search (Algorithm 2).
+ *
+ * Conventions shared by every call:
+ *  - Every call returns a mafat_status; nothing aborts, exits or throws.  On
+ *    failure mafat_last_error() returns a message for the calling thread.
+ *  - Handles are created and destroyed only by this library.
+ *  - Layers are numbered from 0.  A "cut" is the index of the first layer of
+ *    group 2 (the paper's cut); cut <= 0 or cut >= n means a single group.
+ *  - Rectangles are int32_t[4] = {y0, y1, x0, x1}, half-open, in the
+ *    coordinates of the feature map they live on.
+ *  - A grid N x M has N tiles along rows (height) and M along columns.
+ *  - Streams are passed as void* holding a cudaStream_t (NULL = legacy default).
+ *  - Device pointers must be 16-byte aligned and must not alias each other.
+ *
+ * Supported layers: 3x3 / stride 1 / pad 1 and 1x1 / stride 1 / pad 0
+ * convolutions with folded batch-norm (per-channel scale and bias) followed by
+ * leaky ReLU with slope 0.1, and 2x2 / stride 2 max-pool layers that directly
+ * follow a convolution of the same group (they are fused into it).  Output
+ * channel counts must be multiples of 8; input channel counts above 8 must be
+ * multiples of 16; a 1x1 convolution needs at least 9 input channels.
+ */
+#ifndef MAFAT_H
+#define MAFAT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MAFAT_OK = 0,
+    MAFAT_EINVAL = 1,        /* bad argument (null pointer, bad size, misaligned pointer) */
+    MAFAT_EUNSUPPORTED = 2,  /* valid request this library does not implement */
+    MAFAT_ENOMEM = 3,        /* host or device allocation failed */
+    MAFAT_ECUDA = 4,         /* a CUDA runtime call failed */
+    MAFAT_ETIMEOUT = 5,      /* a bounded device-side wait on another tile ran out */
+    MAFAT_ENOFIT = 6,        /* a plan's per-tile working set cannot be scheduled */
+    MAFAT_EDEVICE = 7        /* a bounded device-side pipeline wait ran out (internal error) */
+} mafat_status;
+
+typedef enum { MAFAT_CONV = 0, MAFAT_MAXPOOL = 1 } mafat_layer_type;
+
+/* Arithmetic of a plan.  BF16: bf16 activations and weights, fp32 accumulation
+ * on the tensor cores (tcgen05), every layer output rounded to bf16.  FP32: the
+ * same fused tiling computed in fp32 on the CUDA cores (a check mode). */
+typedef enum { MAFAT_BF16 = 0, MAFAT_FP32 = 1 } mafat_dtype;
+
+/* One layer of the network description (the W, H, F, S vectors of Sec. 4.1 and
+ * Algorithm 2: filter size k = F_l, stride = S_l; W_l, H_l and channel counts
+ * are inferred).  `filters` is the output channel count of a convolution and is
+ * ignored for a max-pool. */
+typedef struct {
+    int32_t type;     /* mafat_layer_type */
+    int32_t k;
+    int32_t stride;
+    int32_t pad;
+    int32_t filters;
+} mafat_layer_desc;
+
+typedef struct mafat_net_s mafat_net_t;
+typedef struct mafat_plan_s mafat_plan_t;
+
+/* Optional knobs of mafat_plan_ex.  Zero-initialise and set struct_size. */
+typedef struct {
+    int32_t struct_size;        /* sizeof(mafat_plan_options) */
+    int32_t ring_slots;         /* tiles whose intermediate buffers may be live at once (0: default) */
+    int32_t wave_tiles;         /* tiles whose layers are interleaved in the work order (0: = ring_slots) */
+    int32_t max_ctas;           /* persistent CTAs (0: one per SM) */
+    int64_t wait_timeout_ns;    /* limit of a device-side wait before MAFAT_ETIMEOUT (0: 2 s) */
+    int32_t test_unpublished_task; /* test hook: index of a task whose completion is never
+                                      published, so that waits on it run out (-1: none) */
+    int32_t dry_run;            /* 1: build the host-side tables only (statistics and region
+                                   queries work; runs are refused); needs no GPU */
+    int32_t reserved[6];
+} mafat_plan_options;
+
+/* Statistics of a plan (all per batch unless stated). */
+typedef struct {
+    int32_t struct_size;
+    int32_t n_groups;
+    int32_t n_tiles;            /* non-empty tiles over all groups and frames */
+    int32_t n_tasks;            /* (frame, tile, fused conv stage) units */
+    int64_t n_items;            /* work items handed out by the persistent scheduler */
+    double useful_flops;        /* 2*MAC of the convolutions of the unfused network */
+    double executed_flops;      /* 2*MAC over all tile regions (includes halo recompute) */
+    double issued_flops;        /* 2*MAC issued to the arithmetic units (includes block padding) */
+    double predicted_mib;       /* Algorithm 1 (literal reading, bias 31 MiB) for this configuration */
+    int64_t group_io_bytes;     /* group inputs + group outputs, once each */
+    int64_t weight_bytes;       /* packed weights + scale/bias */
+    int64_t scratch_bytes;      /* device buffers of live tile intermediates */
+    int64_t workspace_bytes;    /* all device memory the plan owns */
+    int64_t smem_bytes_per_cta; /* on-chip shared memory per CTA */
+    int32_t ring_slots;
+    int32_t wave_tiles;
+    int32_t max_ctas;
+    int32_t dtype;
+} mafat_plan_stats;
+
+/* Build a network description: validates the layers and infers every layer's
+ * shape, out = floor((in + 2*pad - k) / stride) + 1 (Sec. 4.1, Algorithm 2's
+ * W, H, F, S).  in_c is the channel count of the input image.  The caller keeps
+ * ownership of `layers`.  EUNSUPPORTED for layer types/shapes outside the
+ * supported set above (e.g. a max-pool on an odd-sized map). */
+mafat_status mafat_describe_net(const mafat_layer_desc* layers, int32_t n,
+                                int32_t in_h, int32_t in_w, int32_t in_c,
+                                mafat_net_t** out);
+
+/* Shape of layer `layer`: shape[6] = {h_in, w_in, c_in, h_out, w_out, c_out}. */
+mafat_status mafat_net_shape(const mafat_net_t* net, int32_t layer, int32_t shape[6]);
+
+/* Set the parameters of convolution layer `layer`: w_host [Cout][Cin][k][k]
+ * (cross-correlation), scale[Cout] and bias[Cout] of the folded batch-norm,
+ * all host fp32.  The library copies them; the caller keeps ownership.
+ * Plans created afterwards use these values (bf16 plans round w to bf16,
+ * nearest-even). */
+mafat_status mafat_set_weights(mafat_net_t* net, int32_t layer, const float* w_host,
+                               const float* scale, const float* bias);
+
+/* Plan fused-tile execution (Sec. 4): n_groups (1 or 2) layer groups split at
+ * cuts[0] (ignored for one group), group g tiled grid_n[g] x grid_m[g], for
+ * `batch` images, in dtype dt.  The plan owns its device workspace (packed
+ * weights, cut tensor, tile buffers, counters) on the current device; every
+ * convolution must have weights set.  ENOFIT if a tile cannot be scheduled,
+ * EUNSUPPORTED if a max-pool would be separated from its convolution.
+ * Allocates device memory; not for use during stream capture. */
+mafat_status mafat_plan(const mafat_net_t* net, int32_t n_groups, const int32_t* cuts,
+                        const int32_t* grid_n, const int32_t* grid_m, int32_t batch,
+                        int32_t dt, mafat_plan_t** out);
+
+/* mafat_plan with options (may be NULL). */
+mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32_t* cuts,
+                           const int32_t* grid_n, const int32_t* grid_m, int32_t batch,
+                           int32_t dt, const mafat_plan_options* opt, mafat_plan_t** out);
+
+/* Run the plan on `stream` (asynchronous): one persistent fused kernel.
+ *   input : device, [batch][ceil(C/8)][H][W][8] elements of the plan's dtype
+ *           (channel octets outermost; for C <= 8 this is NHWC with the
+ *           channel dimension padded to 8), padded channels zero.
+ *   output: device, NHWC [batch][H_out][W_out][C_out] of the plan's dtype.
+ * Both caller-owned.  Returns launch errors only; device-side wait errors are
+ * reported by mafat_sync_status.  Calls on one plan must not overlap in time
+ * (they share the plan's workspace).  Capturable into a CUDA graph. */
+mafat_status mafat_run(const mafat_plan_t* plan, const void* input, void* output, void* stream);
+
+/* mafat_run, then copy the group-1 output (the cut tensor, layout
+ * [batch][C/8][H][W][8]) into cut_out (device, caller-owned); for a
+ * single-group plan cut_out is ignored. */
+mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* cut_out,
+                             void* output, void* stream);
+
+/* End-to-end call on HOST buffers (same layouts as mafat_run): copies the input
+ * to plan-owned device memory, runs, copies the output back and synchronises
+ * `stream`; returns the device status as mafat_sync_status does.  Pinned host
+ * memory gives asynchronous copies. */
+mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, void* output_host,
+                            void* stream);
+
+/* Synchronise `stream` and read (and clear) the plan's device status word:
+ * MAFAT_OK, MAFAT_ETIMEOUT (a tile waited on another that never finished) or
+ * MAFAT_EDEVICE. */
+mafat_status mafat_sync_status(const mafat_plan_t* plan, void* stream);
+
+/* Host-side query of the Grid traversal (Sec. 4.1): input and output
+ * rectangle of layer `layer` for tile (ti, tj) of group `group`. */
+mafat_status mafat_tile_region(const mafat_plan_t* plan, int32_t group, int32_t ti, int32_t tj,
+                               int32_t layer, int32_t in_rect[4], int32_t out_rect[4]);
+
+/* Same traversal without a plan: tile (ti, tj) of an n x m grid over the
+ * output of layers first..last. */
+mafat_status mafat_net_tile_region(const mafat_net_t* net, int32_t first, int32_t last,
+                                   int32_t n, int32_t m, int32_t ti, int32_t tj, int32_t layer,
+                                   int32_t in_rect[4], int32_t out_rect[4]);
+
+/* Algorithm 1 for one layer group (layers first..last, n x m tiles): the
+ * maximum over tiles and layers of scratch + output + input_factor*input
+ * elements (scratch = w_out*h_out*c_in*F^2/S), times 4 bytes, in MiB, plus
+ * bias_mib (the paper uses input_factor 2 and a 31 MB bias). */
+mafat_status mafat_predict_layer_group(const mafat_net_t* net, int32_t first, int32_t last,
+                                       int32_t n, int32_t m, double bias_mib,
+                                       int32_t input_factor, double* out_mib);
+
+/* predictMem of Algorithm 2: the maximum of Algorithm 1 over the groups of a
+ * configuration (cut, n1 x m1 top tiling, n2 x m2 bottom tiling), MiB. */
+mafat_status mafat_predict_mem(const mafat_net_t* net, int32_t cut, int32_t n1, int32_t m1,
+                               int32_t n2, int32_t m2, double bias_mib, double* out_mib);
+
+/* Algorithm 2: search cut in {n (no cut), 12, 8} x square top tilings 1..5
+ * with a 2x2 bottom tiling, returning the first configuration predicted
+ * strictly below limit_mib, else 5x5 / cut 8 / 2x2.  *cut == n means no cut. */
+mafat_status mafat_search(const mafat_net_t* net, double limit_mib, double bias_mib,
+                          int32_t* top_tile, int32_t* cut, int32_t* bottom_tile);
+
+/* Plan statistics (struct_size must be set by the caller). */
+mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out);
+
+/* Number of kernel launches one mafat_run makes. */
+int32_t mafat_launches_per_run(const mafat_plan_t* plan);
+
+void mafat_plan_destroy(mafat_plan_t* plan);
+void mafat_net_destroy(mafat_net_t* net);
+
+/* Message of the last failure on the calling thread ("" if none). */
+const char* mafat_last_error(void);
+
+/* Library version string. */
+const char* mafat_version(void);
+
+/* Diagnostic with no counterpart in the paper: one 128 x n x 16 bf16 tensor-core
+ * product D = A * B^T on one CTA, to check the operand and accumulator layouts
+ * the kernels use.  a_dev [128][16], b_dev [n][16] (bf16, row-major, device),
+ * d_dev [128][n] fp32 (device); n in {16, 32, ..., 256}.  lbo_is_k selects which
+ * descriptor offset field carries the K-direction stride.  Synchronous. */
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n,
+                             int32_t lbo_is_k, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MAFAT_H */

@@ -1,0 +1,97 @@
+// Plan tables shared by the host planner and the persistent kernels.
+//
+// A plan is lowered to three flat tables that live in device memory:
+//   * MafatStageDev  -- one per fused convolution stage of the network (a conv
+//                       layer, with the 2x2/s2 max-pool that follows it folded
+//                       into its epilogue), with packed-weight offsets;
+//   * MafatTaskDev   -- one per (frame, tile, stage): which buffer the stage
+//                       reads, which rectangle of the conv output it computes
+//                       (the tile's region from the Grid back-traversal,
+//                       Sec. 4.1) and where the result goes;
+//   * MafatItemDev   -- the work list in hand-out order: one item is a
+//                       16 x 8 block of conv output pixels x one block of
+//                       output channels of a task, with up to two completion
+//                       counters it must wait for.
+//
+// Activations are stored in "octet-planar" layout [C/8][H][W][8]: 8 channels of
+// one pixel are 16 bytes (bf16) or 32 bytes (fp32) and consecutive pixels of a
+// row are adjacent, so 8 pixels x 8 channels form one contiguous 128-byte
+// tensor-core core matrix at any pixel offset.
+#pragma once
+#include <stdint.h>
+
+#define MAFAT_BLK_ROWS 16   // conv output rows of one M block
+#define MAFAT_BLK_COLS 8    // conv output columns of one M block (M = 128)
+#define MAFAT_MAX_NBLK 256  // output channels of one item (MMA N)
+#define MAFAT_A_STAGE_BYTES 23552  // shared-memory A halo stage of the tensor-core kernel
+#define MAFAT_B_STAGE_BYTES 32768  // shared-memory weight-blob stage of the tensor-core kernel
+
+enum { MAFAT_BUF_USER_IN = 0, MAFAT_BUF_CUT = 1, MAFAT_BUF_SCRATCH = 2, MAFAT_BUF_USER_OUT = 3 };
+
+struct MafatStageDev {
+    int32_t layer;        // network layer index of the conv
+    int32_t k, pad;       // 3/1 or 1/0
+    int32_t cin, cin8;    // input channels and octets (cin8 = ceil(cin/8))
+    int32_t cout;         // output channels
+    int32_t pool;         // 1: a 2x2/s2 max-pool follows and is fused
+    // tensor-core packing
+    int32_t n_blk;        // output channels per item (MMA N)
+    int32_t n_nblk;       // cout / n_blk
+    int32_t chunk8;       // input octets per A chunk (8 = 64 channels, or cin8 if smaller)
+    int32_t n_chunks;     // cin8 / chunk8
+    int32_t paired;       // 1: cin8 == 1, two taps share one K=16 step
+    int32_t n_bsteps;     // weight blobs per chunk (taps, or tap pairs)
+    int32_t kst;          // K=16 MMA steps per blob
+    int32_t rows_box, cols_box;  // A halo box (pixels)
+    int64_t w_off;        // element offset of this stage's packed bf16 weights
+    int32_t blob_elems;   // elements of one blob (n_blk * 16 * kst)
+    int32_t sb_off;       // offset into the scale / bias arrays
+    int64_t w32_off;      // element offset of the fp32 weights [cout][cin][k][k]
+};
+
+struct MafatTaskDev {
+    int32_t stage;        // index into the stage table
+    int32_t frame;
+    // input buffer
+    int32_t in_kind;      // MAFAT_BUF_*
+    int32_t in_tmap;      // tensor map index (-1: the user-input map passed to the kernel)
+    int64_t in_off;       // element offset from the buffer base (frame included)
+    int32_t in_h, in_w;   // buffer extent (pixels)
+    int32_t in_y0, in_x0; // map position of buffer pixel (0, 0)
+    // conv output rectangle computed by this task (map coordinates, before pooling)
+    int32_t cy0, cx0, ch, cw;
+    int32_t nby, nbx;     // M blocks along rows / columns
+    // output buffer
+    int32_t out_kind;     // MAFAT_BUF_*
+    int32_t out_nhwc;     // 1: NHWC (user output), 0: octet-planar
+    int64_t out_off;      // element offset (frame included)
+    int32_t out_h, out_w; // buffer extent (pixels, after pooling)
+    int32_t out_y0, out_x0; // map position of buffer pixel (0, 0) (pooled map)
+    int32_t done_ctr;     // counter bumped once per finished item
+    int32_t n_items;
+};
+
+struct MafatItemDev {
+    int32_t task;
+    int16_t by, bx;       // M block
+    int16_t nb;           // output-channel block
+    int16_t flags;        // bit 0: do not publish completion (test hook)
+    int32_t dep0, dep0_target;  // counter index (-1: none) and value to wait for
+    int32_t dep1, dep1_target;
+    int32_t extra_ctr;    // second counter bumped on completion (-1: none)
+};
+
+// Counter block layout (uint32 words).  Zeroed when the plan is created; the
+// last CTA to leave a run sets every word except the status back to zero, so
+// a run is exactly one kernel launch.
+//   [0] ticket, [1] status, [2] abort, [3] CTAs finished, [4 ...] task / frame counters
+#define MAFAT_CTR_TICKET 0
+#define MAFAT_CTR_STATUS 1
+#define MAFAT_CTR_ABORT 2
+#define MAFAT_CTR_EXIT 3
+#define MAFAT_CTR_BASE 4
+
+// Device status codes (written with atomicCAS from 0).
+#define MAFAT_DEV_OK 0u
+#define MAFAT_DEV_TIMEOUT 1u
+#define MAFAT_DEV_PIPE 2u

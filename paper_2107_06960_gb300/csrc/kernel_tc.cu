@@ -1,0 +1,574 @@
+// bf16 tensor-core kernel for fused-tile execution of CNN layer groups
+// (MAFAT, Sec. 3-4) on sm_103a: tcgen05 MMA with TMEM accumulators, operands
+// staged in shared memory by TMA, one persistent launch per plan.
+//
+// One work item = one 16 x 8 block of a tile's conv output (M = 128 pixels)
+// times one block of n_blk <= 256 output channels, i.e. an implicit GEMM
+//   D[m][n] = sum_{c, ky, kx} A[pixel m shifted by (ky, kx)][c] * W[n][c][ky][kx]
+// (M = 128, N = n_blk, K = k*k*Cin) accumulated in fp32 in tensor memory.
+//
+// Operand layouts (no-swizzle, K-major canonical layout of the tcgen05 shared
+// memory descriptor: 8-row x 16-byte core matrices, LBO = stride between the
+// two core matrices along K, SBO = stride between 8-row groups along M/N):
+//  * A: one TMA box per chunk of <= 64 input channels holds the block's input
+//    halo, (16 + k - 1) x (8 + k - 1) pixels, as [octet][row][col][8 ch].  Eight
+//    consecutive pixels of a row x 8 channels are one 128-byte core matrix at any
+//    pixel offset, so the A operand of tap (ky, kx) is the same buffer at byte
+//    offset (ky * cols + kx) * 16: the halo is loaded once and reused for all
+//    taps, with no im2col copy.  SBO = one halo row, LBO = one octet plane.
+//    With 8 input channels (the first layer), one K=16 step covers two taps:
+//    its two K core matrices sit at the two taps' offsets (LBO = their
+//    distance).
+//  * B: weights pre-packed on the host in exactly the shared-memory image of
+//    one (chunk, tap) blob, fetched with one bulk copy.
+//
+// Warp roles (192 threads): warps 0-3 epilogue (warp w reads TMEM lanes
+// 32w..32w+31 = conv rows 4w..4w+3 of the block), warp 4 scheduler + TMA
+// producer, warp 5 TMEM allocator + MMA issuer.  Rings: 2 A stages, 5 B stages,
+// 2 TMEM accumulators of 256 columns (the epilogue of one item overlaps the
+// MMAs of the next), and a 4-deep queue of item indices.
+//
+// Epilogue: y = leaky_0.1(scale[n] * acc + bias[n]); for a fused 2x2/s2
+// max-pool the quad of pixels {(r, c), (r, c+1), (r+1, c), (r+1, c+1)} are lanes
+// {l, l^1, l^8, l^8^1} of one warp and are reduced with two shuffles; rounded
+// to bf16 (nearest-even) and stored to the tile's region buffer (octet-planar),
+// the cut tensor, or the NHWC output.
+#include <cuda_bf16.h>
+
+#include "sched.cuh"
+
+#ifndef MAFAT_NOSWZ_LBO_IS_K
+#define MAFAT_NOSWZ_LBO_IS_K 1
+#endif
+
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kAStages = 2;
+constexpr int kBStages = 5;
+constexpr int kQDepth = 4;
+constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;  // >= 8 octets x 18 x 10 pixels x 16 B, multiple of 1024
+constexpr int kBStageBytes = MAFAT_B_STAGE_BYTES;  // 256 rows x 64 channels x 2 B
+constexpr int kTmemCols = 512;        // two accumulators of up to 256 fp32 columns
+constexpr int kAccStride = 256;
+
+// shared-memory map (offsets from a 1024-aligned base)
+constexpr int kBarAFull = 0;
+constexpr int kBarAEmpty = kBarAFull + kAStages;
+constexpr int kBarBFull = kBarAEmpty + kAStages;
+constexpr int kBarBEmpty = kBarBFull + kBStages;
+constexpr int kBarAccFull = kBarBEmpty + kBStages;
+constexpr int kBarAccEmpty = kBarAccFull + 2;
+constexpr int kBarQFull = kBarAccEmpty + 2;
+constexpr int kBarQEmpty = kBarQFull + kQDepth;
+constexpr int kBarDone = kBarQEmpty + kQDepth;
+constexpr int kNumBars = kBarDone + 1;
+constexpr int kOffQItems = 512;
+constexpr int kOffTmem = kOffQItems + 4 * kQDepth;
+constexpr int kOffBroken = kOffTmem + 4;
+constexpr int kOffA = 1024;
+constexpr int kOffB = kOffA + kAStages * kAStageBytes;
+constexpr int kSmemUsed = kOffB + kBStages * kBStageBytes;
+constexpr int kSmemBytes = kSmemUsed + 1024;  // slack for aligning the base
+static_assert(kNumBars * 8 <= kOffQItems, "barrier area");
+static_assert(kSmemBytes <= 232448, "shared memory");
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+// Bounded wait on a pipeline barrier phase.  These waits depend only on work
+// inside the CTA, so they always finish unless something is broken; as a safety
+// net the first one to run out records MAFAT_DEV_PIPE and marks the CTA broken,
+// after which every pipeline wait of the CTA gives up after 1 ms, so the launch
+// still ends in bounded time (with garbage results and an error status).
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, uint32_t* ctr, int64_t limit_ns,
+                                          volatile int* broken) {
+    if (mbar_try_wait(bar, parity)) return;
+    const int64_t lim = *broken ? 1000000LL : limit_ns;
+    uint64_t t0 = mafat_dev::globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return;
+        if ((i & 255u) == 0u && (int64_t)(mafat_dev::globaltimer_ns() - t0) > lim) {
+            mafat_dev::record_status(ctr, MAFAT_DEV_PIPE);
+            *broken = 1;
+            return;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+// Shared-memory matrix descriptor, no swizzle: start >> 4 in bits 0-13, LBO >> 4
+// in 16-29, SBO >> 4 in 32-45, descriptor version 1 in bits 46-47, layout 0.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t k_stride, uint32_t mn_stride) {
+#if MAFAT_NOSWZ_LBO_IS_K
+    const uint32_t lbo = k_stride, sbo = mn_stride;
+#else
+    const uint32_t lbo = mn_stride, sbo = k_stride;
+#endif
+    uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;
+    d |= (uint64_t)((sbo & 0x3FFFFu) >> 4) << 32;
+    d |= (uint64_t)1 << 46;
+    return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A and
+// B (bits 7-9 = 1, 10-12 = 1), both K-major, N >> 3 in bits 17-22, M >> 4 in 24-28.
+__device__ __forceinline__ uint32_t instr_desc_bf16(int n, int m) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Byte offset of tap t inside an A halo buffer.
+__device__ __forceinline__ uint32_t tap_off(int t, int k, int cols) {
+    return (uint32_t)(((t / k) * cols + (t % k)) * 16);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    mafat_tc_kernel(const __grid_constant__ MafatKParams p, const __grid_constant__ CUtensorMap in_map) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t sbase = smem_u32(smem);
+    volatile int* q_items = reinterpret_cast<volatile int*>(smem + kOffQItems);
+    volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + kOffTmem);
+    volatile int* broken = reinterpret_cast<volatile int*>(smem + kOffBroken);
+    auto bar = [&](int i) { return sbase + (uint32_t)(i * 8); };
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t pipe_limit = 4 * p.timeout_ns + 1000000000LL;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kAStages; ++i) {
+            mbar_init(bar(kBarAFull + i), 1);
+            mbar_init(bar(kBarAEmpty + i), 1);
+        }
+        for (int i = 0; i < kBStages; ++i) {
+            mbar_init(bar(kBarBFull + i), 1);
+            mbar_init(bar(kBarBEmpty + i), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(kBarAccFull + i), 1);
+            mbar_init(bar(kBarAccEmpty + i), 128);
+        }
+        for (int i = 0; i < kQDepth; ++i) {
+            mbar_init(bar(kBarQFull + i), 1);
+            mbar_init(bar(kBarQEmpty + i), 5);
+        }
+        mbar_init(bar(kBarDone), 1);
+        *broken = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == kMmaWarp) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         sbase + (uint32_t)kOffTmem),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------ scheduler + TMA producer
+        if (lane == 0) {
+            uint32_t a_cnt = 0, b_cnt = 0, q_cnt = 0;
+            while (true) {
+                int ticket = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                if (ticket >= p.n_items) ticket = -1;
+                const int qs = (int)(q_cnt % kQDepth);
+                mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                q_items[qs] = ticket;
+                mbar_arrive(bar(kBarQFull + qs));
+                ++q_cnt;
+                if (ticket < 0) break;
+                const MafatItemDev it = p.items[ticket];
+                const MafatTaskDev tk = p.tasks[it.task];
+                const MafatStageDev st = p.stages[tk.stage];
+                const CUtensorMap* map = tk.in_kind == MAFAT_BUF_USER_IN ? &in_map
+                                         : tk.in_kind == MAFAT_BUF_CUT   ? p.tmaps + p.cut_tmap
+                                                                         : p.tmaps + tk.in_tmap;
+                const int c3 = tk.in_kind == MAFAT_BUF_SCRATCH ? 0 : tk.frame;
+                const int x0 = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * 8;
+                const int y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS - st.pad - tk.in_y0;
+                const uint32_t a_bytes = (uint32_t)(st.chunk8 * st.rows_box * st.cols_box * 16);
+                const uint32_t b_bytes = (uint32_t)(st.blob_elems * 2);
+                const uint16_t* wblob = p.w_bf16 + st.w_off +
+                                        (size_t)it.nb * st.n_chunks * st.n_bsteps * st.blob_elems;
+                mafat_dev::wait_item_deps(p.ctr, it, p.timeout_ns);
+                for (int c = 0; c < st.n_chunks; ++c) {
+                    const int as = (int)(a_cnt % kAStages);
+                    mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                    mbar_arrive_expect_tx(bar(kBarAFull + as), a_bytes);
+                    tma_load_4d(sbase + kOffA + as * kAStageBytes, map, x0, y0, c * st.chunk8, c3,
+                                bar(kBarAFull + as));
+                    ++a_cnt;
+                    for (int t = 0; t < st.n_bsteps; ++t) {
+                        const int bs = (int)(b_cnt % kBStages);
+                        mbar_wait(bar(kBarBEmpty + bs), ((b_cnt / kBStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                        mbar_arrive_expect_tx(bar(kBarBFull + bs), b_bytes);
+                        bulk_load(sbase + kOffB + bs * kBStageBytes,
+                                  wblob + ((size_t)c * st.n_bsteps + t) * st.blob_elems, b_bytes,
+                                  bar(kBarBFull + bs));
+                        ++b_cnt;
+                    }
+                }
+            }
+            // Drain: every copy issued into a stage has landed before the CTA may exit.
+            for (uint32_t i = 0; i < kAStages && i < a_cnt; ++i) {
+                uint32_t n = a_cnt - 1 - i;
+                mbar_wait(bar(kBarAFull + (int)(n % kAStages)), (n / kAStages) & 1u, p.ctr, pipe_limit, broken);
+            }
+            for (uint32_t i = 0; i < kBStages && i < b_cnt; ++i) {
+                uint32_t n = b_cnt - 1 - i;
+                mbar_wait(bar(kBarBFull + (int)(n % kBStages)), (n / kBStages) & 1u, p.ctr, pipe_limit, broken);
+            }
+        }
+        __syncwarp();
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            uint32_t a_cnt = 0, b_cnt = 0, q_cnt = 0, acc_cnt = 0;
+            bool issued = false;
+            while (true) {
+                const int qs = (int)(q_cnt % kQDepth);
+                mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
+                const int ticket = q_items[qs];
+                mbar_arrive(bar(kBarQEmpty + qs));
+                ++q_cnt;
+                if (ticket < 0) break;
+                const MafatItemDev it = p.items[ticket];
+                const MafatTaskDev tk = p.tasks[it.task];
+                const MafatStageDev st = p.stages[tk.stage];
+                const int buf = (int)(acc_cnt & 1u);
+                mbar_wait(bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kAccStride);
+                const uint32_t idesc = instr_desc_bf16(st.n_blk, 128);
+                const uint32_t a_plane = (uint32_t)(st.rows_box * st.cols_box * 16);
+                const uint32_t a_row = (uint32_t)(st.cols_box * 16);
+                const uint32_t b_half = (uint32_t)(st.n_blk * 16);
+                const int taps = st.k * st.k;
+                uint32_t accumulate = 0;
+                for (int c = 0; c < st.n_chunks; ++c) {
+                    const int as = (int)(a_cnt % kAStages);
+                    mbar_wait(bar(kBarAFull + as), (a_cnt / kAStages) & 1u, p.ctr, pipe_limit, broken);
+                    tc_fence_after();
+                    const uint32_t a_base = sbase + kOffA + as * kAStageBytes;
+                    for (int t = 0; t < st.n_bsteps; ++t) {
+                        const int bs = (int)(b_cnt % kBStages);
+                        mbar_wait(bar(kBarBFull + bs), (b_cnt / kBStages) & 1u, p.ctr, pipe_limit, broken);
+                        tc_fence_after();
+                        const uint32_t b_base = sbase + kOffB + bs * kBStageBytes;
+                        for (int j = 0; j < st.kst; ++j) {
+                            uint32_t a_addr, a_k;
+                            if (st.paired) {
+                                int ta = 2 * t, tb = 2 * t + 1;
+                                if (tb >= taps) {
+                                    ta = taps - 2;
+                                    tb = taps - 1;
+                                }
+                                const uint32_t oa = tap_off(ta, st.k, st.cols_box);
+                                a_addr = a_base + oa;
+                                a_k = tap_off(tb, st.k, st.cols_box) - oa;
+                            } else {
+                                a_addr = a_base + (uint32_t)(2 * j) * a_plane + tap_off(t, st.k, st.cols_box);
+                                a_k = a_plane;
+                            }
+                            const uint64_t adesc = smem_desc(a_addr, a_k, a_row);
+                            const uint64_t bdesc = smem_desc(b_base + (uint32_t)j * 2u * b_half, b_half, 128u);
+                            mma_bf16(d_tmem, adesc, bdesc, idesc, accumulate);
+                            accumulate = 1;
+                            issued = true;
+                        }
+                        tc_commit(bar(kBarBEmpty + bs));
+                        ++b_cnt;
+                    }
+                    tc_commit(bar(kBarAEmpty + as));
+                    ++a_cnt;
+                }
+                tc_commit(bar(kBarAccFull + buf));
+                ++acc_cnt;
+            }
+            // Every MMA this thread issued has completed before TMEM is released.
+            if (issued) {
+                tc_commit(bar(kBarDone));
+                mbar_wait(bar(kBarDone), 0u, p.ctr, pipe_limit, broken);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 0-3)
+        uint32_t q_cnt = 0, acc_cnt = 0;
+        const int r = warp * 4 + (lane >> 3);  // conv row within the block
+        const int cc = lane & 7;               // conv column within the block
+        while (true) {
+            const int qs = (int)(q_cnt % kQDepth);
+            mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
+            const int ticket = q_items[qs];
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
+            ++q_cnt;
+            if (ticket < 0) break;
+            const MafatItemDev it = p.items[ticket];
+            const MafatTaskDev tk = p.tasks[it.task];
+            const MafatStageDev st = p.stages[tk.stage];
+            const int buf = (int)(acc_cnt & 1u);
+            mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken);
+            __syncwarp();
+            tc_fence_after();
+
+            const int Y = tk.cy0 + it.by * MAFAT_BLK_ROWS + r;
+            const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
+            const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
+            bool store = valid;
+            int oy = Y, ox = X;
+            if (st.pool) {
+                store = valid && ((r & 1) == 0) && ((cc & 1) == 0);
+                oy = Y >> 1;
+                ox = X >> 1;
+            }
+            const int ly = oy - tk.out_y0, lx = ox - tk.out_x0;
+            __nv_bfloat16* out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
+                                                  : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
+                                                                                    : p.scratch) +
+                                 tk.out_off;
+            const float* sc = p.scale + st.sb_off + it.nb * st.n_blk;
+            const float* bi = p.bias + st.sb_off + it.nb * st.n_blk;
+            const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * kAccStride);
+            for (int q = 0; q < st.n_blk / 16; ++q) {
+                uint32_t raw[16];
+                tmem_ld16(taddr + (uint32_t)(q * 16), raw);
+                float v[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    float z = __ldg(sc + q * 16 + i) * __uint_as_float(raw[i]) + __ldg(bi + q * 16 + i);
+                    v[i] = z > 0.f ? z : 0.1f * z;
+                }
+                if (st.pool) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 1));
+                        v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 8));
+                    }
+                }
+                if (store) {
+                    const int ch0 = it.nb * st.n_blk + q * 16;
+                    uint4 lo, hi;
+                    lo.x = pack_bf16x2(v[0], v[1]);
+                    lo.y = pack_bf16x2(v[2], v[3]);
+                    lo.z = pack_bf16x2(v[4], v[5]);
+                    lo.w = pack_bf16x2(v[6], v[7]);
+                    hi.x = pack_bf16x2(v[8], v[9]);
+                    hi.y = pack_bf16x2(v[10], v[11]);
+                    hi.z = pack_bf16x2(v[12], v[13]);
+                    hi.w = pack_bf16x2(v[14], v[15]);
+                    // channels past cout belong to the zero-padded MMA N and are not stored
+                    const bool st_lo = ch0 < st.cout, st_hi = ch0 + 8 < st.cout;
+                    if (tk.out_nhwc) {
+                        uint4* dst = reinterpret_cast<uint4*>(out + ((size_t)ly * tk.out_w + lx) * st.cout + ch0);
+                        if (st_lo) dst[0] = lo;
+                        if (st_hi) dst[1] = hi;
+                    } else {
+                        const size_t plane = (size_t)tk.out_h * tk.out_w * 8;
+                        __nv_bfloat16* d0 = out + ((size_t)(ch0 >> 3) * tk.out_h + ly) * tk.out_w * 8 + (size_t)lx * 8;
+                        if (st_lo) *reinterpret_cast<uint4*>(d0) = lo;
+                        if (st_hi) *reinterpret_cast<uint4*>(d0 + plane) = hi;
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(bar(kBarAccEmpty + buf));
+            ++acc_cnt;
+            mafat_dev::fence_proxy_async_global();
+            __threadfence();
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            if (threadIdx.x == 0) mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == kMmaWarp) {
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
+                     : "memory");
+    }
+    mafat_dev::finish_cta(p.ctr, p.n_ctr);
+}
+
+// ---------------------------------------------------------------------------
+// Diagnostic: one 128 x n x 16 MMA.  Operands are written to shared memory in
+// an interleaved core-matrix order [8-row group][K half][8 rows][8 k] (K stride
+// 128 B, M/N stride 256 B), chosen so that both assignments of the two
+// descriptor offset fields stay inside the operand buffers.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(128, 1)
+    mafat_diag_umma_kernel(const __nv_bfloat16* a, const __nv_bfloat16* b, float* d, int n, int lbo_is_k) {
+    __shared__ __align__(1024) __nv_bfloat16 sa[128 * 16];
+    __shared__ __align__(1024) __nv_bfloat16 sb[256 * 16];
+    __shared__ __align__(8) uint64_t done_bar;
+    __shared__ uint32_t tmem_slot;
+    const int tid = threadIdx.x;
+    for (int idx = tid; idx < 128 * 16; idx += 128) {
+        int m = idx / 16, kk = idx % 16;
+        sa[((m / 8) * 2 + kk / 8) * 64 + (m % 8) * 8 + kk % 8] = a[idx];
+    }
+    for (int idx = tid; idx < n * 16; idx += 128) {
+        int m = idx / 16, kk = idx % 16;
+        sb[((m / 8) * 2 + kk / 8) * 64 + (m % 8) * 8 + kk % 8] = b[idx];
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (tid == 0) {
+        mbar_init(smem_u32(&done_bar), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if ((tid >> 5) == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                     "r"(256)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    if (tid == 0) {
+        uint64_t adesc, bdesc;
+        const uint32_t kst = 128, mst = 256;
+        auto mk = [&](uint32_t addr, uint32_t lbo, uint32_t sbo) {
+            uint64_t dd = (uint64_t)((addr & 0x3FFFFu) >> 4);
+            dd |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;
+            dd |= (uint64_t)((sbo & 0x3FFFFu) >> 4) << 32;
+            dd |= (uint64_t)1 << 46;
+            return dd;
+        };
+        if (lbo_is_k) {
+            adesc = mk(smem_u32(sa), kst, mst);
+            bdesc = mk(smem_u32(sb), kst, mst);
+        } else {
+            adesc = mk(smem_u32(sa), mst, kst);
+            bdesc = mk(smem_u32(sb), mst, kst);
+        }
+        mma_bf16(tmem, adesc, bdesc, instr_desc_bf16(n, 128), 0u);
+        tc_commit(smem_u32(&done_bar));
+    }
+    __syncwarp();
+    // bounded wait (1 s) for the product
+    {
+        uint64_t t0 = mafat_dev::globaltimer_ns();
+        while (!mbar_try_wait(smem_u32(&done_bar), 0u)) {
+            if ((int64_t)(mafat_dev::globaltimer_ns() - t0) > 1000000000LL) break;
+        }
+    }
+    __syncwarp();
+    tc_fence_after();
+    const int warp = tid >> 5;
+    for (int q = 0; q < n / 16; ++q) {
+        uint32_t raw[16];
+        tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)(q * 16), raw);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) d[(size_t)tid * n + q * 16 + i] = __uint_as_float(raw[i]);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) {
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256) : "memory");
+    }
+}
+
+}  // namespace
+
+size_t mafat_tc_smem_bytes() { return (size_t)kSmemBytes; }
+
+cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(mafat_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    mafat_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
+    return cudaGetLastError();
+}
+
+cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int lbo_is_k, cudaStream_t s) {
+    mafat_diag_umma_kernel<<<1, 128, 0, s>>>((const __nv_bfloat16*)a, (const __nv_bfloat16*)b, d, n, lbo_is_k);
+    return cudaGetLastError();
+}

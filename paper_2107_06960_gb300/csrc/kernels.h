@@ -1,0 +1,39 @@
+// Launch interface of the persistent fused-tile kernels (host and device visible).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "device_types.h"
+
+struct MafatKParams {
+    const MafatStageDev* stages;
+    const MafatTaskDev* tasks;
+    const MafatItemDev* items;
+    int32_t n_items;
+    int32_t pad0;
+    const CUtensorMap* tmaps;     // scratch-input and cut tensor maps (bf16 path)
+    int32_t cut_tmap;             // index of the cut tensor map (-1: none)
+    int32_t pad1;
+    const uint16_t* w_bf16;       // packed tensor-core weights
+    const float* w_f32;           // fp32 weights [cout][cin][k][k] per stage
+    const float* scale;
+    const float* bias;
+    const void* user_in;
+    void* user_out;
+    void* cut;
+    void* scratch;
+    uint32_t* ctr;                // counter block (ticket, status, abort, exit, task / frame counters)
+    int32_t n_ctr;                // words of the counter block
+    int32_t pad2;
+    int64_t timeout_ns;
+};
+
+// bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.
+cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, cudaStream_t s);
+size_t mafat_tc_smem_bytes();
+// fp32 CUDA-core check kernel: same work list, same scheduler.
+cudaError_t mafat_launch_fp32(const MafatKParams& p, int grid, cudaStream_t s);
+// Diagnostic single-MMA kernel.
+cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int lbo_is_k,
+                                   cudaStream_t s);

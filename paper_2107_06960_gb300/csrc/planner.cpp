@@ -1,0 +1,639 @@
+// Host-side planner of fused-tile execution (MAFAT, Sec. 4).  See planner.h.
+#include "planner.h"
+
+#include <algorithm>
+#include <cstring>
+#include <string>
+
+namespace mafat {
+
+static int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+std::string build_net(const int32_t* d, int n, int in_h, int in_w, int in_c, Net& net) {
+    if (n <= 0) return "network needs at least one layer";
+    if (in_h <= 0 || in_w <= 0 || in_c <= 0) return "input size must be positive";
+    net.layers.clear();
+    net.in_h = in_h;
+    net.in_w = in_w;
+    net.in_c = in_c;
+    int h = in_h, w = in_w, c = in_c;
+    for (int l = 0; l < n; ++l) {
+        Layer L{};
+        L.type = d[5 * l + 0];
+        L.k = d[5 * l + 1];
+        L.stride = d[5 * l + 2];
+        L.pad = d[5 * l + 3];
+        L.filters = d[5 * l + 4];
+        L.h_in = h;
+        L.w_in = w;
+        L.c_in = c;
+        if (L.type == L_CONV) {
+            if (!((L.k == 3 && L.pad == 1) || (L.k == 1 && L.pad == 0)) || L.stride != 1)
+                return "layer " + std::to_string(l) + ": only 3x3/s1/p1 and 1x1/s1/p0 convolutions are supported";
+            if (L.filters <= 0 || L.filters % 8 != 0)
+                return "layer " + std::to_string(l) + ": output channels must be a positive multiple of 8";
+            if (L.k == 1 && c <= 8)
+                return "layer " + std::to_string(l) + ": a 1x1 convolution needs more than 8 input channels";
+            L.c_out = L.filters;
+        } else if (L.type == L_MAXPOOL) {
+            if (L.k != 2 || L.stride != 2 || L.pad != 0)
+                return "layer " + std::to_string(l) + ": only 2x2/s2 max-pool is supported";
+            if (h % 2 != 0 || w % 2 != 0)
+                return "layer " + std::to_string(l) + ": max-pool input must have even height and width";
+            L.c_out = c;
+        } else {
+            return "layer " + std::to_string(l) + ": unknown layer type";
+        }
+        L.h_out = (h + 2 * L.pad - L.k) / L.stride + 1;
+        L.w_out = (w + 2 * L.pad - L.k) / L.stride + 1;
+        if (L.h_out <= 0 || L.w_out <= 0) return "layer " + std::to_string(l) + ": empty output";
+        h = L.h_out;
+        w = L.w_out;
+        c = L.c_out;
+        net.layers.push_back(L);
+    }
+    net.w.assign(n, {});
+    net.scale.assign(n, {});
+    net.bias.assign(n, {});
+    net.has_w.assign(n, 0);
+    return "";
+}
+
+void back_interval(int a, int b, int k, int s, int p, int size_in, int* lo, int* hi) {
+    if (b <= a) {
+        *lo = 0;
+        *hi = 0;
+        return;
+    }
+    // The window of output a starts at a*s - p; that of output b-1 ends at (b-1)*s - p + k - 1.
+    *lo = std::max(a * s - p, 0);
+    *hi = std::min((b - 1) * s - p + k, size_in);
+}
+
+void tile_regions(const Net& net, int first, int last, int n, int m, int i, int j,
+                  std::vector<Rect>& out_rects, std::vector<Rect>& in_rects) {
+    const Layer& Ll = net.layers[last];
+    Rect r;
+    r.y0 = grid_bound(Ll.h_out, n, i);
+    r.y1 = grid_bound(Ll.h_out, n, i + 1);
+    r.x0 = grid_bound(Ll.w_out, m, j);
+    r.x1 = grid_bound(Ll.w_out, m, j + 1);
+    if ((int)out_rects.size() < (int)net.layers.size()) out_rects.resize(net.layers.size());
+    if ((int)in_rects.size() < (int)net.layers.size()) in_rects.resize(net.layers.size());
+    for (int l = last; l >= first; --l) {
+        const Layer& L = net.layers[l];
+        Rect in;
+        back_interval(r.y0, r.y1, L.k, L.stride, L.pad, L.h_in, &in.y0, &in.y1);
+        back_interval(r.x0, r.x1, L.k, L.stride, L.pad, L.w_in, &in.x0, &in.x1);
+        if (r.empty()) in = Rect{};
+        out_rects[l] = r;
+        in_rects[l] = in;
+        r = in;
+    }
+}
+
+double predict_layer_group(const Net& net, int first, int last, int n, int m, double bias_mib,
+                           int input_factor) {
+    double best = 0.0;
+    std::vector<Rect> outs, ins;
+    for (int i = 0; i < n; ++i)
+        for (int j = 0; j < m; ++j) {
+            tile_regions(net, first, last, n, m, i, j, outs, ins);
+            for (int l = first; l <= last; ++l) {
+                const Layer& L = net.layers[l];
+                double w_out = outs[l].w(), h_out = outs[l].h();
+                double w_in = ins[l].w(), h_in = ins[l].h();
+                double scratch = w_out * h_out * (double)L.c_in * (double)(L.k * L.k) / (double)L.stride;
+                double input = w_in * h_in * (double)L.c_in;
+                double output = w_out * h_out * (double)L.c_out;
+                double mem = scratch + output + input * (double)input_factor;
+                if (mem > best) best = mem;
+            }
+        }
+    return best * 4.0 / (double)(1 << 20) + bias_mib;
+}
+
+double predict_mem(const Net& net, int cut, int n1, int m1, int n2, int m2, double bias_mib) {
+    int n = (int)net.layers.size();
+    if (cut <= 0 || cut >= n) return predict_layer_group(net, 0, n - 1, n1, m1, bias_mib, 2);
+    double a = predict_layer_group(net, 0, cut - 1, n1, m1, bias_mib, 2);
+    double b = predict_layer_group(net, cut, n - 1, n2, m2, bias_mib, 2);
+    return std::max(a, b);
+}
+
+void search(const Net& net, double limit_mib, double bias_mib, int* top, int* cut, int* bottom) {
+    const int n = (int)net.layers.size();
+    const int cuts[3] = {n, 12, 8};
+    const int bottom_tile = 2;
+    int lg1 = 0, c = 0;
+    for (int ci = 0; ci < 3; ++ci) {
+        c = cuts[ci];
+        for (int tile = 1; tile <= 5; ++tile) {
+            lg1 = tile;
+            double p = predict_mem(net, c, tile, tile, bottom_tile, bottom_tile, bias_mib);
+            if (p < limit_mib) {
+                *top = lg1;
+                *cut = c;
+                *bottom = bottom_tile;
+                return;
+            }
+        }
+    }
+    *top = lg1;
+    *cut = c;
+    *bottom = bottom_tile;
+}
+
+uint16_t f32_to_bf16_rne(float f) {
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    if ((u & 0x7f800000u) == 0x7f800000u && (u & 0x007fffffu)) return (uint16_t)((u >> 16) | 0x40);  // quiet NaN
+    u += 0x7fffu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+namespace {
+
+struct TileInfo {
+    int i, j;
+    std::vector<Rect> outs, ins;
+};
+
+// Largest even divisor of x that is <= 8 (x even).
+int chunk_octets(int x) {
+    for (int d = 8; d >= 2; d -= 2)
+        if (x % d == 0) return d;
+    return 2;
+}
+
+int largest_nblk(int cout) {
+    for (int d = MAFAT_MAX_NBLK; d >= 16; d -= 16)
+        if (cout % d == 0) return d;
+    return 16;
+}
+
+}  // namespace
+
+std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, bool* unsupported) {
+    *unsupported = false;
+    const int n = (int)net.layers.size();
+    t = PlanTables{};
+    t.cfg = cfg;
+    if (cfg.n_groups != 1 && cfg.n_groups != 2) return "n_groups must be 1 or 2";
+    if (cfg.n_groups == 2 && (cfg.cut <= 0 || cfg.cut >= n)) return "cut must be in 1..n-1";
+    if (cfg.batch <= 0) return "batch must be positive";
+    if (cfg.dtype != 0 && cfg.dtype != 1) return "unknown dtype";
+    for (int g = 0; g < cfg.n_groups; ++g)
+        if (cfg.grid_n[g] <= 0 || cfg.grid_m[g] <= 0) return "grid sizes must be positive";
+    const int G = cfg.n_groups;
+    t.groups[0][0] = 0;
+    t.groups[0][1] = G == 2 ? cfg.cut - 1 : n - 1;
+    if (G == 2) {
+        t.groups[1][0] = cfg.cut;
+        t.groups[1][1] = n - 1;
+    }
+
+    // ---- fused stages: a conv, plus the max-pool that directly follows it in the same group
+    std::vector<int> stage_pool_layer;
+    for (int g = 0; g < G; ++g) {
+        int first = t.groups[g][0], last = t.groups[g][1];
+        t.stage_first[g] = (int)t.stages.size();
+        for (int l = first; l <= last; ++l) {
+            const Layer& L = net.layers[l];
+            if (L.type == L_MAXPOOL) {
+                *unsupported = true;
+                return "layer " + std::to_string(l) + ": a max-pool must directly follow a convolution of its group";
+            }
+            if (!net.has_w[l]) return "layer " + std::to_string(l) + ": weights not set";
+            MafatStageDev s{};
+            s.layer = l;
+            s.k = L.k;
+            s.pad = L.pad;
+            s.cin = L.c_in;
+            s.cin8 = ceil_div(L.c_in, 8);
+            s.cout = L.c_out;
+            s.pool = (l + 1 <= last && net.layers[l + 1].type == L_MAXPOOL) ? 1 : 0;
+            // the MMA N must be a multiple of 16: pad with zero weights, store only cout channels
+            const int cout_pad = (L.c_out + 15) / 16 * 16;
+            s.n_blk = largest_nblk(cout_pad);
+            s.n_nblk = cout_pad / s.n_blk;
+            if (s.cin8 == 1) {
+                s.paired = 1;
+                s.chunk8 = 1;
+                s.n_chunks = 1;
+                s.n_bsteps = ceil_div(L.k * L.k, 2);
+                s.kst = 1;
+            } else {
+                if (s.cin8 % 2 != 0) {
+                    *unsupported = true;
+                    return "layer " + std::to_string(l) + ": input channels above 8 must be a multiple of 16";
+                }
+                s.paired = 0;
+                s.chunk8 = chunk_octets(s.cin8);
+                s.n_chunks = s.cin8 / s.chunk8;
+                s.n_bsteps = L.k * L.k;
+                s.kst = s.chunk8 / 2;
+            }
+            s.rows_box = MAFAT_BLK_ROWS + L.k - 1;
+            s.cols_box = MAFAT_BLK_COLS + L.k - 1;
+            s.blob_elems = s.n_blk * 16 * s.kst;
+            s.w_off = t.weight_elems;
+            t.weight_elems += (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems;
+            s.w32_off = t.weight32_elems;
+            t.weight32_elems += (int64_t)L.c_out * L.c_in * L.k * L.k;
+            s.sb_off = (int)t.sb_elems;
+            t.sb_elems += cout_pad;
+            t.stages.push_back(s);
+            stage_pool_layer.push_back(s.pool ? l + 1 : -1);
+            if (s.pool) ++l;
+        }
+        t.stage_last[g] = (int)t.stages.size() - 1;
+    }
+
+    // ---- geometry of the group inputs / outputs
+    const Layer& L0 = net.layers[0];
+    t.in_c8 = ceil_div(L0.c_in, 8);
+    const MafatStageDev& s_in = t.stages[t.stage_first[0]];
+    t.in_rows_box = s_in.rows_box;
+    t.in_cols_box = s_in.cols_box;
+    t.in_chunk8 = s_in.chunk8;
+    if (G == 2) {
+        const Layer& Lc = net.layers[t.groups[0][1]];
+        t.cut_h = Lc.h_out;
+        t.cut_w = Lc.w_out;
+        t.cut_c8 = ceil_div(Lc.c_out, 8);
+        const MafatStageDev& s2 = t.stages[t.stage_first[1]];
+        t.cut_rows_box = s2.rows_box;
+        t.cut_cols_box = s2.cols_box;
+        t.cut_chunk8 = s2.chunk8;
+    }
+    const Layer& Ln = net.layers[n - 1];
+    t.out_h = Ln.h_out;
+    t.out_w = Ln.w_out;
+    t.out_c = Ln.c_out;
+    const int64_t in_frame = (int64_t)t.in_c8 * 8 * L0.h_in * L0.w_in;
+    const int64_t cut_frame = (int64_t)t.cut_c8 * 8 * t.cut_h * t.cut_w;
+    const int64_t out_frame = (int64_t)t.out_h * t.out_w * t.out_c;
+
+    // ---- tiles of every group (non-empty only)
+    std::vector<std::vector<TileInfo>> tiles(G);
+    int max_tiles = 1;
+    for (int g = 0; g < G; ++g) {
+        for (int i = 0; i < cfg.grid_n[g]; ++i)
+            for (int j = 0; j < cfg.grid_m[g]; ++j) {
+                TileInfo ti;
+                ti.i = i;
+                ti.j = j;
+                tile_regions(net, t.groups[g][0], t.groups[g][1], cfg.grid_n[g], cfg.grid_m[g], i, j,
+                             ti.outs, ti.ins);
+                if (ti.outs[t.groups[g][1]].empty()) continue;
+                tiles[g].push_back(std::move(ti));
+            }
+        max_tiles = std::max(max_tiles, (int)tiles[g].size());
+    }
+    int S = cfg.ring_slots > 0 ? cfg.ring_slots : std::min(max_tiles, 64);
+    int W = cfg.wave_tiles > 0 ? std::min(cfg.wave_tiles, S) : S;
+    t.ring_slots = S;
+    t.wave_tiles = W;
+
+    // ---- scratch buffer size: largest non-final stage output of any tile
+    int64_t buf = 0;
+    for (int g = 0; g < G; ++g)
+        for (const TileInfo& ti : tiles[g])
+            for (int s = t.stage_first[g]; s < t.stage_last[g]; ++s) {
+                const MafatStageDev& st = t.stages[s];
+                int ol = stage_pool_layer[s] >= 0 ? stage_pool_layer[s] : st.layer;
+                const Rect& r = ti.outs[ol];
+                buf = std::max(buf, (int64_t)r.h() * r.w() * ceil_div(st.cout, 8) * 8);
+            }
+    t.slot_buf_elems = (buf + 127) / 128 * 128;  // 256-byte aligned for bf16, 512 for fp32
+
+    // ---- tasks in hand-out order, with their dependencies expressed as task indices
+    struct TaskDep {
+        int prev_task = -1;    // previous stage of the same tile, or the ring predecessor's last stage
+        int frame_g1 = -1;     // frame whose group 1 must be complete
+        bool last_g1 = false;  // last stage of group 1 (bumps the frame counter)
+    };
+    std::vector<TaskDep> deps;
+    std::vector<int> last_task_of_seq;
+    int seq = 0;
+    for (int f = 0; f < cfg.batch; ++f) {
+        for (int g = 0; g < G; ++g) {
+            const auto& tl = tiles[g];
+            for (size_t w0 = 0; w0 < tl.size(); w0 += W) {
+                size_t w1 = std::min(tl.size(), w0 + (size_t)W);
+                std::vector<int> prev_of_tile(w1 - w0, -1);
+                for (int s = t.stage_first[g]; s <= t.stage_last[g]; ++s) {
+                    const MafatStageDev& st = t.stages[s];
+                    const Layer& Lc = net.layers[st.layer];
+                    for (size_t q = w0; q < w1; ++q) {
+                        const TileInfo& ti = tl[q];
+                        int tseq = seq + (int)(q - w0);
+                        int slot = tseq % S;
+                        MafatTaskDev tk{};
+                        tk.stage = s;
+                        tk.frame = f;
+                        const Rect& cr = ti.outs[st.layer];
+                        const Rect& ir = ti.ins[st.layer];
+                        int ol = stage_pool_layer[s] >= 0 ? stage_pool_layer[s] : st.layer;
+                        const Rect& orr = ti.outs[ol];
+                        if (st.pool) {
+                            // the conv region of a pooled stage is exactly twice the pooled region
+                            if (!(cr.y0 == 2 * orr.y0 && cr.y1 == 2 * orr.y1 && cr.x0 == 2 * orr.x0 &&
+                                  cr.x1 == 2 * orr.x1))
+                                return "internal: pooled region mismatch";
+                        }
+                        tk.cy0 = cr.y0;
+                        tk.cx0 = cr.x0;
+                        tk.ch = cr.h();
+                        tk.cw = cr.w();
+                        tk.nby = ceil_div(tk.ch, MAFAT_BLK_ROWS);
+                        tk.nbx = ceil_div(tk.cw, MAFAT_BLK_COLS);
+                        int rel = s - t.stage_first[g];
+                        if (s == t.stage_first[g]) {
+                            tk.in_kind = g == 0 ? MAFAT_BUF_USER_IN : MAFAT_BUF_CUT;
+                            tk.in_tmap = -1;
+                            tk.in_off = g == 0 ? f * in_frame : f * cut_frame;
+                            tk.in_h = Lc.h_in;
+                            tk.in_w = Lc.w_in;
+                            tk.in_y0 = 0;
+                            tk.in_x0 = 0;
+                        } else {
+                            int b = (slot * 2) + ((rel - 1) & 1);
+                            tk.in_kind = MAFAT_BUF_SCRATCH;
+                            tk.in_off = (int64_t)b * t.slot_buf_elems;
+                            tk.in_h = ir.h();
+                            tk.in_w = ir.w();
+                            tk.in_y0 = ir.y0;
+                            tk.in_x0 = ir.x0;
+                            TmapReq req{};
+                            req.task = (int)t.tasks.size();
+                            req.slot = slot;
+                            req.buf = b;
+                            req.h = ir.h();
+                            req.w = ir.w();
+                            req.c8 = st.cin8;
+                            req.rows_box = st.rows_box;
+                            req.cols_box = st.cols_box;
+                            req.chunk8 = st.chunk8;
+                            tk.in_tmap = (int)t.tmaps.size();
+                            t.tmaps.push_back(req);
+                        }
+                        if (s == t.stage_last[g]) {
+                            if (g == G - 1) {
+                                tk.out_kind = MAFAT_BUF_USER_OUT;
+                                tk.out_nhwc = 1;
+                                tk.out_off = f * out_frame;
+                                tk.out_h = t.out_h;
+                                tk.out_w = t.out_w;
+                            } else {
+                                tk.out_kind = MAFAT_BUF_CUT;
+                                tk.out_nhwc = 0;
+                                tk.out_off = f * cut_frame;
+                                tk.out_h = t.cut_h;
+                                tk.out_w = t.cut_w;
+                            }
+                            tk.out_y0 = 0;
+                            tk.out_x0 = 0;
+                        } else {
+                            int b = (slot * 2) + (rel & 1);
+                            tk.out_kind = MAFAT_BUF_SCRATCH;
+                            tk.out_nhwc = 0;
+                            tk.out_off = (int64_t)b * t.slot_buf_elems;
+                            tk.out_h = orr.h();
+                            tk.out_w = orr.w();
+                            tk.out_y0 = orr.y0;
+                            tk.out_x0 = orr.x0;
+                        }
+                        tk.n_items = tk.nby * tk.nbx * st.n_nblk;
+                        TaskDep d;
+                        int qi = (int)(q - w0);
+                        if (s == t.stage_first[g]) {
+                            if (tseq >= S) d.prev_task = last_task_of_seq[tseq - S];
+                            if (g == 1) d.frame_g1 = f;
+                        } else {
+                            d.prev_task = prev_of_tile[qi];
+                        }
+                        d.last_g1 = (G == 2 && g == 0 && s == t.stage_last[g]);
+                        prev_of_tile[qi] = (int)t.tasks.size();
+                        t.tasks.push_back(tk);
+                        deps.push_back(d);
+                        // statistics
+                        double kk = (double)Lc.k * Lc.k;
+                        t.executed_flops += 2.0 * cr.h() * cr.w() * (double)st.cout * st.cin * kk;
+                        t.issued_flops += 2.0 * tk.nby * tk.nbx * (double)(MAFAT_BLK_ROWS * MAFAT_BLK_COLS) *
+                                          (double)st.n_nblk * st.n_blk * st.n_chunks * st.n_bsteps * st.kst * 16.0;
+                    }
+                }
+                for (size_t q = w0; q < w1; ++q) last_task_of_seq.push_back(prev_of_tile[q - w0]);
+                seq += (int)(w1 - w0);
+            }
+        }
+    }
+    t.n_tiles = seq;
+
+    // ---- counters: one per task, then one per frame (group-1 completion)
+    const int n_tasks = (int)t.tasks.size();
+    t.frame_ctr_base = MAFAT_CTR_BASE + n_tasks;
+    t.n_counters = n_tasks + cfg.batch;
+    std::vector<int> g1_items(cfg.batch, 0);
+    for (int ti = 0; ti < n_tasks; ++ti) {
+        t.tasks[ti].done_ctr = MAFAT_CTR_BASE + ti;
+        if (deps[ti].last_g1) g1_items[t.tasks[ti].frame] += t.tasks[ti].n_items;
+    }
+    // ---- items
+    for (int ti = 0; ti < n_tasks; ++ti) {
+        const MafatTaskDev& tk = t.tasks[ti];
+        const MafatStageDev& st = t.stages[tk.stage];
+        const TaskDep& d = deps[ti];
+        for (int by = 0; by < tk.nby; ++by)
+            for (int bx = 0; bx < tk.nbx; ++bx)
+                for (int nb = 0; nb < st.n_nblk; ++nb) {
+                    MafatItemDev it{};
+                    it.task = ti;
+                    it.by = (int16_t)by;
+                    it.bx = (int16_t)bx;
+                    it.nb = (int16_t)nb;
+                    it.flags = (ti == cfg.unpublished_task) ? 1 : 0;
+                    it.dep0 = -1;
+                    it.dep1 = -1;
+                    it.extra_ctr = -1;
+                    if (d.prev_task >= 0) {
+                        it.dep0 = MAFAT_CTR_BASE + d.prev_task;
+                        it.dep0_target = t.tasks[d.prev_task].n_items;
+                    }
+                    if (d.frame_g1 >= 0) {
+                        it.dep1 = t.frame_ctr_base + d.frame_g1;
+                        it.dep1_target = g1_items[d.frame_g1];
+                    }
+                    if (d.last_g1) it.extra_ctr = t.frame_ctr_base + tk.frame;
+                    t.items.push_back(it);
+                }
+    }
+    if (t.items.size() > (size_t)0x7fffffff) return "too many work items";
+
+    // ---- statistics
+    for (int l = 0; l < n; ++l) {
+        const Layer& L = net.layers[l];
+        if (L.type == L_CONV)
+            t.useful_flops += 2.0 * L.h_out * L.w_out * (double)L.c_out * L.c_in * L.k * L.k * cfg.batch;
+    }
+    int64_t io = in_frame + out_frame + (G == 2 ? 2 * cut_frame : 0);
+    t.group_io_elems = io * cfg.batch;
+    t.predicted_mib = predict_mem(net, G == 2 ? cfg.cut : 0, cfg.grid_n[0], cfg.grid_m[0],
+                                  G == 2 ? cfg.grid_n[1] : 1, G == 2 ? cfg.grid_m[1] : 1, 31.0);
+    return validate_plan(net, t);
+}
+
+std::string validate_plan(const Net& net, const PlanTables& t) {
+    const int n_tasks = (int)t.tasks.size();
+    const Layer& L0 = net.layers[0];
+    const int64_t in_total = (int64_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in;
+    const int64_t cut_total = (int64_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w;
+    const int64_t out_total = (int64_t)t.cfg.batch * t.out_h * t.out_w * t.out_c;
+    const int64_t scratch_total = (int64_t)t.ring_slots * 2 * t.slot_buf_elems;
+    auto buf_total = [&](int kind) {
+        return kind == MAFAT_BUF_USER_IN ? in_total
+               : kind == MAFAT_BUF_CUT   ? cut_total
+               : kind == MAFAT_BUF_USER_OUT ? out_total
+                                          : scratch_total;
+    };
+    for (const MafatStageDev& s : t.stages) {
+        if ((int64_t)s.chunk8 * s.rows_box * s.cols_box * 16 > MAFAT_A_STAGE_BYTES) return "A box exceeds its stage";
+        if ((int64_t)s.blob_elems * 2 > MAFAT_B_STAGE_BYTES) return "weight blob exceeds its stage";
+        if (s.cols_box * 8 > 256 || s.rows_box > 256 || s.chunk8 > 256) return "TMA box dimension above 256";
+        if ((s.cols_box * 16) % 16 != 0) return "TMA inner box not a multiple of 16 bytes";
+        if (s.n_blk % 16 != 0 || s.n_blk < 16 || s.n_blk > MAFAT_MAX_NBLK) return "bad MMA N";
+        if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
+            return "weight blobs outside the packed weights";
+        if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
+    }
+    std::vector<int> first_item(n_tasks, -1), last_item(n_tasks, -1);
+    for (size_t i = 0; i < t.items.size(); ++i) {
+        int tk = t.items[i].task;
+        if (tk < 0 || tk >= n_tasks) return "item with a bad task";
+        if (first_item[tk] < 0) first_item[tk] = (int)i;
+        last_item[tk] = (int)i;
+    }
+    for (int ti = 0; ti < n_tasks; ++ti) {
+        const MafatTaskDev& k = t.tasks[ti];
+        const MafatStageDev& s = t.stages[k.stage];
+        const Layer& L = net.layers[s.layer];
+        if (last_item[ti] - first_item[ti] + 1 != k.n_items) return "task items not contiguous";
+        // input buffer extent and coverage of every in-map tap of the conv rectangle
+        if (k.in_off < 0 || k.in_off + (int64_t)s.cin8 * 8 * k.in_h * k.in_w > buf_total(k.in_kind))
+            return "input buffer outside its allocation";
+        int ny0 = std::max(k.cy0 - s.pad, 0), ny1 = std::min(k.cy0 + k.ch - 1 - s.pad + s.k, L.h_in);
+        int nx0 = std::max(k.cx0 - s.pad, 0), nx1 = std::min(k.cx0 + k.cw - 1 - s.pad + s.k, L.w_in);
+        if (k.in_y0 > ny0 || k.in_y0 + k.in_h < ny1 || k.in_x0 > nx0 || k.in_x0 + k.in_w < nx1)
+            return "input region does not cover the conv rectangle's taps";
+        if (k.in_y0 + k.in_h > L.h_in || k.in_x0 + k.in_w > L.w_in || k.in_y0 < 0 || k.in_x0 < 0)
+            return "input region outside the map";
+        if (k.in_kind == MAFAT_BUF_SCRATCH && k.in_off % t.slot_buf_elems != 0) return "scratch input misaligned";
+        // output extent of the valid pixels
+        int oy0 = k.cy0, oy1 = k.cy0 + k.ch, ox0 = k.cx0, ox1 = k.cx0 + k.cw;
+        if (s.pool) {
+            if (k.cy0 % 2 || k.ch % 2 || k.cx0 % 2 || k.cw % 2) return "pooled rectangle not quad aligned";
+            oy0 /= 2; oy1 /= 2; ox0 /= 2; ox1 /= 2;
+        }
+        if (oy0 < k.out_y0 || ox0 < k.out_x0 || oy1 > k.out_y0 + k.out_h || ox1 > k.out_x0 + k.out_w)
+            return "output rectangle outside its buffer";
+        int64_t out_elems = k.out_nhwc ? (int64_t)k.out_h * k.out_w * s.cout
+                                       : (int64_t)((s.cout + 7) / 8) * 8 * k.out_h * k.out_w;
+        if (k.out_off < 0 || k.out_off + out_elems > buf_total(k.out_kind)) return "output buffer outside its allocation";
+        if (k.out_kind == MAFAT_BUF_SCRATCH && out_elems > t.slot_buf_elems) return "scratch output above buffer size";
+        if (k.done_ctr < MAFAT_CTR_BASE || k.done_ctr >= MAFAT_CTR_BASE + t.n_counters) return "bad done counter";
+    }
+    // dependencies: every counter an item waits on is fed only by items handed out before it
+    std::vector<int> frame_last(t.cfg.batch, -1);
+    for (size_t i = 0; i < t.items.size(); ++i) {
+        const MafatItemDev& it = t.items[i];
+        const MafatTaskDev& k = t.tasks[it.task];
+        const MafatStageDev& s = t.stages[k.stage];
+        if (it.by >= k.nby || it.bx >= k.nbx || it.nb >= s.n_nblk || it.by < 0 || it.bx < 0 || it.nb < 0)
+            return "item block out of range";
+        const int deps[2] = {it.dep0, it.dep1};
+        const int tgts[2] = {it.dep0_target, it.dep1_target};
+        for (int d = 0; d < 2; ++d) {
+            if (deps[d] < 0) continue;
+            if (deps[d] < MAFAT_CTR_BASE || deps[d] >= MAFAT_CTR_BASE + t.n_counters) return "bad dependency counter";
+            if (deps[d] < t.frame_ctr_base) {
+                int dt = deps[d] - MAFAT_CTR_BASE;
+                if (last_item[dt] >= (int)i) return "dependency on a later item";
+                if (tgts[d] != t.tasks[dt].n_items) return "dependency target mismatch";
+            } else {
+                int f = deps[d] - t.frame_ctr_base;
+                if (frame_last[f] < 0 || frame_last[f] >= (int)i) return "frame dependency on a later item";
+            }
+        }
+        if (it.extra_ctr >= 0) {
+            if (it.extra_ctr < t.frame_ctr_base || it.extra_ctr >= MAFAT_CTR_BASE + t.n_counters)
+                return "bad extra counter";
+            frame_last[it.extra_ctr - t.frame_ctr_base] = (int)i;
+        }
+    }
+    return "";
+}
+
+// Packed bf16 weight order, per stage: [n-block][chunk][blob][K step][K half][N/8][8 rows][8 k].
+// One K=16 step holds two 8 x 8 core-matrix columns (K halves) of the B operand; within a
+// half, the n_blk rows are groups of 8 rows x 16 bytes (one core matrix each).
+//  - regular stages: blob = tap (ky, kx), K half h of step j = input octet chunk*chunk8 + 2j + h;
+//  - paired stages (8 input channels): blob p holds taps (a, b) = (2p, 2p+1), or for an odd
+//    tap count the last blob holds (zero weights, last tap); K half 0 = tap a, half 1 = tap b.
+void pack_weights_bf16(const Net& net, const PlanTables& t, std::vector<uint16_t>& out) {
+    out.assign((size_t)t.weight_elems, 0);
+    for (const MafatStageDev& s : t.stages) {
+        const Layer& L = net.layers[s.layer];
+        const std::vector<float>& w = net.w[s.layer];
+        const int k = L.k, cin = L.c_in, taps = k * k;
+        for (int nb = 0; nb < s.n_nblk; ++nb)
+            for (int c = 0; c < s.n_chunks; ++c)
+                for (int b = 0; b < s.n_bsteps; ++b) {
+                    size_t blob = (size_t)s.w_off +
+                                  ((size_t)(nb * s.n_chunks + c) * s.n_bsteps + b) * (size_t)s.blob_elems;
+                    for (int j = 0; j < s.kst; ++j)
+                        for (int h = 0; h < 2; ++h)
+                            for (int nn = 0; nn < s.n_blk; ++nn)
+                                for (int e = 0; e < 8; ++e) {
+                                    int o = nb * s.n_blk + nn;
+                                    int ci, tap;
+                                    if (s.paired) {
+                                        int a = 2 * b, bb = 2 * b + 1;
+                                        if (bb >= taps) {
+                                            a = -1;  // zero weights paired with the last tap
+                                            bb = taps - 1;
+                                        }
+                                        tap = h == 0 ? a : bb;
+                                        ci = e;
+                                    } else {
+                                        tap = b;
+                                        ci = ((c * s.chunk8) + 2 * j + h) * 8 + e;
+                                    }
+                                    float v = 0.f;
+                                    if (tap >= 0 && ci < cin && o < L.c_out) {
+                                        int ky = tap / k, kx = tap % k;
+                                        v = w[(((size_t)o * cin + ci) * k + ky) * k + kx];
+                                    }
+                                    size_t idx = blob + (size_t)j * 2 * s.n_blk * 8 + (size_t)h * s.n_blk * 8 +
+                                                 (size_t)(nn / 8) * 64 + (size_t)(nn % 8) * 8 + e;
+                                    out[idx] = f32_to_bf16_rne(v);
+                                }
+                }
+    }
+}
+
+void pack_weights_fp32(const Net& net, const PlanTables& t, std::vector<float>& w32,
+                       std::vector<float>& scale, std::vector<float>& bias) {
+    w32.assign((size_t)t.weight32_elems, 0.f);
+    scale.assign((size_t)t.sb_elems, 0.f);
+    bias.assign((size_t)t.sb_elems, 0.f);
+    for (const MafatStageDev& s : t.stages) {
+        const std::vector<float>& w = net.w[s.layer];
+        std::copy(w.begin(), w.end(), w32.begin() + s.w32_off);
+        std::copy(net.scale[s.layer].begin(), net.scale[s.layer].end(), scale.begin() + s.sb_off);
+        std::copy(net.bias[s.layer].begin(), net.bias[s.layer].end(), bias.begin() + s.sb_off);
+    }
+}
+
+}  // namespace mafat

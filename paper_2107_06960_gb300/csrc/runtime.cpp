@@ -1,0 +1,535 @@
+// C ABI of the fused-tile runtime: network description, planning, device
+// workspace, weight packing, tensor maps and launches.  See include/mafat.h.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/mafat.h"
+#include "kernels.h"
+#include "planner.h"
+
+struct mafat_net_s {
+    mafat::Net net;
+};
+
+struct mafat_plan_s {
+    mafat::Net shapes;  // layers only (no weights)
+    mafat::PlanTables t;
+    int device = 0;
+    int dtype = 0;
+    int esz = 2;
+    bool dry_run = false;
+    int grid = 0;
+    int64_t timeout_ns = 2000000000LL;
+    std::vector<void*> allocs;
+    int64_t workspace_bytes = 0;
+    MafatStageDev* d_stages = nullptr;
+    MafatTaskDev* d_tasks = nullptr;
+    MafatItemDev* d_items = nullptr;
+    CUtensorMap* d_tmaps = nullptr;
+    void* d_w = nullptr;
+    float* d_scale = nullptr;
+    float* d_bias = nullptr;
+    void* d_cut = nullptr;
+    void* d_scratch = nullptr;
+    uint32_t* d_ctr = nullptr;
+    size_t ctr_bytes = 0;
+    int64_t weight_bytes = 0, scratch_bytes = 0;
+    size_t in_bytes = 0, out_bytes = 0, cut_bytes = 0;
+    // user-input tensor map, re-encoded when the input pointer changes
+    CUtensorMap in_map;
+    const void* in_map_ptr = nullptr;
+    // staging for mafat_run_host
+    void* d_in_stage = nullptr;
+    void* d_out_stage = nullptr;
+    std::mutex mu;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+mafat_status fail(mafat_status s, const std::string& msg) {
+    g_err = msg;
+    return s;
+}
+
+mafat_status cuda_fail(cudaError_t e, const char* what) {
+    g_err = std::string(what) + ": " + cudaGetErrorString(e);
+    return e == cudaErrorMemoryAllocation ? MAFAT_ENOMEM : MAFAT_ECUDA;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    });
+    return fn;
+}
+
+// 4-D tiled map over an octet-planar bf16 tensor [frames][c8][h][w][8]:
+// dim0 = w*8 elements (one row of pixels), dim1 = h, dim2 = c8, dim3 = frames.
+// Box = one A halo: cols_box pixels x rows_box rows x chunk8 octets x 1 frame.
+// Out-of-range elements read as zero (the convolution's zero padding).
+bool encode_planar_map(CUtensorMap* m, const void* base, int w, int h, int c8, int frames, int cols_box,
+                       int rows_box, int chunk8, std::string* err) {
+    auto fn = encode_fn();
+    if (!fn) {
+        *err = "cuTensorMapEncodeTiled unavailable";
+        return false;
+    }
+    cuuint64_t dims[4] = {(cuuint64_t)w * 8, (cuuint64_t)h, (cuuint64_t)c8, (cuuint64_t)frames};
+    cuuint64_t strides[3] = {(cuuint64_t)w * 16, (cuuint64_t)h * w * 16, (cuuint64_t)c8 * h * w * 16};
+    cuuint32_t box[4] = {(cuuint32_t)cols_box * 8, (cuuint32_t)rows_box, (cuuint32_t)chunk8, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+        return false;
+    }
+    return true;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+void free_plan_memory(mafat_plan_s* p) {
+    for (void* a : p->allocs) cudaFree(a);
+    p->allocs.clear();
+    if (p->d_in_stage) cudaFree(p->d_in_stage);
+    if (p->d_out_stage) cudaFree(p->d_out_stage);
+    p->d_in_stage = p->d_out_stage = nullptr;
+}
+
+template <class T>
+cudaError_t dalloc(mafat_plan_s* p, T** out, size_t bytes) {
+    void* d = nullptr;
+    if (bytes == 0) bytes = 256;
+    cudaError_t e = cudaMalloc(&d, bytes);
+    if (e != cudaSuccess) return e;
+    p->allocs.push_back(d);
+    p->workspace_bytes += (int64_t)bytes;
+    *out = (T*)d;
+    return cudaSuccess;
+}
+
+mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream_t s) {
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    if (!input || !output) return fail(MAFAT_EINVAL, "null input or output");
+    if (!aligned16(input) || !aligned16(output)) return fail(MAFAT_EINVAL, "input and output must be 16-byte aligned");
+    const char* ib = (const char*)input;
+    const char* ob = (const char*)output;
+    if (ib < ob + p->out_bytes && ob < ib + p->in_bytes) return fail(MAFAT_EINVAL, "input and output overlap");
+    cudaError_t e;
+    MafatKParams kp{};
+    kp.stages = p->d_stages;
+    kp.tasks = p->d_tasks;
+    kp.items = p->d_items;
+    kp.n_items = (int32_t)p->t.items.size();
+    kp.tmaps = p->d_tmaps;
+    kp.cut_tmap = p->t.cfg.n_groups == 2 ? (int)p->t.tmaps.size() : -1;
+    kp.w_bf16 = (const uint16_t*)p->d_w;
+    kp.w_f32 = (const float*)p->d_w;
+    kp.scale = p->d_scale;
+    kp.bias = p->d_bias;
+    kp.user_in = input;
+    kp.user_out = output;
+    kp.cut = p->d_cut;
+    kp.scratch = p->d_scratch;
+    kp.ctr = p->d_ctr;
+    kp.n_ctr = (int32_t)(p->ctr_bytes / sizeof(uint32_t));
+    kp.timeout_ns = p->timeout_ns;
+    if (p->dtype == MAFAT_BF16) {
+        if (p->in_map_ptr != input) {
+            std::string err;
+            const mafat::Layer& L0 = p->shapes.layers[0];
+            if (!encode_planar_map(&p->in_map, input, L0.w_in, L0.h_in, p->t.in_c8, p->t.cfg.batch,
+                                   p->t.in_cols_box, p->t.in_rows_box, p->t.in_chunk8, &err))
+                return fail(MAFAT_ECUDA, err);
+            p->in_map_ptr = input;
+        }
+        e = mafat_launch_tc(kp, p->in_map, p->grid, s);
+    } else {
+        e = mafat_launch_fp32(kp, p->grid, s);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+    return MAFAT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* mafat_last_error(void) { return g_err.c_str(); }
+
+const char* mafat_version(void) { return "mafat-gb300 0.1 (sm_103a tcgen05)"; }
+
+mafat_status mafat_describe_net(const mafat_layer_desc* layers, int32_t n, int32_t in_h, int32_t in_w, int32_t in_c,
+                                mafat_net_t** out) {
+    if (!layers || !out) return fail(MAFAT_EINVAL, "null argument");
+    *out = nullptr;
+    static_assert(sizeof(mafat_layer_desc) == 5 * sizeof(int32_t), "layer desc layout");
+    mafat_net_s* net = new (std::nothrow) mafat_net_s();
+    if (!net) return fail(MAFAT_ENOMEM, "host allocation failed");
+    std::string err = mafat::build_net((const int32_t*)layers, n, in_h, in_w, in_c, net->net);
+    if (!err.empty()) {
+        delete net;
+        bool unsup = err.find("only") != std::string::npos || err.find("multiple of") != std::string::npos ||
+                     err.find("even") != std::string::npos || err.find("needs more") != std::string::npos;
+        return fail(unsup ? MAFAT_EUNSUPPORTED : MAFAT_EINVAL, err);
+    }
+    *out = net;
+    g_err.clear();
+    return MAFAT_OK;
+}
+
+mafat_status mafat_net_shape(const mafat_net_t* net, int32_t layer, int32_t shape[6]) {
+    if (!net || !shape) return fail(MAFAT_EINVAL, "null argument");
+    if (layer < 0 || layer >= (int)net->net.layers.size()) return fail(MAFAT_EINVAL, "layer out of range");
+    const mafat::Layer& L = net->net.layers[layer];
+    shape[0] = L.h_in;
+    shape[1] = L.w_in;
+    shape[2] = L.c_in;
+    shape[3] = L.h_out;
+    shape[4] = L.w_out;
+    shape[5] = L.c_out;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_set_weights(mafat_net_t* net, int32_t layer, const float* w, const float* scale,
+                               const float* bias) {
+    if (!net || !w || !scale || !bias) return fail(MAFAT_EINVAL, "null argument");
+    if (layer < 0 || layer >= (int)net->net.layers.size()) return fail(MAFAT_EINVAL, "layer out of range");
+    const mafat::Layer& L = net->net.layers[layer];
+    if (L.type != mafat::L_CONV) return fail(MAFAT_EINVAL, "layer is not a convolution");
+    size_t nw = (size_t)L.c_out * L.c_in * L.k * L.k;
+    net->net.w[layer].assign(w, w + nw);
+    net->net.scale[layer].assign(scale, scale + L.c_out);
+    net->net.bias[layer].assign(bias, bias + L.c_out);
+    net->net.has_w[layer] = 1;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32_t* cuts, const int32_t* grid_n,
+                           const int32_t* grid_m, int32_t batch, int32_t dt, const mafat_plan_options* opt,
+                           mafat_plan_t** out) {
+    if (!net || !grid_n || !grid_m || !out) return fail(MAFAT_EINVAL, "null argument");
+    *out = nullptr;
+    if (n_groups == 2 && !cuts) return fail(MAFAT_EINVAL, "two groups need a cut");
+    if (n_groups != 1 && n_groups != 2) return fail(MAFAT_EINVAL, "n_groups must be 1 or 2");
+    if (dt != MAFAT_BF16 && dt != MAFAT_FP32) return fail(MAFAT_EINVAL, "unknown dtype");
+    mafat_plan_options o{};
+    if (opt) {
+        if (opt->struct_size < (int32_t)offsetof(mafat_plan_options, dry_run))
+            return fail(MAFAT_EINVAL, "mafat_plan_options.struct_size too small");
+        std::memcpy(&o, opt, std::min((size_t)opt->struct_size, sizeof(o)));
+    } else {
+        o.test_unpublished_task = -1;
+    }
+    mafat::PlanConfig cfg;
+    cfg.n_groups = n_groups;
+    cfg.cut = n_groups == 2 ? cuts[0] : 0;
+    for (int g = 0; g < n_groups; ++g) {
+        cfg.grid_n[g] = grid_n[g];
+        cfg.grid_m[g] = grid_m[g];
+    }
+    cfg.batch = batch;
+    cfg.dtype = dt;
+    cfg.ring_slots = o.ring_slots;
+    cfg.wave_tiles = o.wave_tiles;
+    cfg.unpublished_task = o.test_unpublished_task;
+
+    mafat_plan_s* p = new (std::nothrow) mafat_plan_s();
+    if (!p) return fail(MAFAT_ENOMEM, "host allocation failed");
+    bool unsup = false;
+    std::string err = mafat::build_plan(net->net, cfg, p->t, &unsup);
+    if (!err.empty()) {
+        delete p;
+        return fail(unsup ? MAFAT_EUNSUPPORTED : MAFAT_EINVAL, err);
+    }
+    p->shapes.layers = net->net.layers;
+    p->shapes.in_h = net->net.in_h;
+    p->shapes.in_w = net->net.in_w;
+    p->shapes.in_c = net->net.in_c;
+    p->dtype = dt;
+    p->esz = dt == MAFAT_BF16 ? 2 : 4;
+    p->timeout_ns = o.wait_timeout_ns > 0 ? o.wait_timeout_ns : 2000000000LL;
+    p->dry_run = o.dry_run != 0;
+    const mafat::PlanTables& t = p->t;
+    const mafat::Layer& L0 = net->net.layers[0];
+    p->in_bytes = (size_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in * p->esz;
+    p->out_bytes = (size_t)t.cfg.batch * t.out_h * t.out_w * t.out_c * p->esz;
+    p->cut_bytes = (size_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w * p->esz;
+    p->ctr_bytes = (size_t)(MAFAT_CTR_BASE + t.n_counters) * sizeof(uint32_t);
+    p->scratch_bytes = (int64_t)t.ring_slots * 2 * t.slot_buf_elems * p->esz;
+    p->weight_bytes = (dt == MAFAT_BF16 ? t.weight_elems * 2 : t.weight32_elems * 4) + 2 * t.sb_elems * 4;
+    if (p->dry_run) {
+        *out = p;
+        return MAFAT_OK;
+    }
+
+    cudaError_t e = cudaGetDevice(&p->device);
+    if (e != cudaSuccess) {
+        delete p;
+        return cuda_fail(e, "cudaGetDevice");
+    }
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+    // tensor-core kernel: one CTA per SM (shared memory and TMEM); check kernel: 8 small CTAs per SM
+    p->grid = o.max_ctas > 0 ? o.max_ctas : (dt == MAFAT_BF16 ? sms : 8 * sms);
+    if (p->grid <= 0) p->grid = 1;
+
+    auto bail = [&](cudaError_t ee, const char* what) {
+        free_plan_memory(p);
+        delete p;
+        return cuda_fail(ee, what);
+    };
+    if ((e = dalloc(p, &p->d_stages, t.stages.size() * sizeof(MafatStageDev))) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_tasks, t.tasks.size() * sizeof(MafatTaskDev))) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_items, t.items.size() * sizeof(MafatItemDev))) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_ctr, p->ctr_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_scale, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_bias, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if ((e = dalloc(p, &p->d_scratch, (size_t)p->scratch_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if (t.cfg.n_groups == 2 && (e = dalloc(p, &p->d_cut, p->cut_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
+
+    std::vector<float> w32, sc, bi;
+    mafat::pack_weights_fp32(net->net, t, w32, sc, bi);
+    if (dt == MAFAT_BF16) {
+        std::vector<uint16_t> wb;
+        mafat::pack_weights_bf16(net->net, t, wb);
+        if ((e = dalloc(p, &p->d_w, wb.size() * 2)) != cudaSuccess) return bail(e, "cudaMalloc");
+        if ((e = cudaMemcpy(p->d_w, wb.data(), wb.size() * 2, cudaMemcpyHostToDevice)) != cudaSuccess)
+            return bail(e, "cudaMemcpy");
+    } else {
+        if ((e = dalloc(p, &p->d_w, w32.size() * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
+        if ((e = cudaMemcpy(p->d_w, w32.data(), w32.size() * 4, cudaMemcpyHostToDevice)) != cudaSuccess)
+            return bail(e, "cudaMemcpy");
+    }
+    if ((e = cudaMemcpy(p->d_scale, sc.data(), sc.size() * 4, cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
+    if ((e = cudaMemcpy(p->d_bias, bi.data(), bi.size() * 4, cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
+    if ((e = cudaMemcpy(p->d_stages, t.stages.data(), t.stages.size() * sizeof(MafatStageDev), cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
+    if ((e = cudaMemcpy(p->d_tasks, t.tasks.data(), t.tasks.size() * sizeof(MafatTaskDev), cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
+    if ((e = cudaMemcpy(p->d_items, t.items.data(), t.items.size() * sizeof(MafatItemDev), cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
+    if ((e = cudaMemset(p->d_scratch, 0, (size_t)p->scratch_bytes)) != cudaSuccess) return bail(e, "cudaMemset");
+    if ((e = cudaMemset(p->d_ctr, 0, p->ctr_bytes)) != cudaSuccess) return bail(e, "cudaMemset");
+
+    if (dt == MAFAT_BF16) {
+        // one map per scratch-input task, then the cut tensor map
+        std::vector<CUtensorMap> maps(t.tmaps.size() + (t.cfg.n_groups == 2 ? 1 : 0));
+        std::string merr;
+        for (size_t i = 0; i < t.tmaps.size(); ++i) {
+            const mafat::TmapReq& q = t.tmaps[i];
+            const char* base = (const char*)p->d_scratch + (size_t)q.buf * t.slot_buf_elems * 2;
+            if (!encode_planar_map(&maps[i], base, q.w, q.h, q.c8, 1, q.cols_box, q.rows_box, q.chunk8, &merr)) {
+                free_plan_memory(p);
+                delete p;
+                return fail(MAFAT_ECUDA, merr);
+            }
+        }
+        if (t.cfg.n_groups == 2) {
+            if (!encode_planar_map(&maps.back(), p->d_cut, t.cut_w, t.cut_h, t.cut_c8, t.cfg.batch, t.cut_cols_box,
+                                   t.cut_rows_box, t.cut_chunk8, &merr)) {
+                free_plan_memory(p);
+                delete p;
+                return fail(MAFAT_ECUDA, merr);
+            }
+        }
+        if ((e = dalloc(p, &p->d_tmaps, maps.size() * sizeof(CUtensorMap))) != cudaSuccess) return bail(e, "cudaMalloc");
+        if (!maps.empty() &&
+            (e = cudaMemcpy(p->d_tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice)) !=
+                cudaSuccess)
+            return bail(e, "cudaMemcpy");
+    }
+    *out = p;
+    g_err.clear();
+    return MAFAT_OK;
+}
+
+mafat_status mafat_plan(const mafat_net_t* net, int32_t n_groups, const int32_t* cuts, const int32_t* grid_n,
+                        const int32_t* grid_m, int32_t batch, int32_t dt, mafat_plan_t** out) {
+    return mafat_plan_ex(net, n_groups, cuts, grid_n, grid_m, batch, dt, nullptr, out);
+}
+
+mafat_status mafat_run(const mafat_plan_t* plan, const void* input, void* output, void* stream) {
+    if (!plan) return fail(MAFAT_EINVAL, "null plan");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    std::lock_guard<std::mutex> lk(p->mu);
+    return launch(p, input, output, (cudaStream_t)stream);
+}
+
+mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* cut_out, void* output,
+                             void* stream) {
+    if (!plan) return fail(MAFAT_EINVAL, "null plan");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    std::lock_guard<std::mutex> lk(p->mu);
+    mafat_status s = launch(p, input, output, (cudaStream_t)stream);
+    if (s != MAFAT_OK) return s;
+    if (p->t.cfg.n_groups == 2 && cut_out) {
+        cudaError_t e = cudaMemcpyAsync(cut_out, p->d_cut, p->cut_bytes, cudaMemcpyDeviceToDevice, (cudaStream_t)stream);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
+    }
+    return MAFAT_OK;
+}
+
+mafat_status mafat_sync_status(const mafat_plan_t* plan, void* stream) {
+    if (!plan) return fail(MAFAT_EINVAL, "null plan");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    uint32_t st = 0;
+    e = cudaMemcpy(&st, p->d_ctr + MAFAT_CTR_STATUS, sizeof(st), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+    if (st == MAFAT_DEV_OK) return MAFAT_OK;
+    cudaMemset(p->d_ctr + MAFAT_CTR_STATUS, 0, sizeof(uint32_t));
+    if (st == MAFAT_DEV_TIMEOUT) return fail(MAFAT_ETIMEOUT, "a tile waited on another tile that never completed");
+    return fail(MAFAT_EDEVICE, "a device pipeline wait ran out");
+}
+
+mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, void* output_host, void* stream) {
+    if (!plan || !input_host || !output_host) return fail(MAFAT_EINVAL, "null argument");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    cudaStream_t s = (cudaStream_t)stream;
+    {
+        std::lock_guard<std::mutex> lk(p->mu);
+        cudaError_t e;
+        if (!p->d_in_stage) {
+            if ((e = cudaMalloc(&p->d_in_stage, p->in_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+            if ((e = cudaMalloc(&p->d_out_stage, p->out_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+        }
+        if ((e = cudaMemcpyAsync(p->d_in_stage, input_host, p->in_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+            return cuda_fail(e, "cudaMemcpyAsync");
+        mafat_status st = launch(p, p->d_in_stage, p->d_out_stage, s);
+        if (st != MAFAT_OK) return st;
+        if ((e = cudaMemcpyAsync(output_host, p->d_out_stage, p->out_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+            return cuda_fail(e, "cudaMemcpyAsync");
+    }
+    return mafat_sync_status(plan, stream);
+}
+
+mafat_status mafat_tile_region(const mafat_plan_t* plan, int32_t group, int32_t ti, int32_t tj, int32_t layer,
+                               int32_t in_rect[4], int32_t out_rect[4]) {
+    if (!plan || !in_rect || !out_rect) return fail(MAFAT_EINVAL, "null argument");
+    const mafat::PlanTables& t = plan->t;
+    if (group < 0 || group >= t.cfg.n_groups) return fail(MAFAT_EINVAL, "group out of range");
+    if (ti < 0 || ti >= t.cfg.grid_n[group] || tj < 0 || tj >= t.cfg.grid_m[group])
+        return fail(MAFAT_EINVAL, "tile out of range");
+    if (layer < t.groups[group][0] || layer > t.groups[group][1]) return fail(MAFAT_EINVAL, "layer not in group");
+    std::vector<mafat::Rect> outs, ins;
+    mafat::tile_regions(plan->shapes, t.groups[group][0], t.groups[group][1], t.cfg.grid_n[group],
+                        t.cfg.grid_m[group], ti, tj, outs, ins);
+    const mafat::Rect& i = ins[layer];
+    const mafat::Rect& o = outs[layer];
+    in_rect[0] = i.y0; in_rect[1] = i.y1; in_rect[2] = i.x0; in_rect[3] = i.x1;
+    out_rect[0] = o.y0; out_rect[1] = o.y1; out_rect[2] = o.x0; out_rect[3] = o.x1;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_net_tile_region(const mafat_net_t* net, int32_t first, int32_t last, int32_t n, int32_t m,
+                                   int32_t ti, int32_t tj, int32_t layer, int32_t in_rect[4], int32_t out_rect[4]) {
+    if (!net || !in_rect || !out_rect) return fail(MAFAT_EINVAL, "null argument");
+    const int nl = (int)net->net.layers.size();
+    if (first < 0 || last >= nl || first > last) return fail(MAFAT_EINVAL, "bad layer range");
+    if (n <= 0 || m <= 0 || ti < 0 || ti >= n || tj < 0 || tj >= m) return fail(MAFAT_EINVAL, "tile out of range");
+    if (layer < first || layer > last) return fail(MAFAT_EINVAL, "layer not in range");
+    std::vector<mafat::Rect> outs, ins;
+    mafat::tile_regions(net->net, first, last, n, m, ti, tj, outs, ins);
+    const mafat::Rect& i = ins[layer];
+    const mafat::Rect& o = outs[layer];
+    in_rect[0] = i.y0; in_rect[1] = i.y1; in_rect[2] = i.x0; in_rect[3] = i.x1;
+    out_rect[0] = o.y0; out_rect[1] = o.y1; out_rect[2] = o.x0; out_rect[3] = o.x1;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_predict_layer_group(const mafat_net_t* net, int32_t first, int32_t last, int32_t n, int32_t m,
+                                       double bias_mib, int32_t input_factor, double* out_mib) {
+    if (!net || !out_mib) return fail(MAFAT_EINVAL, "null argument");
+    const int nl = (int)net->net.layers.size();
+    if (first < 0 || last >= nl || first > last || n <= 0 || m <= 0) return fail(MAFAT_EINVAL, "bad arguments");
+    *out_mib = mafat::predict_layer_group(net->net, first, last, n, m, bias_mib, input_factor);
+    return MAFAT_OK;
+}
+
+mafat_status mafat_predict_mem(const mafat_net_t* net, int32_t cut, int32_t n1, int32_t m1, int32_t n2, int32_t m2,
+                               double bias_mib, double* out_mib) {
+    if (!net || !out_mib) return fail(MAFAT_EINVAL, "null argument");
+    if (n1 <= 0 || m1 <= 0 || n2 <= 0 || m2 <= 0) return fail(MAFAT_EINVAL, "grid sizes must be positive");
+    *out_mib = mafat::predict_mem(net->net, cut, n1, m1, n2, m2, bias_mib);
+    return MAFAT_OK;
+}
+
+mafat_status mafat_search(const mafat_net_t* net, double limit_mib, double bias_mib, int32_t* top_tile,
+                          int32_t* cut, int32_t* bottom_tile) {
+    if (!net || !top_tile || !cut || !bottom_tile) return fail(MAFAT_EINVAL, "null argument");
+    int a, b, c;
+    mafat::search(net->net, limit_mib, bias_mib, &a, &b, &c);
+    *top_tile = a;
+    *cut = b;
+    *bottom_tile = c;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out) {
+    if (!plan || !out) return fail(MAFAT_EINVAL, "null argument");
+    if (out->struct_size < (int32_t)sizeof(mafat_plan_stats)) return fail(MAFAT_EINVAL, "struct_size too small");
+    const mafat::PlanTables& t = plan->t;
+    mafat_plan_stats s{};
+    s.struct_size = (int32_t)sizeof(mafat_plan_stats);
+    s.n_groups = t.cfg.n_groups;
+    s.n_tiles = t.n_tiles;
+    s.n_tasks = (int32_t)t.tasks.size();
+    s.n_items = (int64_t)t.items.size();
+    s.useful_flops = t.useful_flops;
+    s.executed_flops = t.executed_flops * 1.0;
+    s.issued_flops = t.issued_flops;
+    s.predicted_mib = t.predicted_mib;
+    s.group_io_bytes = t.group_io_elems * plan->esz;
+    s.weight_bytes = plan->weight_bytes;
+    s.scratch_bytes = plan->scratch_bytes;
+    s.workspace_bytes = plan->workspace_bytes;
+    s.smem_bytes_per_cta = plan->dtype == MAFAT_BF16 ? (int64_t)mafat_tc_smem_bytes() : 4;
+    s.ring_slots = t.ring_slots;
+    s.wave_tiles = t.wave_tiles;
+    s.max_ctas = plan->grid;
+    s.dtype = plan->dtype;
+    *out = s;
+    return MAFAT_OK;
+}
+
+int32_t mafat_launches_per_run(const mafat_plan_t* plan) { return plan ? 1 : 0; }
+
+void mafat_plan_destroy(mafat_plan_t* plan) {
+    if (!plan) return;
+    free_plan_memory(plan);
+    delete plan;
+}
+
+void mafat_net_destroy(mafat_net_t* net) { delete net; }
+
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, int32_t lbo_is_k,
+                             void* stream) {
+    if (!a_dev || !b_dev || !d_dev) return fail(MAFAT_EINVAL, "null argument");
+    if (n < 16 || n > 256 || n % 16 != 0) return fail(MAFAT_EINVAL, "n must be a multiple of 16 in 16..256");
+    cudaError_t e = mafat_launch_diag_umma(a_dev, b_dev, d_dev, n, lbo_is_k ? 1 : 0, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "diag launch");
+    e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "diag sync");
+    return MAFAT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,105 @@
+// Device side of the persistent tile scheduler shared by both kernels.
+//
+// Work items are handed out in a fixed global order by an atomic ticket.  Every
+// dependency of an item (the previous fused stage of its tile, the tile that
+// last used its scratch slot, or all group-1 tiles of its frame) consists of
+// items with smaller tickets, and a CTA only takes a ticket while it runs, so
+// the smallest unfinished ticket can always make progress.  Waits are bounded
+// by a wall-clock limit: when it runs out the kernel records
+// MAFAT_DEV_TIMEOUT, raises the abort word and every later wait returns at
+// once, so the launch always ends.
+#pragma once
+#include "kernels.h"
+
+namespace mafat_dev {
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void red_release_add(uint32_t* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ void record_status(uint32_t* ctr, uint32_t code) {
+    atomicCAS(&ctr[MAFAT_CTR_STATUS], 0u, code);
+    atomicExch(&ctr[MAFAT_CTR_ABORT], 1u);
+}
+
+__device__ __forceinline__ bool aborted(const uint32_t* ctr) {
+    return *(volatile const uint32_t*)&ctr[MAFAT_CTR_ABORT] != 0u;
+}
+
+// Wait until ctr[idx] >= target (acquire), bounded by timeout_ns.
+__device__ __forceinline__ void wait_counter(uint32_t* ctr, int idx, int target, int64_t timeout_ns) {
+    if (idx < 0) return;
+    const uint32_t* p = ctr + idx;
+    if (ld_acquire_u32(p) >= (uint32_t)target) return;
+    uint64_t t0 = globaltimer_ns();
+    uint32_t ns = 32;
+    while (true) {
+        if (ld_acquire_u32(p) >= (uint32_t)target) return;
+        if (aborted(ctr)) return;
+        if ((int64_t)(globaltimer_ns() - t0) > timeout_ns) {
+            record_status(ctr, MAFAT_DEV_TIMEOUT);
+            return;
+        }
+        __nanosleep(ns);
+        if (ns < 1024) ns <<= 1;
+    }
+}
+
+// Wait for both dependencies of an item; afterwards the data they published is
+// visible to this thread's generic and async-proxy (TMA) reads.
+__device__ __forceinline__ void wait_item_deps(uint32_t* ctr, const MafatItemDev& it, int64_t timeout_ns) {
+    wait_counter(ctr, it.dep0, it.dep0_target, timeout_ns);
+    wait_counter(ctr, it.dep1, it.dep1_target, timeout_ns);
+    fence_proxy_async_global();
+}
+
+// Publish completion of an item (call once, after all of its stores are
+// ordered before this thread by a CTA-level barrier).
+__device__ __forceinline__ void publish_item(uint32_t* ctr, const MafatItemDev& it, int done_ctr) {
+    if (it.flags & 1) return;  // test hook: never published
+    __threadfence();
+    red_release_add(ctr + done_ctr, 1u);
+    if (it.extra_ctr >= 0) red_release_add(ctr + it.extra_ctr, 1u);
+}
+
+// Called by every thread of a CTA after its last use of the counters: the last
+// CTA of the launch to get here zeroes the counter block (all but the status
+// word) for the next run on the same stream.
+__device__ __forceinline__ void finish_cta(uint32_t* ctr, int n_ctr) {
+    __shared__ int s_last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const uint32_t done = atomicAdd(&ctr[MAFAT_CTR_EXIT], 1u);
+        s_last = (done == gridDim.x - 1) ? 1 : 0;
+        __threadfence();
+    }
+    __syncthreads();
+    if (!s_last) return;
+    for (int i = threadIdx.x; i < n_ctr; i += blockDim.x)
+        if (i != MAFAT_CTR_STATUS && i != MAFAT_CTR_EXIT) ctr[i] = 0u;
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        ctr[MAFAT_CTR_EXIT] = 0u;
+        __threadfence();
+    }
+}
+
+}  // namespace mafat_dev

@@ -1,0 +1,147 @@
+"""Host planner of the C ABI (shapes, Grid regions, Algorithms 1-2, work tables) against the oracle.
+
+All on the CPU: network queries need no device, and plans are built with
+dry_run so that no device memory is touched.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+
+@pytest.fixture(scope="module")
+def mf():
+    import __graft_entry__ as g
+    g.build()
+    import paper_2107_06960_gb300 as mf
+    return mf
+
+
+def _net(mf, layers, size, c=3, dtype="bf16", seed=1):
+    net = mf.Net(layers, size, size, c)
+    net.set_params(synth.make_params(layers, c, seed, dtype))
+    return net
+
+
+@pytest.mark.parametrize("size", [608, 416, 1216, 64, 96])
+def test_shapes_match_oracle(mf, size):
+    net = _net(mf, synth.YOLO16, size)
+    ref = oracle.layer_shapes(synth.YOLO16, size, size, 3)
+    for l, sh in enumerate(ref):
+        assert net.shape(l) == (sh["h_in"], sh["w_in"], sh["c_in"], sh["h_out"], sh["w_out"], sh["c_out"])
+
+
+@pytest.mark.parametrize("size,first,last,n,m", [
+    (608, 0, 7, 5, 5), (608, 8, 15, 2, 2), (416, 0, 15, 3, 3), (1216, 0, 7, 8, 8), (1216, 8, 15, 4, 4),
+    (608, 0, 1, 5, 5), (608, 2, 15, 3, 2), (64, 0, 11, 5, 5), (96, 12, 15, 4, 3), (608, 0, 15, 7, 1)])
+def test_tile_regions_match_oracle(mf, size, first, last, n, m):
+    layers = synth.YOLO16
+    net = _net(mf, layers, size)
+    shapes = oracle.layer_shapes(layers, size, size, 3)
+    for i in range(n):
+        for j in range(m):
+            ref = oracle.tile_regions(layers, shapes, (first, last), n, m, i, j)
+            for l in range(first, last + 1):
+                out_r, in_r = net.tile_region(first, last, n, m, i, j, l)
+                if ref[l][0][1] <= ref[l][0][0] or ref[l][0][3] <= ref[l][0][2]:
+                    assert out_r[1] <= out_r[0] or out_r[3] <= out_r[2]
+                    continue
+                assert out_r == ref[l][0] and in_r == ref[l][1]
+
+
+@pytest.mark.parametrize("size", [608, 416])
+def test_predictor_matches_oracle_exactly(mf, size):
+    layers = synth.YOLO16
+    net = _net(mf, layers, size)
+    shapes = oracle.layer_shapes(layers, size, size, 3)
+    for cut in (None, 2, 4, 8, 12):
+        for t1 in range(1, 6):
+            for t2 in (1, 2, 3):
+                grids = [(t1, t1)] if cut is None else [(t1, t1), (t2, t2)]
+                ref = oracle.predict_mem(layers, shapes, cut, grids)
+                got = net.predict_mem(cut if cut is not None else 16, t1, t1, t2, t2)
+                assert got == ref
+    for first, last in ((0, 15), (0, 7), (8, 15), (2, 2)):
+        for f in (1, 2):
+            ref = oracle.predict_layer_group(layers, shapes, (first, last), 3, 2, 31.0, input_factor=f)
+            assert net.predict_layer_group(first, last, 3, 2, 31.0, f) == ref
+
+
+def test_search_matches_oracle_for_table1_limits(mf):
+    layers = synth.YOLO16
+    net = _net(mf, layers, 608)
+    shapes = oracle.layer_shapes(layers, 608, 608, 3)
+    for limit in (256, 192, 128, 96, 80, 64, 48, 32, 16, 1000, 1):
+        assert net.search(float(limit)) == oracle.get_config(layers, shapes, float(limit))
+
+
+def _region_flops(layers, size, cut, grids, batch):
+    shapes = oracle.layer_shapes(layers, size, size, 3)
+    tot = 0
+    for g, (n, m) in zip(oracle.groups_of(len(layers), cut), grids):
+        for i in range(n):
+            for j in range(m):
+                regs = oracle.tile_regions(layers, shapes, g, n, m, i, j)
+                for l in range(g[0], g[1] + 1):
+                    t, k, s, p, f = layers[l]
+                    if t != "conv":
+                        continue
+                    (y0, y1, x0, x1), _ = regs[l]
+                    tot += 2 * max(y1 - y0, 0) * max(x1 - x0, 0) * f * shapes[l]["c_in"] * k * k
+    return tot * batch
+
+
+@pytest.mark.parametrize("name", ["yolo16_416_1x3x3", "yolo16_608_5x5_c8_2x2", "yolo16_1216_b8_8x8_c8_4x4"])
+def test_plan_statistics(mf, name):
+    wl = synth.WORKLOADS[name]
+    layers, size, batch = wl["layers"], wl["h"], wl["batch"]
+    net = _net(mf, layers, size)
+    plan = mf.Plan(net, wl["cut"], wl["grids"], batch=batch, dtype=mf.BF16, dry_run=True)
+    st = plan.stats()
+    shapes = oracle.layer_shapes(layers, size, size, 3)
+    assert st["useful_flops"] == oracle.conv_flops(layers, shapes) * batch
+    assert st["executed_flops"] == _region_flops(layers, size, wl["cut"], wl["grids"], batch)
+    assert st["issued_flops"] >= st["executed_flops"] >= st["useful_flops"]
+    ref_pred = oracle.predict_mem(layers, shapes, wl["cut"], wl["grids"])
+    assert st["predicted_mib"] == ref_pred
+    ntiles = sum(n * m for n, m in wl["grids"][:1 if wl["cut"] is None else 2])
+    assert st["n_tiles"] == ntiles * batch
+
+
+def test_headline_plan_numbers(mf):
+    # 608x608, cut after layer 7, 5x5 / 2x2: 26.0 GFLOP useful, 13.7 % halo recompute
+    wl = synth.WORKLOADS["yolo16_608_5x5_c8_2x2"]
+    net = _net(mf, wl["layers"], 608)
+    st = mf.Plan(net, 8, wl["grids"], dry_run=True).stats()
+    assert abs(st["useful_flops"] / 1e9 - 26.0007) < 1e-3
+    assert abs(st["executed_flops"] / st["useful_flops"] - 1.137) < 0.01
+
+
+def test_plan_validation_errors(mf):
+    layers = synth.YOLO16
+    net = _net(mf, layers, 64)
+    with pytest.raises(mf.MafatError) as e:     # cut between a conv and its max-pool
+        mf.Plan(net, 1, [(2, 2), (2, 2)], dry_run=True)
+    assert e.value.status == 2
+    with pytest.raises(mf.MafatError) as e:
+        mf.Plan(net, 16, [(2, 2), (2, 2)], dry_run=True)
+    assert e.value.status == 1
+    with pytest.raises(mf.MafatError) as e:
+        mf.Plan(net, None, [(0, 2)], dry_run=True)
+    assert e.value.status == 1
+    bare = mf.Net(layers, 64, 64, 3)             # weights never set
+    with pytest.raises(mf.MafatError) as e:
+        mf.Plan(bare, None, [(1, 1)], dry_run=True)
+    assert e.value.status == 1
+    with pytest.raises(mf.MafatError) as e:      # odd map under a max-pool
+        mf.Net(layers, 66, 66, 3)
+    assert e.value.status == 2
+
+
+def test_grid_finer_than_output_skips_empty_tiles(mf):
+    layers = synth.YOLO16
+    net = _net(mf, layers, 64)
+    # group 1 output at cut 12 is 4x4; a 5x5 grid has empty rows/columns of tiles
+    st = mf.Plan(net, 12, [(5, 5), (3, 3)], dry_run=True).stats()
+    assert st["n_tiles"] == 4 * 4 + 3 * 3
