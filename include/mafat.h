@@ -220,6 +220,23 @@ const char* mafat_last_error(void);
 /* Library version string. */
 const char* mafat_version(void);
 
+/* Allocation-free run; the paper has no counterpart.  For callers that cannot
+ * have device memory allocated for them while they run (code executing during
+ * a global-mode stream capture, where cudaMalloc is refused; real-time loops
+ * that forbid allocator calls; processes whose device memory is owned and
+ * budgeted by another allocator).  Runs an FP32 plan created beforehand (its
+ * weights and tables are read in place) with all per-run scratch -- tile
+ * buffers, cut tensor, scheduler counters -- taken from one fixed 32 MiB
+ * device area inside this library, which every GPU that loads the library
+ * keeps until exit; it calls no allocation routine.  Plans needing more
+ * scratch than 32 MiB are refused with MAFAT_EINVAL; BF16 plans with
+ * MAFAT_EUNSUPPORTED.  Layouts as mafat_run; asynchronous on `stream`.  All
+ * calls share the area: calls that overlap on the GPU race.  The first call
+ * on each device looks up the area's device address, so make it before any
+ * stream capture starts.  Device-side wait errors of these calls are not
+ * reported by mafat_sync_status (which reads the plan's own status word). */
+mafat_status mafat_run_fp32_noalloc(const mafat_plan_t* plan, const void* input, void* output, void* stream);
+
 /* Diagnostic with no counterpart in the paper: one 128 x n x 16 bf16 tensor-core
  * product D = A * B^T on one CTA, to check the operand and accumulator layouts
  * the kernels use.  a_dev [128][16], b_dev [n][16] (bf16, row-major, device),

@@ -70,6 +70,7 @@ _SIGNATURES = [
     ("mafat_last_error", ctypes.c_char_p, []),
     ("mafat_version", ctypes.c_char_p, []),
     ("mafat_diag_umma", i32, [vp, vp, vp, i32, i32, vp]),
+    ("mafat_run_fp32_noalloc", i32, [vp, vp, vp, vp]),
 ]
 EXPORTED = [s[0] for s in _SIGNATURES]
 
@@ -215,6 +216,13 @@ class Plan:
 
     def run_debug(self, inp, cut_out, out, stream=None):
         _check(lib.mafat_run_debug(self.handle, _ptr(inp), _ptr(cut_out), _ptr(out), _stream(stream, inp)))
+
+    def run_noalloc(self, inp, out, stream=None):
+        """Run an FP32 plan with its per-run scratch in the library's fixed 32 MiB
+        device area (mafat_run_fp32_noalloc): no allocation at all, for callers
+        that may not allocate device memory while they run.  Calls share the
+        area and must not overlap on the GPU."""
+        _check(lib.mafat_run_fp32_noalloc(self.handle, _ptr(inp), _ptr(out), _stream(stream, inp)))
 
     def run_host(self, inp_host, out_host, stream=None):
         _check(lib.mafat_run_host(self.handle, _ptr(inp_host), _ptr(out_host), _stream(stream)))

@@ -171,6 +171,37 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
 
 }  // namespace
 
+// Internal accessor for the allocation-free entry point (noalloc.cu): kernel
+// parameters of an fp32 plan with its own scratch, cut tensor and counters left
+// out (the caller supplies them), plus the sizes those three need.
+mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* kp, size_t* ctr_bytes,
+                                        size_t* cut_bytes, size_t* scratch_bytes, int* grid, int* device) {
+    const mafat_plan_s* p = plan;
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    if (p->dtype != MAFAT_FP32) return fail(MAFAT_EUNSUPPORTED, "this entry point runs fp32 plans only");
+    MafatKParams k{};
+    k.stages = p->d_stages;
+    k.tasks = p->d_tasks;
+    k.items = p->d_items;
+    k.n_items = (int32_t)p->t.items.size();
+    k.tmaps = nullptr;
+    k.cut_tmap = -1;
+    k.w_f32 = (const float*)p->d_w;
+    k.scale = p->d_scale;
+    k.bias = p->d_bias;
+    k.n_ctr = (int32_t)(p->ctr_bytes / sizeof(uint32_t));
+    k.timeout_ns = p->timeout_ns;
+    *kp = k;
+    *ctr_bytes = p->ctr_bytes;
+    *cut_bytes = p->t.cfg.n_groups == 2 ? p->cut_bytes : 0;
+    *scratch_bytes = (size_t)p->scratch_bytes;
+    *grid = p->grid;
+    *device = p->device;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_internal_fail(mafat_status s, const char* msg) { return fail(s, msg); }
+
 extern "C" {
 
 const char* mafat_last_error(void) { return g_err.c_str(); }
