@@ -86,7 +86,10 @@ typedef struct {
                                       published, so that waits on it run out (-1: none) */
     int32_t dry_run;            /* 1: build the host-side tables only (statistics and region
                                    queries work; runs are refused); needs no GPU */
-    int32_t reserved[6];
+    int32_t trace;              /* 1: record per-item timestamps on every run (mafat_plan_trace) */
+    int32_t force_nblk;         /* output channels per work item for every stage (0: chosen per stage) */
+    int32_t force_mb;           /* 16x8 pixel blocks per work item for every stage (0: chosen per stage) */
+    int32_t reserved[3];
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */
@@ -207,6 +210,17 @@ mafat_status mafat_search(const mafat_net_t* net, double limit_mib, double bias_
 
 /* Plan statistics (struct_size must be set by the caller). */
 mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out);
+
+/* Per-item trace of the last run of a plan created with options.trace = 1
+ * (synchronises `stream`).  out receives n_items records of MAFAT_TRACE_WORDS
+ * uint64 in hand-out order: {global ns when the item's ticket was taken, when
+ * its dependencies were satisfied, when its accumulator was ready for the
+ * epilogue, when its completion was published, SM id, task index << 16 |
+ * network layer of its convolution, when its first input halo had landed in
+ * shared memory, when its last MMA was issued}.  max_words bounds what is
+ * written. */
+#define MAFAT_TRACE_WORDS 8
+mafat_status mafat_plan_trace(const mafat_plan_t* plan, uint64_t* out, int64_t max_words, void* stream);
 
 /* Number of kernel launches one mafat_run makes. */
 int32_t mafat_launches_per_run(const mafat_plan_t* plan);

@@ -33,7 +33,7 @@ class LayerDesc(ctypes.Structure):
 class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
-                ("reserved", i32 * 6)]
+                ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("reserved", i32 * 3)]
 
 
 class PlanStats(ctypes.Structure):
@@ -65,6 +65,7 @@ _SIGNATURES = [
     ("mafat_search", i32, [vp, dbl, dbl, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_plan_stats_get", i32, [vp, ctypes.POINTER(PlanStats)]),
     ("mafat_launches_per_run", i32, [vp]),
+    ("mafat_plan_trace", i32, [vp, vp, i64, vp]),
     ("mafat_plan_destroy", None, [vp]),
     ("mafat_net_destroy", None, [vp]),
     ("mafat_last_error", ctypes.c_char_p, []),
@@ -192,7 +193,8 @@ class Plan:
     """mafat_plan_ex / mafat_run: fused-tile execution of a network on the current CUDA device."""
 
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
-                 max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False):
+                 max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
+                 force_nblk=0, force_mb=0):
         self.net = net
         n_groups = 1 if cut is None else 2
         grids = list(grids)[:n_groups]
@@ -205,6 +207,8 @@ class Plan:
         opt.wait_timeout_ns = wait_timeout_ns
         opt.test_unpublished_task = test_unpublished_task
         opt.dry_run = 1 if dry_run else 0
+        opt.trace = 1 if trace else 0
+        opt.force_nblk, opt.force_mb = force_nblk, force_mb
         h = vp()
         _check(lib.mafat_plan_ex(net.handle, n_groups, cuts, gn, gm, batch, dtype, ctypes.byref(opt),
                                  ctypes.byref(h)))
@@ -244,6 +248,16 @@ class Plan:
         s.struct_size = ctypes.sizeof(PlanStats)
         _check(lib.mafat_plan_stats_get(self.handle, ctypes.byref(s)))
         return {k: getattr(s, k) for k, _ in PlanStats._fields_ if k != "struct_size"}
+
+    def trace(self, stream=None):
+        """Per-item records of the last run (plan made with trace=True): numpy uint64
+        [n_items][8] = ticket taken, deps satisfied, accumulator ready, published (ns), SM,
+        task << 16 | layer, first halo landed, last MMA issued (ns)."""
+        import numpy as np
+        n = self.stats()["n_items"]
+        out = np.zeros((n, 8), dtype=np.uint64)
+        _check(lib.mafat_plan_trace(self.handle, out.ctypes.data, out.size, _stream(stream)))
+        return out
 
     def launches_per_run(self):
         return lib.mafat_launches_per_run(self.handle)

@@ -8,10 +8,11 @@
 //                       reads, which rectangle of the conv output it computes
 //                       (the tile's region from the Grid back-traversal,
 //                       Sec. 4.1) and where the result goes;
-//   * MafatItemDev   -- the work list in hand-out order: one item is a
-//                       16 x 8 block of conv output pixels x one block of
-//                       output channels of a task, with up to two completion
-//                       counters it must wait for.
+//   * MafatItemDev   -- the work list in hand-out order: one item is up to
+//                       `mb` 16 x 8 blocks of conv output pixels (stacked
+//                       along rows) x one block of output channels of a
+//                       task, with up to two completion counters it must
+//                       wait for.
 //
 // Activations are stored in "octet-planar" layout [C/8][H][W][8]: 8 channels of
 // one pixel are 16 bytes (bf16) or 32 bytes (fp32) and consecutive pixels of a
@@ -23,8 +24,8 @@
 #define MAFAT_BLK_ROWS 16   // conv output rows of one M block
 #define MAFAT_BLK_COLS 8    // conv output columns of one M block (M = 128)
 #define MAFAT_MAX_NBLK 256  // output channels of one item (MMA N)
-#define MAFAT_A_STAGE_BYTES 23552  // shared-memory A halo stage of the tensor-core kernel
-#define MAFAT_B_STAGE_BYTES 32768  // shared-memory weight-blob stage of the tensor-core kernel
+#define MAFAT_A_STAGE_BYTES 36864   // shared-memory A halo stage of the tensor-core kernel (x2)
+#define MAFAT_B_PIECE_BYTES 75776   // one of the two shared-memory weight buffers (x2)
 
 enum { MAFAT_BUF_USER_IN = 0, MAFAT_BUF_CUT = 1, MAFAT_BUF_SCRATCH = 2, MAFAT_BUF_USER_OUT = 3 };
 
@@ -42,9 +43,13 @@ struct MafatStageDev {
     int32_t paired;       // 1: cin8 == 1, two taps share one K=16 step
     int32_t n_bsteps;     // weight blobs per chunk (taps, or tap pairs)
     int32_t kst;          // K=16 MMA steps per blob
-    int32_t rows_box, cols_box;  // A halo box (pixels)
+    int32_t mb;           // M blocks per item (stacked along rows, one TMEM accumulator each)
+    int32_t rows_box, cols_box;  // A halo box (pixels): 16*mb + k - 1 rows, 8 + k - 1 columns
     int64_t w_off;        // element offset of this stage's packed bf16 weights
     int32_t blob_elems;   // elements of one blob (n_blk * 16 * kst)
+    int32_t set_bytes;    // bytes of the weights of one output-channel block (all chunks and blobs)
+    int32_t bpp;          // blobs per weight piece (a piece fills at most one shared-memory buffer)
+    int32_t n_pieces;     // pieces per channel block (1: the set stays resident across items)
     int32_t sb_off;       // offset into the scale / bias arrays
     int64_t w32_off;      // element offset of the fp32 weights [cout][cin][k][k]
 };
@@ -75,7 +80,9 @@ struct MafatItemDev {
     int32_t task;
     int16_t by, bx;       // M block
     int16_t nb;           // output-channel block
+    int16_t nbk;          // M blocks of this item (rows by .. by+nbk-1)
     int16_t flags;        // bit 0: do not publish completion (test hook)
+    int16_t pad;
     int32_t dep0, dep0_target;  // counter index (-1: none) and value to wait for
     int32_t dep1, dep1_target;
     int32_t extra_ctr;    // second counter bumped on completion (-1: none)

@@ -34,7 +34,14 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
         const MafatItemDev it = p.items[ticket];
         const MafatTaskDev tk = p.tasks[it.task];
         const MafatStageDev st = p.stages[tk.stage];
-        if (tid == 0) mafat_dev::wait_item_deps(p.ctr, it, p.timeout_ns);
+        if (tid == 0) {
+            if (p.trace) {
+                mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
+                mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
+            }
+            mafat_dev::wait_item_deps(p.ctr, it, p.timeout_ns);
+            if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
+        }
         __syncthreads();
 
         const float* in = buf_ptr(p, tk.in_kind) + tk.in_off;
@@ -42,12 +49,13 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
                               : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
                                                                 : p.scratch) + tk.out_off;
         const float* w = p.w_f32 + st.w32_off;
-        const int Y = tk.cy0 + it.by * MAFAT_BLK_ROWS + r;
         const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + c;
-        const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
         const int k = st.k, kk = st.k * st.k;
         const int o_end = min((it.nb + 1) * st.n_blk, st.cout);
+        for (int blk = 0; blk < it.nbk; ++blk)
         for (int o0 = it.nb * st.n_blk; o0 < o_end; o0 += 8) {
+            const int Y = tk.cy0 + (it.by + blk) * MAFAT_BLK_ROWS + r;
+            const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
             float acc[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q) acc[q] = 0.f;
@@ -96,7 +104,14 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
         }
         __threadfence();
         __syncthreads();
-        if (tid == 0) mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
+        if (tid == 0) {
+            mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
+            if (p.trace) {
+                const uint64_t t = mafat_dev::globaltimer_ns();
+                mafat_dev::trace_put(p.trace, ticket, 2, t);
+                mafat_dev::trace_put(p.trace, ticket, 3, t);
+            }
+        }
     }
     mafat_dev::finish_cta(p.ctr, p.n_ctr);
 }

@@ -19,14 +19,18 @@
 //    With 8 input channels (the first layer), one K=16 step covers two taps:
 //    its two K core matrices sit at the two taps' offsets (LBO = their
 //    distance).
-//  * B: weights pre-packed on the host in exactly the shared-memory image of
-//    one (chunk, tap) blob, fetched with one bulk copy.
+//  * B: weights pre-packed on the host in exactly the shared-memory image of the
+//    whole weight set of one (stage, output-channel block), fetched with one bulk
+//    copy and kept resident while the CTA's consecutive items use the same set
+//    (every copy costs a few hundred cycles of TMA time however small it is, so
+//    the per-item copies are only the A halo boxes).
 //
 // Warp roles (192 threads): warps 0-3 epilogue (warp w reads TMEM lanes
 // 32w..32w+31 = conv rows 4w..4w+3 of the block), warp 4 scheduler + TMA
-// producer, warp 5 TMEM allocator + MMA issuer.  Rings: 2 A stages, 5 B stages,
-// 2 TMEM accumulators of 256 columns (the epilogue of one item overlaps the
-// MMAs of the next), and a 4-deep queue of item indices.
+// producer, warp 5 TMEM allocator + MMA issuer.  Shared memory: 2 A halo stages,
+// one resident weight set, and a 4-deep queue of item indices; TMEM: 2
+// accumulators of 256 columns (the epilogue of one item overlaps the MMAs of
+// the next).
 //
 // Epilogue: y = leaky_0.1(scale[n] * acc + bias[n]); for a fused 2x2/s2
 // max-pool the quad of pixels {(r, c), (r, c+1), (r+1, c), (r+1, c+1)} are lanes
@@ -47,19 +51,18 @@ constexpr int kThreads = 192;
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kAStages = 2;
-constexpr int kBStages = 5;
 constexpr int kQDepth = 4;
-constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;  // >= 8 octets x 18 x 10 pixels x 16 B, multiple of 1024
-constexpr int kBStageBytes = MAFAT_B_STAGE_BYTES;  // 256 rows x 64 channels x 2 B
+constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;   // one A halo box, multiple of 1024
+constexpr int kBPieceBytes = MAFAT_B_PIECE_BYTES;   // one of two weight buffers
 constexpr int kTmemCols = 512;        // two accumulators of up to 256 fp32 columns
 constexpr int kAccStride = 256;
 
 // shared-memory map (offsets from a 1024-aligned base)
 constexpr int kBarAFull = 0;
 constexpr int kBarAEmpty = kBarAFull + kAStages;
-constexpr int kBarBFull = kBarAEmpty + kAStages;
-constexpr int kBarBEmpty = kBarBFull + kBStages;
-constexpr int kBarAccFull = kBarBEmpty + kBStages;
+constexpr int kBarBFull = kBarAEmpty + kAStages;   // a weight piece has landed in buffer b
+constexpr int kBarBEmpty = kBarBFull + 2;          // the MMAs reading buffer b's previous piece are done
+constexpr int kBarAccFull = kBarBEmpty + 2;
 constexpr int kBarAccEmpty = kBarAccFull + 2;
 constexpr int kBarQFull = kBarAccEmpty + 2;
 constexpr int kBarQEmpty = kBarQFull + kQDepth;
@@ -70,7 +73,7 @@ constexpr int kOffTmem = kOffQItems + 4 * kQDepth;
 constexpr int kOffBroken = kOffTmem + 4;
 constexpr int kOffA = 1024;
 constexpr int kOffB = kOffA + kAStages * kAStageBytes;
-constexpr int kSmemUsed = kOffB + kBStages * kBStageBytes;
+constexpr int kSmemUsed = kOffB + 2 * kBPieceBytes;
 constexpr int kSmemBytes = kSmemUsed + 1024;  // slack for aligning the base
 static_assert(kNumBars * 8 <= kOffQItems, "barrier area");
 static_assert(kSmemBytes <= 232448, "shared memory");
@@ -192,6 +195,87 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Where one thread's epilogue results go: its pixel's element offset in the
+// output buffer (octet-planar: offset inside an 8-channel plane; NHWC: offset
+// of channel 0), the plane stride, and whether this lane stores at all.
+struct EpiDst {
+    __nv_bfloat16* out;
+    size_t pix, plane;
+    int nhwc, cout, pool;
+    bool store;
+};
+
+// Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1) of one
+// pixel per thread: folded BN, leaky ReLU 0.1, optional 2x2 max over the quad
+// lanes {l, l^1, l^8, l^9}, bf16 (nearest-even) and 16-byte stores per octet.
+template <int NC>
+__device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const float* bi, int ch0,
+                                          const EpiDst& d) {
+    uint32_t raw[NC];
+    if constexpr (NC == 32)
+        tmem_ld32(taddr, raw);
+    else
+        tmem_ld16(taddr, raw);
+    float v[NC];
+#pragma unroll
+    for (int i = 0; i < NC; i += 4) {
+        const float4 s4 = __ldg(reinterpret_cast<const float4*>(sc + i));
+        const float4 b4 = __ldg(reinterpret_cast<const float4*>(bi + i));
+        const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const float z = sv[u] * __uint_as_float(raw[i + u]) + bv[u];
+            v[i + u] = z > 0.f ? z : 0.1f * z;
+        }
+    }
+    if (d.pool) {
+#pragma unroll
+        for (int i = 0; i < NC; ++i) {
+            v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 1));
+            v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 8));
+        }
+    }
+    if (!d.store) return;
+#pragma unroll
+    for (int o = 0; o < NC / 8; ++o) {
+        const int ch = ch0 + 8 * o;
+        if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
+        uint4 w;
+        w.x = pack_bf16x2(v[8 * o + 0], v[8 * o + 1]);
+        w.y = pack_bf16x2(v[8 * o + 2], v[8 * o + 3]);
+        w.z = pack_bf16x2(v[8 * o + 4], v[8 * o + 5]);
+        w.w = pack_bf16x2(v[8 * o + 6], v[8 * o + 7]);
+        __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+        *reinterpret_cast<uint4*>(p) = w;
+    }
+}
+
+// Weight-buffer bookkeeping.  The producer and the MMA issuer each keep a copy and
+// apply the same transitions to the same item sequence, so they agree without
+// talking on which of the two buffers holds which weights.  A set that fits one
+// piece stays resident in its buffer (key >= 0) across items that use it; larger
+// sets stream through both buffers piece by piece.
+struct WeightBufs {
+    int key[2] = {-1, -1};     // resident set held by buffer b (-1: streamed piece or nothing)
+    uint32_t loads[2] = {0, 0};// pieces loaded into buffer b so far
+    int next = 0;              // buffer of the next load
+    bool held[2] = {false, false};  // MMA side: b holds a resident set that is not yet released
+    __device__ int resident(int k) const { return key[0] == k ? 0 : (key[1] == k ? 1 : -1); }
+};
+
 // Byte offset of tap t inside an A halo buffer.
 __device__ __forceinline__ uint32_t tap_off(int t, int k, int cols) {
     return (uint32_t)(((t / k) * cols + (t % k)) * 16);
@@ -216,7 +300,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(bar(kBarAFull + i), 1);
             mbar_init(bar(kBarAEmpty + i), 1);
         }
-        for (int i = 0; i < kBStages; ++i) {
+        for (int i = 0; i < 2; ++i) {
             mbar_init(bar(kBarBFull + i), 1);
             mbar_init(bar(kBarBEmpty + i), 1);
         }
@@ -247,10 +331,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ scheduler + TMA producer
         if (lane == 0) {
-            uint32_t a_cnt = 0, b_cnt = 0, q_cnt = 0;
+            uint32_t a_cnt = 0, q_cnt = 0;
+            WeightBufs wb;
+            // dependency counters already seen at (or above) a target: items of one task
+            // usually follow each other, so most items skip the round trip to L2
+            int ok_idx0 = -1, ok_idx1 = -1, ok_tgt0 = 0, ok_tgt1 = 0;
+            // the next ticket is taken one item ahead, hiding the atomic's latency
+            int next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
             while (true) {
-                int ticket = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
-                if (ticket >= p.n_items) ticket = -1;
+                const int ticket = next < p.n_items ? next : -1;
+                if (ticket >= 0) next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                if (ticket >= 0 && p.trace) {
+                    mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
+                    mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
+                }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
                 q_items[qs] = ticket;
@@ -260,6 +354,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const MafatItemDev it = p.items[ticket];
                 const MafatTaskDev tk = p.tasks[it.task];
                 const MafatStageDev st = p.stages[tk.stage];
+                const int key = tk.stage * 256 + it.nb;
+                const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
+                const uint32_t blob_bytes = (uint32_t)(st.blob_elems * 2);
+                const uint16_t* wset = p.w_bf16 + st.w_off + (size_t)it.nb * (size_t)(st.set_bytes / 2);
+                const bool resident = P == 1 && wb.resident(key) >= 0;
+                // Loads go out in the order the MMA issuer consumes them: piece 0, then for
+                // every chunk its A halo and the pieces that start inside it.
+                auto load_piece = [&](int pc) {
+                    const int b = wb.next;
+                    wb.next ^= 1;
+                    mbar_wait(bar(kBarBEmpty + b), (wb.loads[b] & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                    const int nblob = min(st.bpp, G - pc * st.bpp);
+                    const uint32_t bytes = (uint32_t)nblob * blob_bytes;
+                    mbar_arrive_expect_tx(bar(kBarBFull + b), bytes);
+                    bulk_load(sbase + kOffB + b * kBPieceBytes, wset + (size_t)pc * st.bpp * st.blob_elems, bytes,
+                              bar(kBarBFull + b));
+                    ++wb.loads[b];
+                    wb.key[b] = P == 1 ? key : -1;
+                };
+                if (!resident) load_piece(0);  // weights do not depend on other tiles: fetch first
                 const CUtensorMap* map = tk.in_kind == MAFAT_BUF_USER_IN ? &in_map
                                          : tk.in_kind == MAFAT_BUF_CUT   ? p.tmaps + p.cut_tmap
                                                                          : p.tmaps + tk.in_tmap;
@@ -267,10 +381,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int x0 = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * 8;
                 const int y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS - st.pad - tk.in_y0;
                 const uint32_t a_bytes = (uint32_t)(st.chunk8 * st.rows_box * st.cols_box * 16);
-                const uint32_t b_bytes = (uint32_t)(st.blob_elems * 2);
-                const uint16_t* wblob = p.w_bf16 + st.w_off +
-                                        (size_t)it.nb * st.n_chunks * st.n_bsteps * st.blob_elems;
-                mafat_dev::wait_item_deps(p.ctr, it, p.timeout_ns);
+                bool waited = false;
+                if (it.dep0 >= 0 && !(it.dep0 == ok_idx0 && it.dep0_target <= ok_tgt0)) {
+                    mafat_dev::wait_counter(p.ctr, it.dep0, it.dep0_target, p.timeout_ns);
+                    ok_idx0 = it.dep0;
+                    ok_tgt0 = it.dep0_target;
+                    waited = true;
+                }
+                if (it.dep1 >= 0 && !(it.dep1 == ok_idx1 && it.dep1_target <= ok_tgt1)) {
+                    mafat_dev::wait_counter(p.ctr, it.dep1, it.dep1_target, p.timeout_ns);
+                    ok_idx1 = it.dep1;
+                    ok_tgt1 = it.dep1_target;
+                    waited = true;
+                }
+                if (waited) mafat_dev::fence_proxy_async_global();
+                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
                     mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
@@ -278,32 +403,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_4d(sbase + kOffA + as * kAStageBytes, map, x0, y0, c * st.chunk8, c3,
                                 bar(kBarAFull + as));
                     ++a_cnt;
-                    for (int t = 0; t < st.n_bsteps; ++t) {
-                        const int bs = (int)(b_cnt % kBStages);
-                        mbar_wait(bar(kBarBEmpty + bs), ((b_cnt / kBStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
-                        mbar_arrive_expect_tx(bar(kBarBFull + bs), b_bytes);
-                        bulk_load(sbase + kOffB + bs * kBStageBytes,
-                                  wblob + ((size_t)c * st.n_bsteps + t) * st.blob_elems, b_bytes,
-                                  bar(kBarBFull + bs));
-                        ++b_cnt;
-                    }
+                    if (P > 1)
+                        for (int g = c * st.n_bsteps; g < (c + 1) * st.n_bsteps; ++g)
+                            if (g > 0 && g % st.bpp == 0) load_piece(g / st.bpp);
                 }
             }
-            // Drain: every copy issued into a stage has landed before the CTA may exit.
+            // Drain: every copy issued has landed before the CTA may exit.
             for (uint32_t i = 0; i < kAStages && i < a_cnt; ++i) {
                 uint32_t n = a_cnt - 1 - i;
                 mbar_wait(bar(kBarAFull + (int)(n % kAStages)), (n / kAStages) & 1u, p.ctr, pipe_limit, broken);
             }
-            for (uint32_t i = 0; i < kBStages && i < b_cnt; ++i) {
-                uint32_t n = b_cnt - 1 - i;
-                mbar_wait(bar(kBarBFull + (int)(n % kBStages)), (n / kBStages) & 1u, p.ctr, pipe_limit, broken);
-            }
+            for (int b = 0; b < 2; ++b)
+                if (wb.loads[b] > 0)
+                    mbar_wait(bar(kBarBFull + b), (wb.loads[b] - 1u) & 1u, p.ctr, pipe_limit, broken);
         }
         __syncwarp();
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            uint32_t a_cnt = 0, b_cnt = 0, q_cnt = 0, acc_cnt = 0;
+            uint32_t a_cnt = 0, q_cnt = 0, acc_cnt = 0;
+            WeightBufs wb;
             bool issued = false;
             while (true) {
                 const int qs = (int)(q_cnt % kQDepth);
@@ -315,6 +434,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const MafatItemDev it = p.items[ticket];
                 const MafatTaskDev tk = p.tasks[it.task];
                 const MafatStageDev st = p.stages[tk.stage];
+                const int key = tk.stage * 256 + it.nb;
+                const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
+                const uint32_t blob16 = (uint32_t)(st.blob_elems * 2) >> 4;
+                int cur_b = P == 1 ? wb.resident(key) : -1;
+                const bool resident = cur_b >= 0;
+                // Start consuming piece pc: release the buffer's previous resident set (its
+                // MMAs finish first), then wait for the piece.
+                auto begin_piece = [&]() {
+                    const int b = wb.next;
+                    wb.next ^= 1;
+                    if (wb.held[b]) {
+                        tc_commit(bar(kBarBEmpty + b));
+                        wb.held[b] = false;
+                    }
+                    mbar_wait(bar(kBarBFull + b), wb.loads[b] & 1u, p.ctr, pipe_limit, broken);
+                    ++wb.loads[b];
+                    wb.key[b] = P == 1 ? key : -1;
+                    wb.held[b] = P == 1;
+                    tc_fence_after();
+                    cur_b = b;
+                };
+                if (!resident) begin_piece();
                 const int buf = (int)(acc_cnt & 1u);
                 mbar_wait(bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
                 tc_fence_after();
@@ -323,45 +464,59 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t a_plane = (uint32_t)(st.rows_box * st.cols_box * 16);
                 const uint32_t a_row = (uint32_t)(st.cols_box * 16);
                 const uint32_t b_half = (uint32_t)(st.n_blk * 16);
+                const uint32_t blk16 = (uint32_t)(MAFAT_BLK_ROWS * st.cols_box);  // one block down, 16-B units
                 const int taps = st.k * st.k;
+                const int nbk = it.nbk;
                 uint32_t accumulate = 0;
+                int g = 0;  // blob index within the set
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
                     mbar_wait(bar(kBarAFull + as), (a_cnt / kAStages) & 1u, p.ctr, pipe_limit, broken);
+                    if (c == 0 && p.trace) mafat_dev::trace_put(p.trace, ticket, 6, mafat_dev::globaltimer_ns());
                     tc_fence_after();
                     const uint32_t a_base = sbase + kOffA + as * kAStageBytes;
-                    for (int t = 0; t < st.n_bsteps; ++t) {
-                        const int bs = (int)(b_cnt % kBStages);
-                        mbar_wait(bar(kBarBFull + bs), (b_cnt / kBStages) & 1u, p.ctr, pipe_limit, broken);
-                        tc_fence_after();
-                        const uint32_t b_base = sbase + kOffB + bs * kBStageBytes;
-                        for (int j = 0; j < st.kst; ++j) {
-                            uint32_t a_addr, a_k;
-                            if (st.paired) {
-                                int ta = 2 * t, tb = 2 * t + 1;
-                                if (tb >= taps) {
-                                    ta = taps - 2;
-                                    tb = taps - 1;
-                                }
-                                const uint32_t oa = tap_off(ta, st.k, st.cols_box);
-                                a_addr = a_base + oa;
-                                a_k = tap_off(tb, st.k, st.cols_box) - oa;
-                            } else {
-                                a_addr = a_base + (uint32_t)(2 * j) * a_plane + tap_off(t, st.k, st.cols_box);
-                                a_k = a_plane;
+                    // descriptors are advanced by adding 16-byte units to their start field
+                    const uint64_t a_desc0 = smem_desc(a_base, a_plane, a_row);
+                    int ky = 0, kx = 0;
+                    for (int t = 0; t < st.n_bsteps; ++t, ++g) {
+                        if (!resident && g > 0 && g % st.bpp == 0) begin_piece();
+                        const uint64_t b_desc =
+                            smem_desc(sbase + kOffB + cur_b * kBPieceBytes, b_half, 128u) + (uint64_t)((g % st.bpp) * blob16);
+                        if (st.paired) {
+                            int ta = 2 * t, tb = 2 * t + 1;
+                            if (tb >= taps) {
+                                ta = taps - 2;
+                                tb = taps - 1;
                             }
-                            const uint64_t adesc = smem_desc(a_addr, a_k, a_row);
-                            const uint64_t bdesc = smem_desc(b_base + (uint32_t)j * 2u * b_half, b_half, 128u);
-                            mma_bf16(d_tmem, adesc, bdesc, idesc, accumulate);
+                            const uint32_t oa = tap_off(ta, st.k, st.cols_box);
+                            const uint64_t ad = smem_desc(a_base + oa, tap_off(tb, st.k, st.cols_box) - oa, a_row);
+                            for (int b = 0; b < nbk; ++b)
+                                mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), ad + (uint64_t)(b * blk16), b_desc, idesc,
+                                         accumulate);
                             accumulate = 1;
-                            issued = true;
+                        } else {
+                            const uint64_t at = a_desc0 + (uint64_t)(ky * st.cols_box + kx);
+                            for (int j = 0; j < st.kst; ++j) {
+                                const uint64_t bd = b_desc + (uint64_t)(j * 2 * (b_half >> 4));
+                                const uint64_t aj = at + (uint64_t)(2 * j * (a_plane >> 4));
+                                for (int b = 0; b < nbk; ++b)
+                                    mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), aj + (uint64_t)(b * blk16), bd, idesc,
+                                             accumulate);
+                                accumulate = 1;
+                            }
+                            if (++kx == st.k) {
+                                kx = 0;
+                                ++ky;
+                            }
                         }
-                        tc_commit(bar(kBarBEmpty + bs));
-                        ++b_cnt;
+                        issued = true;
+                        // a streamed piece is released as soon as its last blob has been issued
+                        if (P > 1 && (g % st.bpp == st.bpp - 1 || g == G - 1)) tc_commit(bar(kBarBEmpty + cur_b));
                     }
                     tc_commit(bar(kBarAEmpty + as));
                     ++a_cnt;
                 }
+                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 7, mafat_dev::globaltimer_ns());
                 tc_commit(bar(kBarAccFull + buf));
                 ++acc_cnt;
             }
@@ -390,66 +545,43 @@ __global__ void __launch_bounds__(kThreads, 1)
             const MafatStageDev st = p.stages[tk.stage];
             const int buf = (int)(acc_cnt & 1u);
             mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken);
+            if (p.trace && threadIdx.x == 0) mafat_dev::trace_put(p.trace, ticket, 2, mafat_dev::globaltimer_ns());
             __syncwarp();
             tc_fence_after();
 
-            const int Y = tk.cy0 + it.by * MAFAT_BLK_ROWS + r;
-            const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
-            const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
-            bool store = valid;
-            int oy = Y, ox = X;
-            if (st.pool) {
-                store = valid && ((r & 1) == 0) && ((cc & 1) == 0);
-                oy = Y >> 1;
-                ox = X >> 1;
-            }
-            const int ly = oy - tk.out_y0, lx = ox - tk.out_x0;
             __nv_bfloat16* out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
                                                   : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
                                                                                     : p.scratch) +
                                  tk.out_off;
             const float* sc = p.scale + st.sb_off + it.nb * st.n_blk;
             const float* bi = p.bias + st.sb_off + it.nb * st.n_blk;
-            const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16) + (uint32_t)(buf * kAccStride);
-            for (int q = 0; q < st.n_blk / 16; ++q) {
-                uint32_t raw[16];
-                tmem_ld16(taddr + (uint32_t)(q * 16), raw);
-                float v[16];
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    float z = __ldg(sc + q * 16 + i) * __uint_as_float(raw[i]) + __ldg(bi + q * 16 + i);
-                    v[i] = z > 0.f ? z : 0.1f * z;
-                }
+            const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
+            for (int b = 0; b < it.nbk; ++b) {
+                const int Y = tk.cy0 + (it.by + b) * MAFAT_BLK_ROWS + r;
+                const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
+                bool store = valid;
+                int oy = Y, ox = X;
                 if (st.pool) {
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 1));
-                        v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 8));
-                    }
+                    store = valid && ((r & 1) == 0) && ((cc & 1) == 0);
+                    oy = Y >> 1;
+                    ox = X >> 1;
                 }
-                if (store) {
-                    const int ch0 = it.nb * st.n_blk + q * 16;
-                    uint4 lo, hi;
-                    lo.x = pack_bf16x2(v[0], v[1]);
-                    lo.y = pack_bf16x2(v[2], v[3]);
-                    lo.z = pack_bf16x2(v[4], v[5]);
-                    lo.w = pack_bf16x2(v[6], v[7]);
-                    hi.x = pack_bf16x2(v[8], v[9]);
-                    hi.y = pack_bf16x2(v[10], v[11]);
-                    hi.z = pack_bf16x2(v[12], v[13]);
-                    hi.w = pack_bf16x2(v[14], v[15]);
-                    // channels past cout belong to the zero-padded MMA N and are not stored
-                    const bool st_lo = ch0 < st.cout, st_hi = ch0 + 8 < st.cout;
-                    if (tk.out_nhwc) {
-                        uint4* dst = reinterpret_cast<uint4*>(out + ((size_t)ly * tk.out_w + lx) * st.cout + ch0);
-                        if (st_lo) dst[0] = lo;
-                        if (st_hi) dst[1] = hi;
-                    } else {
-                        const size_t plane = (size_t)tk.out_h * tk.out_w * 8;
-                        __nv_bfloat16* d0 = out + ((size_t)(ch0 >> 3) * tk.out_h + ly) * tk.out_w * 8 + (size_t)lx * 8;
-                        if (st_lo) *reinterpret_cast<uint4*>(d0) = lo;
-                        if (st_hi) *reinterpret_cast<uint4*>(d0 + plane) = hi;
-                    }
+                EpiDst dst;
+                dst.out = out;
+                dst.nhwc = tk.out_nhwc;
+                dst.pix = tk.out_nhwc ? ((size_t)(oy - tk.out_y0) * tk.out_w + (ox - tk.out_x0)) * st.cout
+                                      : ((size_t)(oy - tk.out_y0) * tk.out_w + (ox - tk.out_x0)) * 8;
+                dst.plane = (size_t)tk.out_h * tk.out_w * 8;
+                dst.cout = st.cout;
+                dst.store = store;
+                dst.pool = st.pool;
+                const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16) +
+                                       (uint32_t)(buf * kAccStride + b * st.n_blk);
+                const int ch_base = it.nb * st.n_blk;
+                if ((st.n_blk & 31) == 0) {
+                    for (int q = 0; q < st.n_blk; q += 32) epi_chunk<32>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
+                } else {
+                    for (int q = 0; q < st.n_blk; q += 16) epi_chunk<16>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
                 }
             }
             tc_fence_before();
@@ -458,7 +590,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mafat_dev::fence_proxy_async_global();
             __threadfence();
             asm volatile("bar.sync 1, 128;" ::: "memory");
-            if (threadIdx.x == 0) mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
+            if (threadIdx.x == 0) {
+                mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
+                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 3, mafat_dev::globaltimer_ns());
+            }
         }
     }
 

@@ -27,6 +27,7 @@ struct MafatKParams {
     int32_t n_ctr;                // words of the counter block
     int32_t pad2;
     int64_t timeout_ns;
+    unsigned long long* trace;    // per-item timestamps (null: off)
 };
 
 // bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.

@@ -159,13 +159,6 @@ struct TileInfo {
     std::vector<Rect> outs, ins;
 };
 
-// Largest even divisor of x that is <= 8 (x even).
-int chunk_octets(int x) {
-    for (int d = 8; d >= 2; d -= 2)
-        if (x % d == 0) return d;
-    return 2;
-}
-
 int largest_nblk(int cout) {
     for (int d = MAFAT_MAX_NBLK; d >= 16; d -= 16)
         if (cout % d == 0) return d;
@@ -193,7 +186,25 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         t.groups[1][1] = n - 1;
     }
 
+    // ---- tiles of every group (non-empty only)
+    std::vector<std::vector<TileInfo>> tiles(G);
+    int max_tiles = 1;
+    for (int g = 0; g < G; ++g) {
+        for (int i = 0; i < cfg.grid_n[g]; ++i)
+            for (int j = 0; j < cfg.grid_m[g]; ++j) {
+                TileInfo ti;
+                ti.i = i;
+                ti.j = j;
+                tile_regions(net, t.groups[g][0], t.groups[g][1], cfg.grid_n[g], cfg.grid_m[g], i, j,
+                             ti.outs, ti.ins);
+                if (ti.outs[t.groups[g][1]].empty()) continue;
+                tiles[g].push_back(std::move(ti));
+            }
+        max_tiles = std::max(max_tiles, (int)tiles[g].size());
+    }
+
     // ---- fused stages: a conv, plus the max-pool that directly follows it in the same group
+    const int n_ctas = cfg.n_ctas > 0 ? cfg.n_ctas : 152;
     std::vector<int> stage_pool_layer;
     for (int g = 0; g < G; ++g) {
         int first = t.groups[g][0], last = t.groups[g][1];
@@ -213,30 +224,79 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             s.cin8 = ceil_div(L.c_in, 8);
             s.cout = L.c_out;
             s.pool = (l + 1 <= last && net.layers[l + 1].type == L_MAXPOOL) ? 1 : 0;
-            // the MMA N must be a multiple of 16: pad with zero weights, store only cout channels
+            if (s.cin8 != 1 && s.cin8 % 2 != 0) {
+                *unsupported = true;
+                return "layer " + std::to_string(l) + ": input channels above 8 must be a multiple of 16";
+            }
+            // M blocks of this stage over all tiles and frames
+            int64_t blocks = 0;
+            for (const TileInfo& ti : tiles[g]) {
+                const Rect& cr = ti.outs[l];
+                blocks += (int64_t)ceil_div(cr.h(), MAFAT_BLK_ROWS) * ceil_div(cr.w(), MAFAT_BLK_COLS);
+            }
+            blocks *= cfg.batch;
+            // Output-channel block (MMA N): as wide as possible, narrowed while the stage
+            // would have fewer items than CTAs (short stages then spread over more SMs).
+            // The MMA N must be a multiple of 16: pad with zero weights, store only cout channels.
+            // Output-channel block (MMA N): as wide as possible (up to 256).  Narrower
+            // blocks would spread short stages over more SMs, but every item then streams
+            // the same activations and more weight pieces; measured, the widest block is
+            // fastest.  The MMA N must be a multiple of 16: pad with zero weights, store
+            // only cout channels.
             const int cout_pad = (L.c_out + 15) / 16 * 16;
-            s.n_blk = largest_nblk(cout_pad);
+            s.n_blk = cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0 ? cfg.fixed_nblk : largest_nblk(cout_pad);
             s.n_nblk = cout_pad / s.n_blk;
+            // Blocks per item (stacked along rows, one accumulator each, sharing every
+            // weight blob): grow while the stage keeps at least one item per CTA.
+            s.mb = 1;
+            if (cfg.fixed_mb > 0) {
+                s.mb = cfg.fixed_mb;
+            } else {
+                while (s.mb * 2 * s.n_blk <= 256 && blocks * s.n_nblk / (s.mb * 2) >= n_ctas) s.mb *= 2;
+            }
+            if (s.mb * s.n_blk > 256) s.mb = std::max(1, 256 / s.n_blk);
+            s.cols_box = MAFAT_BLK_COLS + L.k - 1;
+            // input octets per A chunk: the largest that fits the A stage with mb blocks
+            for (;;) {
+                s.rows_box = MAFAT_BLK_ROWS * s.mb + L.k - 1;
+                const int row_bytes = s.cols_box * 16 * s.rows_box;
+                if (s.cin8 == 1) {
+                    s.chunk8 = 1;
+                } else {
+                    s.chunk8 = 0;
+                    for (int d = 8; d >= 2; d -= 2)
+                        if (s.cin8 % d == 0 && d * row_bytes <= MAFAT_A_STAGE_BYTES) {
+                            s.chunk8 = d;
+                            break;
+                        }
+                }
+                if ((s.chunk8 > 0 && s.chunk8 * row_bytes <= MAFAT_A_STAGE_BYTES) || s.mb == 1) break;
+                s.mb /= 2;
+            }
+            if (s.chunk8 == 0) return "internal: no A chunk fits the shared-memory stage";
             if (s.cin8 == 1) {
                 s.paired = 1;
-                s.chunk8 = 1;
                 s.n_chunks = 1;
                 s.n_bsteps = ceil_div(L.k * L.k, 2);
                 s.kst = 1;
             } else {
-                if (s.cin8 % 2 != 0) {
-                    *unsupported = true;
-                    return "layer " + std::to_string(l) + ": input channels above 8 must be a multiple of 16";
-                }
                 s.paired = 0;
-                s.chunk8 = chunk_octets(s.cin8);
                 s.n_chunks = s.cin8 / s.chunk8;
                 s.n_bsteps = L.k * L.k;
                 s.kst = s.chunk8 / 2;
             }
-            s.rows_box = MAFAT_BLK_ROWS + L.k - 1;
-            s.cols_box = MAFAT_BLK_COLS + L.k - 1;
             s.blob_elems = s.n_blk * 16 * s.kst;
+            s.set_bytes = s.n_chunks * s.n_bsteps * s.blob_elems * 2;
+            // Weights travel in pieces of whole blobs that fill one shared-memory buffer:
+            // a set that fits one piece stays resident across items, larger sets stream
+            // through the two buffers (every copy has a fixed cost, so pieces are large).
+            s.bpp = std::max(1, MAFAT_B_PIECE_BYTES / (s.blob_elems * 2));
+            s.bpp = std::min(s.bpp, s.n_chunks * s.n_bsteps);
+            s.n_pieces = ceil_div(s.n_chunks * s.n_bsteps, s.bpp);
+            if (s.blob_elems * 2 > MAFAT_B_PIECE_BYTES) {
+                *unsupported = true;
+                return "layer " + std::to_string(l) + ": one weight blob exceeds a shared-memory buffer";
+            }
             s.w_off = t.weight_elems;
             t.weight_elems += (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems;
             s.w32_off = t.weight32_elems;
@@ -275,22 +335,6 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     const int64_t cut_frame = (int64_t)t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_frame = (int64_t)t.out_h * t.out_w * t.out_c;
 
-    // ---- tiles of every group (non-empty only)
-    std::vector<std::vector<TileInfo>> tiles(G);
-    int max_tiles = 1;
-    for (int g = 0; g < G; ++g) {
-        for (int i = 0; i < cfg.grid_n[g]; ++i)
-            for (int j = 0; j < cfg.grid_m[g]; ++j) {
-                TileInfo ti;
-                ti.i = i;
-                ti.j = j;
-                tile_regions(net, t.groups[g][0], t.groups[g][1], cfg.grid_n[g], cfg.grid_m[g], i, j,
-                             ti.outs, ti.ins);
-                if (ti.outs[t.groups[g][1]].empty()) continue;
-                tiles[g].push_back(std::move(ti));
-            }
-        max_tiles = std::max(max_tiles, (int)tiles[g].size());
-    }
     int S = cfg.ring_slots > 0 ? cfg.ring_slots : std::min(max_tiles, 64);
     int W = cfg.wave_tiles > 0 ? std::min(cfg.wave_tiles, S) : S;
     t.ring_slots = S;
@@ -405,7 +449,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             tk.out_y0 = orr.y0;
                             tk.out_x0 = orr.x0;
                         }
-                        tk.n_items = tk.nby * tk.nbx * st.n_nblk;
+                        tk.n_items = ceil_div(tk.nby, st.mb) * tk.nbx * st.n_nblk;
                         TaskDep d;
                         int qi = (int)(q - w0);
                         if (s == t.stage_first[g]) {
@@ -446,12 +490,14 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         const MafatTaskDev& tk = t.tasks[ti];
         const MafatStageDev& st = t.stages[tk.stage];
         const TaskDep& d = deps[ti];
-        for (int by = 0; by < tk.nby; ++by)
-            for (int bx = 0; bx < tk.nbx; ++bx)
-                for (int nb = 0; nb < st.n_nblk; ++nb) {
+        // channel-block major: consecutive items share a resident weight set
+        for (int nb = 0; nb < st.n_nblk; ++nb)
+            for (int by = 0; by < tk.nby; by += st.mb)
+                for (int bx = 0; bx < tk.nbx; ++bx) {
                     MafatItemDev it{};
                     it.task = ti;
                     it.by = (int16_t)by;
+                    it.nbk = (int16_t)std::min(st.mb, tk.nby - by);
                     it.bx = (int16_t)bx;
                     it.nb = (int16_t)nb;
                     it.flags = (ti == cfg.unpublished_task) ? 1 : 0;
@@ -500,10 +546,15 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     };
     for (const MafatStageDev& s : t.stages) {
         if ((int64_t)s.chunk8 * s.rows_box * s.cols_box * 16 > MAFAT_A_STAGE_BYTES) return "A box exceeds its stage";
-        if ((int64_t)s.blob_elems * 2 > MAFAT_B_STAGE_BYTES) return "weight blob exceeds its stage";
+        if (s.set_bytes != s.n_chunks * s.n_bsteps * s.blob_elems * 2 || s.set_bytes % 16 != 0)
+            return "bad weight set size";
+        if (s.bpp < 1 || (int64_t)s.bpp * s.blob_elems * 2 > MAFAT_B_PIECE_BYTES) return "weight piece exceeds its buffer";
+        if (s.n_pieces != ceil_div(s.n_chunks * s.n_bsteps, s.bpp)) return "bad weight piece count";
         if (s.cols_box * 8 > 256 || s.rows_box > 256 || s.chunk8 > 256) return "TMA box dimension above 256";
         if ((s.cols_box * 16) % 16 != 0) return "TMA inner box not a multiple of 16 bytes";
         if (s.n_blk % 16 != 0 || s.n_blk < 16 || s.n_blk > MAFAT_MAX_NBLK) return "bad MMA N";
+        if (s.mb < 1 || s.mb * s.n_blk > 256) return "blocks of an item exceed one TMEM accumulator buffer";
+        if (s.rows_box != MAFAT_BLK_ROWS * s.mb + s.k - 1) return "A box rows do not cover the item";
         if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
             return "weight blobs outside the packed weights";
         if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
@@ -552,6 +603,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         const MafatStageDev& s = t.stages[k.stage];
         if (it.by >= k.nby || it.bx >= k.nbx || it.nb >= s.n_nblk || it.by < 0 || it.bx < 0 || it.nb < 0)
             return "item block out of range";
+        if (it.nbk < 1 || it.nbk > s.mb || it.by + it.nbk > k.nby) return "item block count out of range";
         const int deps[2] = {it.dep0, it.dep1};
         const int tgts[2] = {it.dep0_target, it.dep1_target};
         for (int d = 0; d < 2; ++d) {

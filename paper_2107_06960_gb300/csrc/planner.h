@@ -65,6 +65,9 @@ struct PlanConfig {
     int ring_slots = 0;
     int wave_tiles = 0;
     int unpublished_task = -1;
+    int n_ctas = 0;           // persistent CTAs (shapes items; 0: 152)
+    int fixed_nblk = 0;       // force the output-channel block of every stage (0: choose)
+    int fixed_mb = 0;         // force blocks per item (0: choose)
 };
 
 // A tensor-map request for a task whose input is a scratch region buffer.

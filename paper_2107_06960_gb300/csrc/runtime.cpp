@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdint>
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -39,6 +40,7 @@ struct mafat_plan_s {
     void* d_cut = nullptr;
     void* d_scratch = nullptr;
     uint32_t* d_ctr = nullptr;
+    unsigned long long* d_trace = nullptr;
     size_t ctr_bytes = 0;
     int64_t weight_bytes = 0, scratch_bytes = 0;
     size_t in_bytes = 0, out_bytes = 0, cut_bytes = 0;
@@ -152,6 +154,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
     kp.ctr = p->d_ctr;
     kp.n_ctr = (int32_t)(p->ctr_bytes / sizeof(uint32_t));
     kp.timeout_ns = p->timeout_ns;
+    kp.trace = p->d_trace;
     if (p->dtype == MAFAT_BF16) {
         if (p->in_map_ptr != input) {
             std::string err;
@@ -282,6 +285,15 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.ring_slots = o.ring_slots;
     cfg.wave_tiles = o.wave_tiles;
     cfg.unpublished_task = o.test_unpublished_task;
+    cfg.fixed_nblk = o.force_nblk;
+    cfg.fixed_mb = o.force_mb;
+    int sms = 0;
+    if (!o.dry_run) {
+        int dev = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    if (sms <= 0) sms = 152;
+    cfg.n_ctas = o.max_ctas > 0 ? o.max_ctas : sms;
 
     mafat_plan_s* p = new (std::nothrow) mafat_plan_s();
     if (!p) return fail(MAFAT_ENOMEM, "host allocation failed");
@@ -317,7 +329,6 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
         delete p;
         return cuda_fail(e, "cudaGetDevice");
     }
-    int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
     // tensor-core kernel: one CTA per SM (shared memory and TMEM); check kernel: 8 small CTAs per SM
     p->grid = o.max_ctas > 0 ? o.max_ctas : (dt == MAFAT_BF16 ? sms : 8 * sms);
@@ -357,6 +368,9 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     if ((e = cudaMemcpy(p->d_items, t.items.data(), t.items.size() * sizeof(MafatItemDev), cudaMemcpyHostToDevice)) != cudaSuccess) return bail(e, "cudaMemcpy");
     if ((e = cudaMemset(p->d_scratch, 0, (size_t)p->scratch_bytes)) != cudaSuccess) return bail(e, "cudaMemset");
     if ((e = cudaMemset(p->d_ctr, 0, p->ctr_bytes)) != cudaSuccess) return bail(e, "cudaMemset");
+    if (o.trace &&
+        (e = dalloc(p, &p->d_trace, t.items.size() * MAFAT_TRACE_WORDS * sizeof(unsigned long long))) != cudaSuccess)
+        return bail(e, "cudaMalloc");
 
     if (dt == MAFAT_BF16) {
         // one map per scratch-input task, then the cut tensor map
@@ -543,6 +557,23 @@ mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* ou
 }
 
 int32_t mafat_launches_per_run(const mafat_plan_t* plan) { return plan ? 1 : 0; }
+
+mafat_status mafat_plan_trace(const mafat_plan_t* plan, uint64_t* out, int64_t max_words, void* stream) {
+    if (!plan || !out) return fail(MAFAT_EINVAL, "null argument");
+    if (!plan->d_trace) return fail(MAFAT_EINVAL, "plan was not created with options.trace = 1");
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int64_t words = std::min<int64_t>(max_words, (int64_t)plan->t.items.size() * MAFAT_TRACE_WORDS);
+    if (words <= 0) return MAFAT_OK;
+    e = cudaMemcpy(out, plan->d_trace, (size_t)words * sizeof(uint64_t), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+    for (int64_t i = 0; (i + 1) * MAFAT_TRACE_WORDS <= words; ++i) {
+        const MafatItemDev& it = plan->t.items[(size_t)i];
+        const int layer = plan->t.stages[plan->t.tasks[it.task].stage].layer;
+        out[i * MAFAT_TRACE_WORDS + 5] = ((uint64_t)it.task << 16) | (uint64_t)layer;
+    }
+    return MAFAT_OK;
+}
 
 void mafat_plan_destroy(mafat_plan_t* plan) {
     if (!plan) return;

@@ -9,6 +9,7 @@
 // MAFAT_DEV_TIMEOUT, raises the abort word and every later wait returns at
 // once, so the launch always ends.
 #pragma once
+#include "../../include/mafat.h"
 #include "kernels.h"
 
 namespace mafat_dev {
@@ -76,6 +77,17 @@ __device__ __forceinline__ void publish_item(uint32_t* ctr, const MafatItemDev& 
     __threadfence();
     red_release_add(ctr + done_ctr, 1u);
     if (it.extra_ctr >= 0) red_release_add(ctr + it.extra_ctr, 1u);
+}
+
+__device__ __forceinline__ uint32_t smid() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
+
+// Trace record of an item: {ticket taken, deps satisfied, accumulator ready, published, SM}.
+__device__ __forceinline__ void trace_put(unsigned long long* tr, int ticket, int field, uint64_t v) {
+    if (tr) tr[(size_t)ticket * MAFAT_TRACE_WORDS + field] = v;
 }
 
 // Called by every thread of a CTA after its last use of the counters: the last

@@ -166,8 +166,10 @@ def test_bf16_1216_batch8_stress(mf):
 
 
 def test_bf16_608_plan_sweep_is_plan_independent(mf):
-    # cut after layer 1, 3, 7, 11 x per-group grids 1..5 (100 plans): all bit-identical,
-    # and equal to the oracle within tolerance.
+    # cut after layer 1, 3, 7, 11 x per-group grids 1..5 (100 plans).  With the MMA
+    # shapes held fixed (32 output channels x one 16x8 block per item) every plan
+    # must give bit-identical outputs -- tiling changes only which tile computes a
+    # pixel, never how -- and equal the oracle within tolerance.
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     layers, params, x = wl["layers"], wl["params"], wl["input"]
     refs = _oracle_groups(layers, params, x, 8, "yolo16_608_5x5_c8_2x2")
@@ -175,11 +177,22 @@ def test_bf16_608_plan_sweep_is_plan_independent(mf):
     for cut in synth.SWEEP_CUTS:
         for t1 in synth.SWEEP_GRIDS:
             for t2 in synth.SWEEP_GRIDS:
-                c, out = run_plan(mf, layers, params, x, cut, [(t1, t1), (t2, t2)], mf.BF16)
+                c, out = run_plan(mf, layers, params, x, cut, [(t1, t1), (t2, t2)], mf.BF16,
+                                  plan_kwargs=dict(force_nblk=32, force_mb=1))
                 if base is None:
                     base = out
                     assert rel_err(out[0], refs[0][-1]) <= TOL_BF16
                 assert np.array_equal(out, base), "plan %d/%dx%d/%dx%d differs" % (cut, t1, t1, t2, t2)
+
+
+@pytest.mark.parametrize("cut,t1,t2", [(2, 1, 2), (4, 3, 3), (8, 5, 2), (8, 2, 5), (12, 4, 1), (12, 5, 5)])
+def test_bf16_608_sweep_default_shapes(mf, cut, t1, t2):
+    # the default per-stage MMA shapes depend on the plan; results stay within tolerance
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    layers, params, x = wl["layers"], wl["params"], wl["input"]
+    refs = _oracle_groups(layers, params, x, 8, "yolo16_608_5x5_c8_2x2")
+    _, out = run_plan(mf, layers, params, x, cut, [(t1, t1), (t2, t2)], mf.BF16)
+    assert rel_err(out[0], refs[0][-1]) <= TOL_BF16
 
 
 # ---------------------------------------------------------------------------
