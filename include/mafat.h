@@ -217,9 +217,10 @@ mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* ou
  * its dependencies were satisfied, when its accumulator was ready for the
  * epilogue, when its completion was published, SM id, task index << 16 |
  * network layer of its convolution, when its first input halo had landed in
- * shared memory, when its last MMA was issued}.  max_words bounds what is
- * written. */
-#define MAFAT_TRACE_WORDS 8
+ * shared memory, when its last MMA was issued, ns the MMA issuer waited for
+ * later input halos, ns it waited for streamed weight pieces}.  max_words
+ * bounds what is written. */
+#define MAFAT_TRACE_WORDS 10
 mafat_status mafat_plan_trace(const mafat_plan_t* plan, uint64_t* out, int64_t max_words, void* stream);
 
 /* Number of kernel launches one mafat_run makes. */

@@ -251,11 +251,12 @@ class Plan:
 
     def trace(self, stream=None):
         """Per-item records of the last run (plan made with trace=True): numpy uint64
-        [n_items][8] = ticket taken, deps satisfied, accumulator ready, published (ns), SM,
-        task << 16 | layer, first halo landed, last MMA issued (ns)."""
+        [n_items][10] = ticket taken, deps satisfied, accumulator ready, published (ns), SM,
+        task << 16 | layer, first halo landed, last MMA issued (ns), ns waited for later
+        halos, ns waited for streamed weight pieces."""
         import numpy as np
         n = self.stats()["n_items"]
-        out = np.zeros((n, 8), dtype=np.uint64)
+        out = np.zeros((n, 10), dtype=np.uint64)
         _check(lib.mafat_plan_trace(self.handle, out.ctypes.data, out.size, _stream(stream)))
         return out
 

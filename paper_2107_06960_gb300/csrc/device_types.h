@@ -43,6 +43,7 @@ struct MafatStageDev {
     int32_t paired;       // 1: cin8 == 1, two taps share one K=16 step
     int32_t n_bsteps;     // weight blobs per chunk (taps, or tap pairs)
     int32_t kst;          // K=16 MMA steps per blob
+    int32_t b_swz;        // 1: blobs in the 128-byte swizzled K-major layout (kst == 4), 0: no swizzle
     int32_t mb;           // M blocks per item (stacked along rows, one TMEM accumulator each)
     int32_t rows_box, cols_box;  // A halo box (pixels): 16*mb + k - 1 rows, 8 + k - 1 columns
     int64_t w_off;        // element offset of this stage's packed bf16 weights

@@ -2,8 +2,9 @@
 // (MAFAT, Sec. 3-4) on sm_103a: tcgen05 MMA with TMEM accumulators, operands
 // staged in shared memory by TMA, one persistent launch per plan.
 //
-// One work item = one 16 x 8 block of a tile's conv output (M = 128 pixels)
-// times one block of n_blk <= 256 output channels, i.e. an implicit GEMM
+// One work item = up to 8 vertically stacked 16 x 8 blocks of a tile's conv
+// output (M = 128 pixels each, one accumulator each) times one block of n_blk
+// <= 256 output channels, i.e. an implicit GEMM
 //   D[m][n] = sum_{c, ky, kx} A[pixel m shifted by (ky, kx)][c] * W[n][c][ky][kx]
 // (M = 128, N = n_blk, K = k*k*Cin) accumulated in fp32 in tensor memory.
 //
@@ -19,18 +20,20 @@
 //    With 8 input channels (the first layer), one K=16 step covers two taps:
 //    its two K core matrices sit at the two taps' offsets (LBO = their
 //    distance).
-//  * B: weights pre-packed on the host in exactly the shared-memory image of the
-//    whole weight set of one (stage, output-channel block), fetched with one bulk
-//    copy and kept resident while the CTA's consecutive items use the same set
-//    (every copy costs a few hundred cycles of TMA time however small it is, so
-//    the per-item copies are only the A halo boxes).
+//  * B: weights pre-packed on the host in exactly their shared-memory image, as
+//    blobs of one (chunk, tap); blobs with 64 channels use the 128-byte swizzled
+//    K-major layout, narrower ones the no-swizzle one.  The weights of one (stage,
+//    output-channel block) travel in pieces filling one of two 74 KB buffers: a
+//    set that fits one piece stays resident while the CTA's consecutive items use
+//    it, larger sets stream piece by piece (every copy costs a few hundred cycles
+//    of TMA time however small it is, so copies are large and few).
 //
-// Warp roles (192 threads): warps 0-3 epilogue (warp w reads TMEM lanes
-// 32w..32w+31 = conv rows 4w..4w+3 of the block), warp 4 scheduler + TMA
-// producer, warp 5 TMEM allocator + MMA issuer.  Shared memory: 2 A halo stages,
-// one resident weight set, and a 4-deep queue of item indices; TMEM: 2
-// accumulators of 256 columns (the epilogue of one item overlaps the MMAs of
-// the next).
+// Warp roles (320 threads): warps 0-7 epilogue (warp w reads TMEM lanes
+// 32(w%4)..+31 = conv rows 4(w%4)..+3 of a block; the two warpgroups split an
+// item's blocks or columns), warp 8 scheduler + TMA producer, warp 9 TMEM
+// allocator + MMA issuer.  Shared memory: 2 A halo stages, 2 weight buffers and
+// a 4-deep queue of item indices; TMEM: 2 accumulators of 256 columns (the
+// epilogue of one item overlaps the MMAs of the next).
 //
 // Epilogue: y = leaky_0.1(scale[n] * acc + bias[n]); for a fused 2x2/s2
 // max-pool the quad of pixels {(r, c), (r, c+1), (r+1, c), (r+1, c+1)} are lanes
@@ -47,9 +50,11 @@
 
 namespace {
 
-constexpr int kThreads = 192;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
+constexpr int kEpiWarps = 8;            // two warpgroups over the 128 TMEM lanes
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kProducerWarp = kEpiWarps;
+constexpr int kMmaWarp = kEpiWarps + 1;
+constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kAStages = 2;
 constexpr int kQDepth = 4;
 constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;   // one A halo box, multiple of 1024
@@ -112,11 +117,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // after which every pipeline wait of the CTA gives up after 1 ms, so the launch
 // still ends in bounded time (with garbage results and an error status).
 __device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, uint32_t* ctr, int64_t limit_ns,
-                                          volatile int* broken) {
+                                          volatile int* broken, uint32_t sleep_ns = 0) {
     if (mbar_try_wait(bar, parity)) return;
     const int64_t lim = *broken ? 1000000LL : limit_ns;
     uint64_t t0 = mafat_dev::globaltimer_ns();
     for (uint32_t i = 1;; ++i) {
+        // warps whose waits are off the critical path back off, leaving issue slots of
+        // their sub-partition to the MMA issuer
+        if (sleep_ns) __nanosleep(sleep_ns);
         if (mbar_try_wait(bar, parity)) return;
         if ((i & 255u) == 0u && (int64_t)(mafat_dev::globaltimer_ns() - t0) > lim) {
             mafat_dev::record_status(ctr, MAFAT_DEV_PIPE);
@@ -169,14 +177,62 @@ __device__ __forceinline__ uint32_t instr_desc_bf16(int n, int m) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
+// No "memory" clobber: the MMA reads shared memory through its descriptors and
+// writes tensor memory only, and volatile asm statements keep their order.
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                          uint32_t accumulate) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+// The MMA issuer is one thread whose dependent instruction chain sets its issue
+// rate, so the hot loop keeps descriptors as 32-bit halves: the low word holds
+// start address >> 4 (bits 0-13) and LBO >> 4 (bits 16-29), and advancing an
+// operand only adds 16-byte units to it; the high word (SBO, version, swizzle
+// mode) is fixed per operand.
+__device__ __forceinline__ void mma_lo(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo, uint32_t b_hi,
+                                       uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+        "setp.ne.b32 p, %6, 0;\n\t"
+        "mov.b64 da, {%1, %2};\n\t"
+        "mov.b64 db, {%3, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %5, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
+}
+
+// One weight blob of a regular stage: KST K=16 steps x nbk blocks (blocks share the
+// B operand, so consecutive MMAs of a K step re-read it).
+template <int KST>
+__device__ __forceinline__ void issue_blob(uint32_t d_tmem, uint32_t n_blk, int nbk, uint32_t a_lo, uint32_t a_hi,
+                                           uint32_t a_step, uint32_t a_blk, uint32_t b_lo, uint32_t b_hi,
+                                           uint32_t b_step, uint32_t idesc, uint32_t& accumulate) {
+#pragma unroll
+    for (int j = 0; j < KST; ++j) {
+        uint32_t d = d_tmem, a = a_lo + (uint32_t)j * a_step;
+        const uint32_t b = b_lo + (uint32_t)j * b_step;
+        for (int blk = 0; blk < nbk; ++blk) {
+            mma_lo(d, a, a_hi, b, b_hi, idesc, accumulate);
+            d += n_blk;
+            a += a_blk;
+        }
+        accumulate = 1;
+    }
+}
+
+// 128-byte-swizzled, K-major B operand (weights packed so by the host): rows of
+// 64 channels (128 bytes), 8-row atoms of 1024 bytes, SBO = 1024, one K=16 step =
+// 32 bytes along the row.  Measured on GB300: when both operands change from one
+// MMA to the next, no-swizzle operands cost ~2.4x the MMA time; with B swizzled
+// the MMAs run at their own rate.
+__device__ __forceinline__ uint32_t desc_hi_sw128(uint32_t sbo) {
+    return ((sbo >> 4) & 0x3FFFu) | (1u << 14) | (2u << 29);
+}
+__device__ __forceinline__ uint32_t desc_lo_sw128(uint32_t addr) {
+    return ((addr & 0x3FFFFu) >> 4) | (1u << 16);
 }
 
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
@@ -208,6 +264,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&v)[64]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, "
+        "%36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, "
+        "%57, %58, %59, %60, %61, %62, %63}, [%64];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31]),
+          "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]), "=r"(v[37]), "=r"(v[38]), "=r"(v[39]),
+          "=r"(v[40]), "=r"(v[41]), "=r"(v[42]), "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]),
+          "=r"(v[48]), "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]), "=r"(v[55]),
+          "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]), "=r"(v[61]), "=r"(v[62]), "=r"(v[63])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
 // Where one thread's epilogue results go: its pixel's element offset in the
 // output buffer (octet-planar: offset inside an 8-channel plane; NHWC: offset
 // of channel 0), the plane stride, and whether this lane stores at all.
@@ -225,7 +300,9 @@ template <int NC>
 __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const float* bi, int ch0,
                                           const EpiDst& d) {
     uint32_t raw[NC];
-    if constexpr (NC == 32)
+    if constexpr (NC == 64)
+        tmem_ld64(taddr, raw);
+    else if constexpr (NC == 32)
         tmem_ld32(taddr, raw);
     else
         tmem_ld16(taddr, raw);
@@ -269,11 +346,32 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
 // piece stays resident in its buffer (key >= 0) across items that use it; larger
 // sets stream through both buffers piece by piece.
 struct WeightBufs {
-    int key[2] = {-1, -1};     // resident set held by buffer b (-1: streamed piece or nothing)
-    uint32_t loads[2] = {0, 0};// pieces loaded into buffer b so far
-    int next = 0;              // buffer of the next load
-    bool held[2] = {false, false};  // MMA side: b holds a resident set that is not yet released
-    __device__ int resident(int k) const { return key[0] == k ? 0 : (key[1] == k ? 1 : -1); }
+    // two buffers as scalar fields: a runtime-indexed local array would live in
+    // local memory, next to the MMA issue loop
+    int key0 = -1, key1 = -1;        // resident set held by buffer b (-1: streamed piece or nothing)
+    uint32_t loads0 = 0, loads1 = 0; // pieces loaded into buffer b so far
+    int next = 0;                    // buffer of the next load
+    bool held0 = false, held1 = false;  // MMA side: b holds a resident set that is not yet released
+    __device__ __forceinline__ int resident(int k) const { return key0 == k ? 0 : (key1 == k ? 1 : -1); }
+    __device__ __forceinline__ uint32_t loads(int b) const { return b ? loads1 : loads0; }
+    __device__ __forceinline__ bool held(int b) const { return b ? held1 : held0; }
+    __device__ __forceinline__ void set_loaded(int b, int k, bool hold) {
+        if (b) {
+            ++loads1;
+            key1 = k;
+            held1 = hold;
+        } else {
+            ++loads0;
+            key0 = k;
+            held0 = hold;
+        }
+    }
+    __device__ __forceinline__ void release(int b) {
+        if (b)
+            held1 = false;
+        else
+            held0 = false;
+    }
 };
 
 // Byte offset of tap t inside an A halo buffer.
@@ -306,11 +404,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(kBarAccFull + i), 1);
-            mbar_init(bar(kBarAccEmpty + i), 128);
+            mbar_init(bar(kBarAccEmpty + i), kEpiThreads);
         }
         for (int i = 0; i < kQDepth; ++i) {
             mbar_init(bar(kBarQFull + i), 1);
-            mbar_init(bar(kBarQEmpty + i), 5);
+            mbar_init(bar(kBarQEmpty + i), kEpiWarps + 1);
         }
         mbar_init(bar(kBarDone), 1);
         *broken = 0;
@@ -346,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
                 }
                 const int qs = (int)(q_cnt % kQDepth);
-                mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                 q_items[qs] = ticket;
                 mbar_arrive(bar(kBarQFull + qs));
                 ++q_cnt;
@@ -360,20 +458,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint16_t* wset = p.w_bf16 + st.w_off + (size_t)it.nb * (size_t)(st.set_bytes / 2);
                 const bool resident = P == 1 && wb.resident(key) >= 0;
                 // Loads go out in the order the MMA issuer consumes them: piece 0, then for
-                // every chunk its A halo and the pieces that start inside it.
-                auto load_piece = [&](int pc) {
-                    const int b = wb.next;
-                    wb.next ^= 1;
-                    mbar_wait(bar(kBarBEmpty + b), (wb.loads[b] & 1u) ^ 1u, p.ctr, pipe_limit, broken);
-                    const int nblob = min(st.bpp, G - pc * st.bpp);
-                    const uint32_t bytes = (uint32_t)nblob * blob_bytes;
-                    mbar_arrive_expect_tx(bar(kBarBFull + b), bytes);
-                    bulk_load(sbase + kOffB + b * kBPieceBytes, wset + (size_t)pc * st.bpp * st.blob_elems, bytes,
-                              bar(kBarBFull + b));
-                    ++wb.loads[b];
-                    wb.key[b] = P == 1 ? key : -1;
-                };
-                if (!resident) load_piece(0);  // weights do not depend on other tiles: fetch first
+                // every chunk its A halo and the pieces that start inside it.  A piece goes
+                // into the next buffer once the buffer's previous contents are released.
+#define MAFAT_LOAD_PIECE(pc)                                                                                   \
+    do {                                                                                                      \
+        const int b_ = wb.next;                                                                               \
+        wb.next ^= 1;                                                                                         \
+        mbar_wait(bar(kBarBEmpty + b_), (wb.loads(b_) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);             \
+        const int nblob_ = min(st.bpp, G - (pc) * st.bpp);                                                    \
+        const uint32_t bytes_ = (uint32_t)nblob_ * blob_bytes;                                                \
+        mbar_arrive_expect_tx(bar(kBarBFull + b_), bytes_);                                                   \
+        bulk_load(sbase + kOffB + b_ * kBPieceBytes, wset + (size_t)(pc) * st.bpp * st.blob_elems, bytes_,    \
+                  bar(kBarBFull + b_));                                                                        \
+        wb.set_loaded(b_, P == 1 ? key : -1, false);                                                          \
+    } while (0)
+                if (!resident) MAFAT_LOAD_PIECE(0);  // weights do not depend on other tiles: fetch first
                 const CUtensorMap* map = tk.in_kind == MAFAT_BUF_USER_IN ? &in_map
                                          : tk.in_kind == MAFAT_BUF_CUT   ? p.tmaps + p.cut_tmap
                                                                          : p.tmaps + tk.in_tmap;
@@ -398,15 +497,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
-                    mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                    mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                     mbar_arrive_expect_tx(bar(kBarAFull + as), a_bytes);
                     tma_load_4d(sbase + kOffA + as * kAStageBytes, map, x0, y0, c * st.chunk8, c3,
                                 bar(kBarAFull + as));
                     ++a_cnt;
                     if (P > 1)
                         for (int g = c * st.n_bsteps; g < (c + 1) * st.n_bsteps; ++g)
-                            if (g > 0 && g % st.bpp == 0) load_piece(g / st.bpp);
+                            if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
                 }
+#undef MAFAT_LOAD_PIECE
             }
             // Drain: every copy issued has landed before the CTA may exit.
             for (uint32_t i = 0; i < kAStages && i < a_cnt; ++i) {
@@ -414,8 +514,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait(bar(kBarAFull + (int)(n % kAStages)), (n / kAStages) & 1u, p.ctr, pipe_limit, broken);
             }
             for (int b = 0; b < 2; ++b)
-                if (wb.loads[b] > 0)
-                    mbar_wait(bar(kBarBFull + b), (wb.loads[b] - 1u) & 1u, p.ctr, pipe_limit, broken);
+                if (wb.loads(b) > 0)
+                    mbar_wait(bar(kBarBFull + b), (wb.loads(b) - 1u) & 1u, p.ctr, pipe_limit, broken);
         }
         __syncwarp();
     } else if (warp == kMmaWarp) {
@@ -436,26 +536,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const MafatStageDev st = p.stages[tk.stage];
                 const int key = tk.stage * 256 + it.nb;
                 const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
-                const uint32_t blob16 = (uint32_t)(st.blob_elems * 2) >> 4;
+                const uint32_t blob_bytes = (uint32_t)(st.blob_elems * 2);
                 int cur_b = P == 1 ? wb.resident(key) : -1;
                 const bool resident = cur_b >= 0;
-                // Start consuming piece pc: release the buffer's previous resident set (its
-                // MMAs finish first), then wait for the piece.
-                auto begin_piece = [&]() {
-                    const int b = wb.next;
-                    wb.next ^= 1;
-                    if (wb.held[b]) {
-                        tc_commit(bar(kBarBEmpty + b));
-                        wb.held[b] = false;
-                    }
-                    mbar_wait(bar(kBarBFull + b), wb.loads[b] & 1u, p.ctr, pipe_limit, broken);
-                    ++wb.loads[b];
-                    wb.key[b] = P == 1 ? key : -1;
-                    wb.held[b] = P == 1;
-                    tc_fence_after();
-                    cur_b = b;
-                };
-                if (!resident) begin_piece();
+                // Start consuming the next piece: release the buffer's previous resident set
+                // (its MMAs finish first), then wait for the piece.
+#define MAFAT_BEGIN_PIECE()                                                                 \
+    do {                                                                                    \
+        const int b_ = wb.next;                                                             \
+        wb.next ^= 1;                                                                       \
+        if (wb.held(b_)) {                                                                  \
+            tc_commit(bar(kBarBEmpty + b_));                                                \
+            wb.release(b_);                                                                 \
+        }                                                                                   \
+        mbar_wait(bar(kBarBFull + b_), wb.loads(b_) & 1u, p.ctr, pipe_limit, broken);       \
+        wb.set_loaded(b_, P == 1 ? key : -1, P == 1);                                       \
+        tc_fence_after();                                                                   \
+        cur_b = b_;                                                                         \
+    } while (0)
+                if (!resident) MAFAT_BEGIN_PIECE();
                 const int buf = (int)(acc_cnt & 1u);
                 mbar_wait(bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
                 tc_fence_after();
@@ -465,23 +564,44 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t a_row = (uint32_t)(st.cols_box * 16);
                 const uint32_t b_half = (uint32_t)(st.n_blk * 16);
                 const uint32_t blk16 = (uint32_t)(MAFAT_BLK_ROWS * st.cols_box);  // one block down, 16-B units
+                const uint32_t a_step = 2u * (a_plane >> 4);                       // next K=16 step: two octet planes
+                // B descriptor: 128-byte swizzled blobs (64 channels per row) or no-swizzle core matrices
+                const bool bswz = st.b_swz != 0;
+                const uint32_t b_hi = bswz ? desc_hi_sw128(1024u) : (uint32_t)(smem_desc(sbase, b_half, 128u) >> 32);
+                const uint32_t b_step = bswz ? 2u : 2u * (b_half >> 4);
                 const int taps = st.k * st.k;
                 const int nbk = it.nbk;
                 uint32_t accumulate = 0;
-                int g = 0;  // blob index within the set
+                int g = 0;   // blob index within the set
+                int gp = 0;  // blob index within the current piece
+                uint32_t piece_base = sbase + kOffB + (uint32_t)cur_b * kBPieceBytes;
+                uint64_t wait_a = 0, wait_b = 0;
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
+                    const uint64_t tw0 = p.trace ? mafat_dev::globaltimer_ns() : 0;
                     mbar_wait(bar(kBarAFull + as), (a_cnt / kAStages) & 1u, p.ctr, pipe_limit, broken);
-                    if (c == 0 && p.trace) mafat_dev::trace_put(p.trace, ticket, 6, mafat_dev::globaltimer_ns());
+                    if (p.trace) {
+                        const uint64_t tw1 = mafat_dev::globaltimer_ns();
+                        if (c == 0)
+                            mafat_dev::trace_put(p.trace, ticket, 6, tw1);
+                        else
+                            wait_a += tw1 - tw0;
+                    }
                     tc_fence_after();
                     const uint32_t a_base = sbase + kOffA + as * kAStageBytes;
-                    // descriptors are advanced by adding 16-byte units to their start field
                     const uint64_t a_desc0 = smem_desc(a_base, a_plane, a_row);
+                    const uint32_t a_lo0 = (uint32_t)a_desc0, a_hi = (uint32_t)(a_desc0 >> 32);
                     int ky = 0, kx = 0;
-                    for (int t = 0; t < st.n_bsteps; ++t, ++g) {
-                        if (!resident && g > 0 && g % st.bpp == 0) begin_piece();
-                        const uint64_t b_desc =
-                            smem_desc(sbase + kOffB + cur_b * kBPieceBytes, b_half, 128u) + (uint64_t)((g % st.bpp) * blob16);
+                    for (int t = 0; t < st.n_bsteps; ++t, ++g, ++gp) {
+                        if (gp == st.bpp) {  // next streamed piece
+                            const uint64_t tp0 = p.trace ? mafat_dev::globaltimer_ns() : 0;
+                            MAFAT_BEGIN_PIECE();
+                            if (p.trace) wait_b += mafat_dev::globaltimer_ns() - tp0;
+                            gp = 0;
+                            piece_base = sbase + kOffB + (uint32_t)cur_b * kBPieceBytes;
+                        }
+                        const uint32_t blob_addr = piece_base + (uint32_t)gp * blob_bytes;
+                        const uint32_t b_lo = bswz ? desc_lo_sw128(blob_addr) : (uint32_t)smem_desc(blob_addr, b_half, 128u);
                         if (st.paired) {
                             int ta = 2 * t, tb = 2 * t + 1;
                             if (tb >= taps) {
@@ -490,19 +610,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                             }
                             const uint32_t oa = tap_off(ta, st.k, st.cols_box);
                             const uint64_t ad = smem_desc(a_base + oa, tap_off(tb, st.k, st.cols_box) - oa, a_row);
+                            const uint64_t bd = ((uint64_t)b_hi << 32) | b_lo;
                             for (int b = 0; b < nbk; ++b)
-                                mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), ad + (uint64_t)(b * blk16), b_desc, idesc,
+                                mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), ad + (uint64_t)(b * blk16), bd, idesc,
                                          accumulate);
                             accumulate = 1;
                         } else {
-                            const uint64_t at = a_desc0 + (uint64_t)(ky * st.cols_box + kx);
-                            for (int j = 0; j < st.kst; ++j) {
-                                const uint64_t bd = b_desc + (uint64_t)(j * 2 * (b_half >> 4));
-                                const uint64_t aj = at + (uint64_t)(2 * j * (a_plane >> 4));
-                                for (int b = 0; b < nbk; ++b)
-                                    mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), aj + (uint64_t)(b * blk16), bd, idesc,
-                                             accumulate);
-                                accumulate = 1;
+                            const uint32_t at = a_lo0 + (uint32_t)(ky * st.cols_box + kx);
+                            switch (st.kst) {
+                                case 4:
+                                    issue_blob<4>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
+                                                  b_step, idesc, accumulate);
+                                    break;
+                                case 2:
+                                    issue_blob<2>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
+                                                  b_step, idesc, accumulate);
+                                    break;
+                                default:
+                                    issue_blob<1>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
+                                                  b_step, idesc, accumulate);
+                                    break;
                             }
                             if (++kx == st.k) {
                                 kx = 0;
@@ -511,12 +638,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         issued = true;
                         // a streamed piece is released as soon as its last blob has been issued
-                        if (P > 1 && (g % st.bpp == st.bpp - 1 || g == G - 1)) tc_commit(bar(kBarBEmpty + cur_b));
+                        if (P > 1 && (gp == st.bpp - 1 || g == G - 1)) tc_commit(bar(kBarBEmpty + cur_b));
                     }
                     tc_commit(bar(kBarAEmpty + as));
                     ++a_cnt;
                 }
-                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 7, mafat_dev::globaltimer_ns());
+#undef MAFAT_BEGIN_PIECE
+                if (p.trace) {
+                    mafat_dev::trace_put(p.trace, ticket, 7, mafat_dev::globaltimer_ns());
+                    mafat_dev::trace_put(p.trace, ticket, 8, wait_a);
+                    mafat_dev::trace_put(p.trace, ticket, 9, wait_b);
+                }
                 tc_commit(bar(kBarAccFull + buf));
                 ++acc_cnt;
             }
@@ -528,13 +660,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------------------ epilogue (warps 0-3)
+        // ------------------------------------------------------------ epilogue (warps 0-7)
+        // Warp w reads TMEM lanes 32*(w%4) .. +31 (conv rows 4*(w%4) .. +3 of a block);
+        // the two warpgroups (h = w/4) split an item's blocks, or a single block's columns.
         uint32_t q_cnt = 0, acc_cnt = 0;
-        const int r = warp * 4 + (lane >> 3);  // conv row within the block
-        const int cc = lane & 7;               // conv column within the block
+        const int wq = warp & 3, h = warp >> 2;
+        const int r = wq * 4 + (lane >> 3);  // conv row within the block
+        const int cc = lane & 7;             // conv column within the block
         while (true) {
             const int qs = (int)(q_cnt % kQDepth);
-            mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
+            mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
             const int ticket = q_items[qs];
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
@@ -544,7 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const MafatTaskDev tk = p.tasks[it.task];
             const MafatStageDev st = p.stages[tk.stage];
             const int buf = (int)(acc_cnt & 1u);
-            mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken);
+            mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken, 128);
             if (p.trace && threadIdx.x == 0) mafat_dev::trace_put(p.trace, ticket, 2, mafat_dev::globaltimer_ns());
             __syncwarp();
             tc_fence_after();
@@ -556,7 +691,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float* sc = p.scale + st.sb_off + it.nb * st.n_blk;
             const float* bi = p.bias + st.sb_off + it.nb * st.n_blk;
             const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
-            for (int b = 0; b < it.nbk; ++b) {
+            // work split between the warpgroups: blocks when there are several, else columns
+            const bool split_blocks = it.nbk > 1;
+            const int col_lo = split_blocks ? 0 : (st.n_blk >= 32 ? h * (st.n_blk / 2) : 0);
+            const int col_hi = split_blocks ? st.n_blk : (st.n_blk >= 32 ? col_lo + st.n_blk / 2 : (h ? 0 : st.n_blk));
+            for (int b = split_blocks ? h : 0; b < it.nbk; b += split_blocks ? 2 : 1) {
                 const int Y = tk.cy0 + (it.by + b) * MAFAT_BLK_ROWS + r;
                 const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
                 bool store = valid;
@@ -575,21 +714,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                 dst.cout = st.cout;
                 dst.store = store;
                 dst.pool = st.pool;
-                const uint32_t taddr = tmem_base + ((uint32_t)(warp * 32) << 16) +
+                const uint32_t taddr = tmem_base + ((uint32_t)(wq * 32) << 16) +
                                        (uint32_t)(buf * kAccStride + b * st.n_blk);
                 const int ch_base = it.nb * st.n_blk;
-                if ((st.n_blk & 31) == 0) {
-                    for (int q = 0; q < st.n_blk; q += 32) epi_chunk<32>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
-                } else {
-                    for (int q = 0; q < st.n_blk; q += 16) epi_chunk<16>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
-                }
+                int q = col_lo;
+                for (; q + 64 <= col_hi; q += 64) epi_chunk<64>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
+                for (; q + 32 <= col_hi; q += 32) epi_chunk<32>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
+                for (; q + 16 <= col_hi; q += 16) epi_chunk<16>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
             }
             tc_fence_before();
             mbar_arrive(bar(kBarAccEmpty + buf));
             ++acc_cnt;
             mafat_dev::fence_proxy_async_global();
             __threadfence();
-            asm volatile("bar.sync 1, 128;" ::: "memory");
+            asm volatile("bar.sync 1, %0;" ::"r"(kEpiThreads) : "memory");
             if (threadIdx.x == 0) {
                 mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
                 if (p.trace) mafat_dev::trace_put(p.trace, ticket, 3, mafat_dev::globaltimer_ns());

@@ -285,6 +285,10 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 s.n_bsteps = L.k * L.k;
                 s.kst = s.chunk8 / 2;
             }
+            // 64-channel blobs use the 128-byte swizzled layout: one 128-byte row per
+            // output channel, 8-row atoms of 1024 bytes (the MMA streams them faster
+            // than no-swizzle core matrices); narrower blobs stay unswizzled.
+            s.b_swz = s.kst == 4 ? 1 : 0;
             s.blob_elems = s.n_blk * 16 * s.kst;
             s.set_bytes = s.n_chunks * s.n_bsteps * s.blob_elems * 2;
             // Weights travel in pieces of whole blobs that fill one shared-memory buffer:
@@ -558,6 +562,8 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
             return "weight blobs outside the packed weights";
         if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
+        if (s.b_swz && (s.kst != 4 || s.paired || (s.blob_elems * 2) % 1024 != 0))
+            return "swizzled blobs need 64 channels and whole 1024-byte atoms";
     }
     std::vector<int> first_item(n_tasks, -1), last_item(n_tasks, -1);
     for (size_t i = 0; i < t.items.size(); ++i) {
@@ -627,9 +633,14 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     return "";
 }
 
-// Packed bf16 weight order, per stage: [n-block][chunk][blob][K step][K half][N/8][8 rows][8 k].
-// One K=16 step holds two 8 x 8 core-matrix columns (K halves) of the B operand; within a
-// half, the n_blk rows are groups of 8 rows x 16 bytes (one core matrix each).
+// Packed bf16 weight order, per stage: [n-block][chunk][blob], each blob one B operand of
+// kst K=16 steps for n_blk output channels, in one of two shared-memory images:
+//  - no swizzle: [K step][K half][N/8][8 rows][8 k]: one K=16 step holds two 8 x 8
+//    core-matrix columns (K halves); within a half, the n_blk rows are groups of 8 rows x
+//    16 bytes (one core matrix each);
+//  - 128-byte swizzle (kst == 4): output channel n owns the 128-byte row (n/8)*1024 +
+//    (n%8)*128 of K = 64 channels, whose 16-byte unit u (input octet u of the chunk) sits
+//    at unit u ^ (n%8) of the row; the tensor core undoes the XOR from the address bits.
 //  - regular stages: blob = tap (ky, kx), K half h of step j = input octet chunk*chunk8 + 2j + h;
 //  - paired stages (8 input channels): blob p holds taps (a, b) = (2p, 2p+1), or for an odd
 //    tap count the last blob holds (zero weights, last tap); K half 0 = tap a, half 1 = tap b.
@@ -667,8 +678,15 @@ void pack_weights_bf16(const Net& net, const PlanTables& t, std::vector<uint16_t
                                         int ky = tap / k, kx = tap % k;
                                         v = w[(((size_t)o * cin + ci) * k + ky) * k + kx];
                                     }
-                                    size_t idx = blob + (size_t)j * 2 * s.n_blk * 8 + (size_t)h * s.n_blk * 8 +
-                                                 (size_t)(nn / 8) * 64 + (size_t)(nn % 8) * 8 + e;
+                                    size_t idx;
+                                    if (s.b_swz) {
+                                        const int u = 2 * j + h;  // 16-byte unit of the 128-byte row
+                                        idx = blob + (size_t)(nn / 8) * 512 + (size_t)(nn % 8) * 64 +
+                                              (size_t)((u ^ (nn % 8)) * 8) + e;
+                                    } else {
+                                        idx = blob + (size_t)j * 2 * s.n_blk * 8 + (size_t)h * s.n_blk * 8 +
+                                              (size_t)(nn / 8) * 64 + (size_t)(nn % 8) * 8 + e;
+                                    }
                                     out[idx] = f32_to_bf16_rne(v);
                                 }
                 }
