@@ -134,6 +134,47 @@ __device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, uint32_
     }
 }
 
+// The MMA warp's wait.  Measured on GB300: a polling loop written in C++ anywhere in
+// the MMA issue loop (even one whose exit is a warp vote) more than halves the MMA
+// issue rate of the whole loop, while the same loop inside one asm statement costs
+// nothing.  So the poll, with its deadline on %globaltimer, lives in the asm, and a
+// timeout is recorded by every lane alike (no branch on the lane).
+__device__ __forceinline__ void mbar_wait_mma(uint32_t bar, uint32_t parity, uint32_t* ctr, int64_t limit_ns,
+                                              volatile int* broken) {
+    const uint64_t lim = (uint64_t)(*broken ? 1000000LL : limit_ns);
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred P1, P2;\n\t.reg .u64 dl, t;\n\t"
+        "mov.u32 %0, 1;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 P1, [%1], %2;\n\t"
+        "@P1 bra MW_DONE_%=;\n\t"
+        "mov.u64 dl, %%globaltimer;\n\t"
+        "add.u64 dl, dl, %3;\n\t"
+        "MW_POLL_%=:\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 P1, [%1], %2;\n\t"
+        "@P1 bra MW_DONE_%=;\n\t"
+        "mov.u64 t, %%globaltimer;\n\t"
+        "setp.lt.u64 P2, t, dl;\n\t"
+        "@P2 bra MW_POLL_%=;\n\t"
+        "mov.u32 %0, 0;\n\t"
+        "MW_DONE_%=:\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "l"(lim)
+        : "memory");
+    if (__any_sync(0xffffffffu, ok == 0u)) {
+        mafat_dev::record_status(ctr, MAFAT_DEV_PIPE);
+        *broken = 1;
+    }
+    __syncwarp();
+}
+
+__device__ __forceinline__ void mbar_arrive_elect(uint32_t bar) {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+        "@e mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}" ::"r"(bar)
+        : "memory");
+}
+
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
                                             uint32_t bar) {
     asm volatile(
@@ -152,8 +193,21 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+// Broadcast from lane 0: marks the value warp-uniform for the compiler.
+__device__ __forceinline__ int wu(int v) { return __shfl_sync(0xffffffffu, v, 0); }
+
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+// Warp-wide forms for the MMA warp, whose 32 lanes all run the issue loop (so that
+// descriptors stay warp-uniform): elect.sync picks one lane, the same lane every time
+// since the warp is converged, to issue the operation.
+__device__ __forceinline__ void tc_commit_warp(uint32_t bar) {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar)
+        : "memory");
 }
 
 // Shared-memory matrix descriptor, no swizzle: start >> 4 in bits 0-13, LBO >> 4
@@ -188,39 +242,22 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
-// The MMA issuer is one thread whose dependent instruction chain sets its issue
-// rate, so the hot loop keeps descriptors as 32-bit halves: the low word holds
+// The MMA warp runs its loop on all 32 lanes and one elected lane issues each MMA
+// (a lone lane in diverged code issues far slower).  The hot loop keeps descriptors
+// as 32-bit halves: the low word holds
 // start address >> 4 (bits 0-13) and LBO >> 4 (bits 16-29), and advancing an
 // operand only adds 16-byte units to it; the high word (SBO, version, swizzle
 // mode) is fixed per operand.
 __device__ __forceinline__ void mma_lo(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo, uint32_t b_hi,
                                        uint32_t idesc, uint32_t accumulate) {
     asm volatile(
-        "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+        "{\n\t.reg .pred p, e;\n\t.reg .b64 da, db;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
         "setp.ne.b32 p, %6, 0;\n\t"
         "mov.b64 da, {%1, %2};\n\t"
         "mov.b64 db, {%3, %4};\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %5, p;\n\t}" ::"r"(d_tmem),
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %5, p;\n\t}" ::"r"(d_tmem),
         "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
-}
-
-// One weight blob of a regular stage: KST K=16 steps x nbk blocks (blocks share the
-// B operand, so consecutive MMAs of a K step re-read it).
-template <int KST>
-__device__ __forceinline__ void issue_blob(uint32_t d_tmem, uint32_t n_blk, int nbk, uint32_t a_lo, uint32_t a_hi,
-                                           uint32_t a_step, uint32_t a_blk, uint32_t b_lo, uint32_t b_hi,
-                                           uint32_t b_step, uint32_t idesc, uint32_t& accumulate) {
-#pragma unroll
-    for (int j = 0; j < KST; ++j) {
-        uint32_t d = d_tmem, a = a_lo + (uint32_t)j * a_step;
-        const uint32_t b = b_lo + (uint32_t)j * b_step;
-        for (int blk = 0; blk < nbk; ++blk) {
-            mma_lo(d, a, a_hi, b, b_hi, idesc, accumulate);
-            d += n_blk;
-            a += a_blk;
-        }
-        accumulate = 1;
-    }
 }
 
 // 128-byte-swizzled, K-major B operand (weights packed so by the host): rows of
@@ -379,6 +416,119 @@ __device__ __forceinline__ uint32_t tap_off(int t, int k, int cols) {
     return (uint32_t)(((t / k) * cols + (t % k)) * 16);
 }
 
+// ----------------------------------------------------------------------------- MMA warp
+// State of the MMA warp that lives across items.
+struct MmaState {
+    WeightBufs wb;
+    uint32_t a_cnt;                 // A halo stages consumed
+    uint32_t sbase;                 // shared-memory base (warp-uniform)
+    uint32_t* ctr;
+    int64_t pipe_limit;
+    volatile int* broken;
+    unsigned long long* trace;
+    __device__ __forceinline__ uint32_t bar(int i) const { return sbase + (uint32_t)(i * 8); }
+};
+
+// One item's MMA parameters, all warp-uniform.
+struct MmaJob {
+    uint32_t d_tmem, idesc;
+    uint32_t a_plane, a_row, a_step, blk16;  // A: octet-plane and row strides (bytes), K step and block (16-B units)
+    uint32_t b_hi, b_half, b_step, blob_bytes, n_blk;
+    int k, cols_box, n_chunks, n_bsteps, bpp, P, G, key, ticket, cur_b;
+    bool bswz;
+    uint64_t wait_a, wait_b;
+};
+
+// Start consuming the next weight piece: release the buffer's previous resident set
+// (its MMAs finish first), then wait for the piece.
+__device__ __forceinline__ void mma_begin_piece(MmaState& s, MmaJob& j) {
+    const int b = s.wb.next;
+    s.wb.next ^= 1;
+    if (s.wb.held(b)) {
+        tc_commit_warp(s.bar(kBarBEmpty + b));
+        s.wb.release(b);
+    }
+    mbar_wait_mma(s.bar(kBarBFull + b), s.wb.loads(b) & 1u, s.ctr, s.pipe_limit, s.broken);
+    s.wb.set_loaded(b, j.P == 1 ? j.key : -1, j.P == 1);
+    tc_fence_after();
+    j.cur_b = b;
+}
+
+// All MMAs of one item, for KST K=16 steps per weight blob, NBK M blocks (sharing every
+// B operand) and the paired-tap form (8 input channels, two taps per K step).  One
+// instance per shape keeps every blob's KST x NBK MMAs one straight run of code: on
+// GB300, MMAs separated by a runtime loop or a branch per MMA, or by a jump per blob into
+// a large switch, issued at half the tensor core's rate or worse.
+template <int KST, int NBK, bool PAIRED>
+__device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
+    uint32_t accumulate = 0;
+    int g = 0;   // blob index within the weight set
+    int gp = 0;  // blob index within the current piece
+    uint32_t piece_base = s.sbase + kOffB + (uint32_t)j.cur_b * kBPieceBytes;
+    const int taps = j.k * j.k;
+    for (int c = 0; c < j.n_chunks; ++c) {
+        const int as = (int)(s.a_cnt % kAStages);
+        const uint64_t tw0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+        mbar_wait_mma(s.bar(kBarAFull + as), (s.a_cnt / kAStages) & 1u, s.ctr, s.pipe_limit, s.broken);
+        if (s.trace) {  // every lane stores (one value wins): no branch on the lane
+            const uint64_t tw1 = mafat_dev::globaltimer_ns();
+            if (c > 0)
+                j.wait_a += tw1 - tw0;
+            else
+                mafat_dev::trace_put(s.trace, j.ticket, 6, tw1);
+        }
+        tc_fence_after();
+        const uint32_t a_base = s.sbase + kOffA + (uint32_t)as * kAStageBytes;
+        const uint64_t a_desc0 = smem_desc(a_base, j.a_plane, j.a_row);
+        const uint32_t a_lo0 = (uint32_t)a_desc0, a_hi = (uint32_t)(a_desc0 >> 32);
+        int ky = 0, kx = 0;
+        for (int t = 0; t < j.n_bsteps; ++t, ++g, ++gp) {
+            if (gp == j.bpp) {  // next streamed piece
+                const uint64_t tp0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+                mma_begin_piece(s, j);
+                if (s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
+                gp = 0;
+                piece_base = s.sbase + kOffB + (uint32_t)j.cur_b * kBPieceBytes;
+            }
+            const uint32_t blob_addr = piece_base + (uint32_t)gp * j.blob_bytes;
+            const uint32_t b_lo =
+                j.bswz ? desc_lo_sw128(blob_addr) : (uint32_t)smem_desc(blob_addr, j.b_half, 128u);
+            uint32_t a_lo, a_hi_t;
+            if (PAIRED) {
+                // taps (2t, 2t+1) as the two K halves: LBO = their distance; for an odd tap
+                // count the last blob pairs zero weights with the last tap
+                int ta = 2 * t, tb = 2 * t + 1;
+                if (tb >= taps) {
+                    ta = taps - 2;
+                    tb = taps - 1;
+                }
+                const uint32_t oa = tap_off(ta, j.k, j.cols_box);
+                const uint64_t ad = smem_desc(a_base + oa, tap_off(tb, j.k, j.cols_box) - oa, j.a_row);
+                a_lo = (uint32_t)ad;  // block offsets only touch the address field (no carry: addresses < 2^18)
+                a_hi_t = (uint32_t)(ad >> 32);
+            } else {
+                a_lo = a_lo0 + (uint32_t)(ky * j.cols_box + kx);
+                a_hi_t = a_hi;
+                if (++kx == j.k) {
+                    kx = 0;
+                    ++ky;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < KST; ++q)
+#pragma unroll
+                for (int b = 0; b < NBK; ++b)
+                    mma_lo(j.d_tmem + (uint32_t)b * j.n_blk, a_lo + (uint32_t)q * j.a_step + (uint32_t)b * j.blk16,
+                           a_hi_t, b_lo + (uint32_t)q * j.b_step, j.b_hi, j.idesc, q == 0 ? accumulate : 1u);
+            accumulate = 1;
+            // a streamed piece is released as soon as its last blob has been issued
+            if (j.P > 1 && (gp == j.bpp - 1 || g == j.G - 1)) tc_commit_warp(s.bar(kBarBEmpty + j.cur_b));
+        }
+        tc_commit_warp(s.bar(kBarAEmpty + as));
+        ++s.a_cnt;
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     mafat_tc_kernel(const __grid_constant__ MafatKParams p, const __grid_constant__ CUtensorMap in_map) {
     extern __shared__ uint8_t smem_raw[];
@@ -415,6 +565,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == kMmaWarp) {
+        __syncwarp();  // .sync.aligned: the whole warp, converged
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          sbase + (uint32_t)kOffTmem),
                      "r"(kTmemCols)
@@ -519,143 +670,88 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __syncwarp();
     } else if (warp == kMmaWarp) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            uint32_t a_cnt = 0, q_cnt = 0, acc_cnt = 0;
-            WeightBufs wb;
+        // ------------------------------------------------------------ MMA issuer (whole warp)
+        // Every value that feeds an MMA operand passes through wu() (a broadcast from lane
+        // 0), so that the compiler knows it is warp-uniform.
+        {
+            MmaState ms;
+            ms.a_cnt = 0;
+            ms.sbase = (uint32_t)wu((int)sbase);
+            ms.ctr = p.ctr;
+            ms.pipe_limit = pipe_limit;
+            ms.broken = broken;
+            ms.trace = p.trace;
+            const uint32_t tmem_u = (uint32_t)wu((int)tmem_base);
+            uint32_t q_cnt = 0, acc_cnt = 0;
             bool issued = false;
             while (true) {
                 const int qs = (int)(q_cnt % kQDepth);
-                mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
-                const int ticket = q_items[qs];
-                mbar_arrive(bar(kBarQEmpty + qs));
+                mbar_wait_mma(ms.bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
+                const int ticket = wu(q_items[qs]);
+                mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
-                const MafatItemDev it = p.items[ticket];
-                const MafatTaskDev tk = p.tasks[it.task];
-                const MafatStageDev st = p.stages[tk.stage];
-                const int key = tk.stage * 256 + it.nb;
-                const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
-                const uint32_t blob_bytes = (uint32_t)(st.blob_elems * 2);
-                int cur_b = P == 1 ? wb.resident(key) : -1;
-                const bool resident = cur_b >= 0;
-                // Start consuming the next piece: release the buffer's previous resident set
-                // (its MMAs finish first), then wait for the piece.
-#define MAFAT_BEGIN_PIECE()                                                                 \
-    do {                                                                                    \
-        const int b_ = wb.next;                                                             \
-        wb.next ^= 1;                                                                       \
-        if (wb.held(b_)) {                                                                  \
-            tc_commit(bar(kBarBEmpty + b_));                                                \
-            wb.release(b_);                                                                 \
-        }                                                                                   \
-        mbar_wait(bar(kBarBFull + b_), wb.loads(b_) & 1u, p.ctr, pipe_limit, broken);       \
-        wb.set_loaded(b_, P == 1 ? key : -1, P == 1);                                       \
-        tc_fence_after();                                                                   \
-        cur_b = b_;                                                                         \
-    } while (0)
-                if (!resident) MAFAT_BEGIN_PIECE();
+                const MafatItemDev& it = p.items[ticket];
+                const MafatTaskDev& tk = p.tasks[it.task];
+                const MafatStageDev& st = p.stages[tk.stage];
+                MmaJob j;
+                j.ticket = ticket;
+                j.k = wu(st.k);
+                j.cols_box = wu(st.cols_box);
+                j.n_blk = (uint32_t)wu(st.n_blk);
+                j.n_chunks = wu(st.n_chunks);
+                j.n_bsteps = wu(st.n_bsteps);
+                j.bpp = wu(st.bpp);
+                j.P = wu(st.n_pieces);
+                j.G = j.n_chunks * j.n_bsteps;
+                j.key = wu(tk.stage * 256 + it.nb);
+                j.blob_bytes = (uint32_t)wu(st.blob_elems * 2);
+                j.a_plane = (uint32_t)wu(st.rows_box * st.cols_box * 16);
+                j.bswz = wu(st.b_swz) != 0;
+                const int kst = wu(st.kst), nbk = wu(it.nbk), paired = wu(st.paired);
+                j.cur_b = j.P == 1 ? ms.wb.resident(j.key) : -1;
+                if (j.cur_b < 0) mma_begin_piece(ms, j);
                 const int buf = (int)(acc_cnt & 1u);
-                mbar_wait(bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
+                mbar_wait_mma(ms.bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kAccStride);
-                const uint32_t idesc = instr_desc_bf16(st.n_blk, 128);
-                const uint32_t a_plane = (uint32_t)(st.rows_box * st.cols_box * 16);
-                const uint32_t a_row = (uint32_t)(st.cols_box * 16);
-                const uint32_t b_half = (uint32_t)(st.n_blk * 16);
-                const uint32_t blk16 = (uint32_t)(MAFAT_BLK_ROWS * st.cols_box);  // one block down, 16-B units
-                const uint32_t a_step = 2u * (a_plane >> 4);                       // next K=16 step: two octet planes
+                j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
+                j.idesc = instr_desc_bf16((int)j.n_blk, 128);
+                j.a_row = (uint32_t)(j.cols_box * 16);
+                j.b_half = j.n_blk * 16u;
+                j.blk16 = (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);  // one block down, 16-B units
+                j.a_step = 2u * (j.a_plane >> 4);                   // next K=16 step: two octet planes
                 // B descriptor: 128-byte swizzled blobs (64 channels per row) or no-swizzle core matrices
-                const bool bswz = st.b_swz != 0;
-                const uint32_t b_hi = bswz ? desc_hi_sw128(1024u) : (uint32_t)(smem_desc(sbase, b_half, 128u) >> 32);
-                const uint32_t b_step = bswz ? 2u : 2u * (b_half >> 4);
-                const int taps = st.k * st.k;
-                const int nbk = it.nbk;
-                uint32_t accumulate = 0;
-                int g = 0;   // blob index within the set
-                int gp = 0;  // blob index within the current piece
-                uint32_t piece_base = sbase + kOffB + (uint32_t)cur_b * kBPieceBytes;
-                uint64_t wait_a = 0, wait_b = 0;
-                for (int c = 0; c < st.n_chunks; ++c) {
-                    const int as = (int)(a_cnt % kAStages);
-                    const uint64_t tw0 = p.trace ? mafat_dev::globaltimer_ns() : 0;
-                    mbar_wait(bar(kBarAFull + as), (a_cnt / kAStages) & 1u, p.ctr, pipe_limit, broken);
-                    if (p.trace) {
-                        const uint64_t tw1 = mafat_dev::globaltimer_ns();
-                        if (c == 0)
-                            mafat_dev::trace_put(p.trace, ticket, 6, tw1);
-                        else
-                            wait_a += tw1 - tw0;
-                    }
-                    tc_fence_after();
-                    const uint32_t a_base = sbase + kOffA + as * kAStageBytes;
-                    const uint64_t a_desc0 = smem_desc(a_base, a_plane, a_row);
-                    const uint32_t a_lo0 = (uint32_t)a_desc0, a_hi = (uint32_t)(a_desc0 >> 32);
-                    int ky = 0, kx = 0;
-                    for (int t = 0; t < st.n_bsteps; ++t, ++g, ++gp) {
-                        if (gp == st.bpp) {  // next streamed piece
-                            const uint64_t tp0 = p.trace ? mafat_dev::globaltimer_ns() : 0;
-                            MAFAT_BEGIN_PIECE();
-                            if (p.trace) wait_b += mafat_dev::globaltimer_ns() - tp0;
-                            gp = 0;
-                            piece_base = sbase + kOffB + (uint32_t)cur_b * kBPieceBytes;
-                        }
-                        const uint32_t blob_addr = piece_base + (uint32_t)gp * blob_bytes;
-                        const uint32_t b_lo = bswz ? desc_lo_sw128(blob_addr) : (uint32_t)smem_desc(blob_addr, b_half, 128u);
-                        if (st.paired) {
-                            int ta = 2 * t, tb = 2 * t + 1;
-                            if (tb >= taps) {
-                                ta = taps - 2;
-                                tb = taps - 1;
-                            }
-                            const uint32_t oa = tap_off(ta, st.k, st.cols_box);
-                            const uint64_t ad = smem_desc(a_base + oa, tap_off(tb, st.k, st.cols_box) - oa, a_row);
-                            const uint64_t bd = ((uint64_t)b_hi << 32) | b_lo;
-                            for (int b = 0; b < nbk; ++b)
-                                mma_bf16(d_tmem + (uint32_t)(b * st.n_blk), ad + (uint64_t)(b * blk16), bd, idesc,
-                                         accumulate);
-                            accumulate = 1;
-                        } else {
-                            const uint32_t at = a_lo0 + (uint32_t)(ky * st.cols_box + kx);
-                            switch (st.kst) {
-                                case 4:
-                                    issue_blob<4>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
-                                                  b_step, idesc, accumulate);
-                                    break;
-                                case 2:
-                                    issue_blob<2>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
-                                                  b_step, idesc, accumulate);
-                                    break;
-                                default:
-                                    issue_blob<1>(d_tmem, (uint32_t)st.n_blk, nbk, at, a_hi, a_step, blk16, b_lo, b_hi,
-                                                  b_step, idesc, accumulate);
-                                    break;
-                            }
-                            if (++kx == st.k) {
-                                kx = 0;
-                                ++ky;
-                            }
-                        }
-                        issued = true;
-                        // a streamed piece is released as soon as its last blob has been issued
-                        if (P > 1 && (gp == st.bpp - 1 || g == G - 1)) tc_commit(bar(kBarBEmpty + cur_b));
-                    }
-                    tc_commit(bar(kBarAEmpty + as));
-                    ++a_cnt;
+                j.b_hi = j.bswz ? desc_hi_sw128(1024u) : (uint32_t)(smem_desc(0u, j.b_half, 128u) >> 32);
+                j.b_step = j.bswz ? 2u : 2u * (j.b_half >> 4);
+                j.wait_a = 0;
+                j.wait_b = 0;
+                // one jump per item into the instance for its shape
+                switch ((paired << 8) | (kst << 4) | nbk) {
+#define MAFAT_MMA_CASE(PA, K, B) \
+    case ((PA) << 8) | ((K) << 4) | (B): mma_item<K, B, PA>(ms, j); break;
+                    MAFAT_MMA_CASE(0, 4, 1) MAFAT_MMA_CASE(0, 4, 2) MAFAT_MMA_CASE(0, 4, 3) MAFAT_MMA_CASE(0, 4, 4)
+                    MAFAT_MMA_CASE(0, 2, 1) MAFAT_MMA_CASE(0, 2, 2) MAFAT_MMA_CASE(0, 2, 3) MAFAT_MMA_CASE(0, 2, 4)
+                    MAFAT_MMA_CASE(0, 1, 1) MAFAT_MMA_CASE(0, 1, 2) MAFAT_MMA_CASE(0, 1, 3) MAFAT_MMA_CASE(0, 1, 4)
+                    MAFAT_MMA_CASE(1, 1, 1) MAFAT_MMA_CASE(1, 1, 2) MAFAT_MMA_CASE(1, 1, 3) MAFAT_MMA_CASE(1, 1, 4)
+#undef MAFAT_MMA_CASE
+                    default:  // a shape the planner never makes: fail loudly, never compute silently wrong
+                        mafat_dev::record_status(p.ctr, MAFAT_DEV_PIPE);
+                        *broken = 1;
+                        break;
                 }
-#undef MAFAT_BEGIN_PIECE
+                issued = true;
                 if (p.trace) {
                     mafat_dev::trace_put(p.trace, ticket, 7, mafat_dev::globaltimer_ns());
-                    mafat_dev::trace_put(p.trace, ticket, 8, wait_a);
-                    mafat_dev::trace_put(p.trace, ticket, 9, wait_b);
+                    mafat_dev::trace_put(p.trace, ticket, 8, j.wait_a);
+                    mafat_dev::trace_put(p.trace, ticket, 9, j.wait_b);
                 }
-                tc_commit(bar(kBarAccFull + buf));
+                tc_commit_warp(ms.bar(kBarAccFull + buf));
                 ++acc_cnt;
             }
-            // Every MMA this thread issued has completed before TMEM is released.
+            // Every MMA this warp issued has completed before TMEM is released.
             if (issued) {
-                tc_commit(bar(kBarDone));
-                mbar_wait(bar(kBarDone), 0u, p.ctr, pipe_limit, broken);
+                tc_commit_warp(ms.bar(kBarDone));
+                mbar_wait_mma(ms.bar(kBarDone), 0u, p.ctr, pipe_limit, broken);
             }
         }
         __syncwarp();
@@ -739,6 +835,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     if (warp == kMmaWarp) {
+        __syncwarp();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(kTmemCols)
                      : "memory");
     }
@@ -772,6 +869,7 @@ __global__ void __launch_bounds__(128, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if ((tid >> 5) == 0) {
+        __syncwarp();  // thread 0 just left a branch of its own; .sync.aligned needs the warp converged
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
                      "r"(256)
                      : "memory");
@@ -822,6 +920,7 @@ __global__ void __launch_bounds__(128, 1)
     __syncthreads();
     tc_fence_after();
     if (warp == 0) {
+        __syncwarp();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256) : "memory");
     }
 }

@@ -255,6 +255,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 while (s.mb * 2 * s.n_blk <= 256 && blocks * s.n_nblk / (s.mb * 2) >= n_ctas) s.mb *= 2;
             }
             if (s.mb * s.n_blk > 256) s.mb = std::max(1, 256 / s.n_blk);
+            s.mb = std::min(s.mb, MAFAT_MAX_MB);  // the kernel has MMA code for 1..4 blocks per item
             s.cols_box = MAFAT_BLK_COLS + L.k - 1;
             // input octets per A chunk: the largest that fits the A stage with mb blocks
             for (;;) {
@@ -264,7 +265,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                     s.chunk8 = 1;
                 } else {
                     s.chunk8 = 0;
-                    for (int d = 8; d >= 2; d -= 2)
+                    for (int d = 8; d >= 2; d /= 2)  // 8, 4 or 2 octets: 4, 2 or 1 K steps per blob
                         if (s.cin8 % d == 0 && d * row_bytes <= MAFAT_A_STAGE_BYTES) {
                             s.chunk8 = d;
                             break;
@@ -562,6 +563,9 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
             return "weight blobs outside the packed weights";
         if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
+        if (s.mb < 1 || s.mb > MAFAT_MAX_MB) return "blocks per item out of range";
+        if (!(s.kst == 1 || s.kst == 2 || s.kst == 4) || (s.paired && s.kst != 1))
+            return "K steps per blob must be 1, 2 or 4 (1 when taps are paired)";
         if (s.b_swz && (s.kst != 4 || s.paired || (s.blob_elems * 2) % 1024 != 0))
             return "swizzled blobs need 64 channels and whole 1024-byte atoms";
     }
