@@ -165,6 +165,13 @@ int largest_nblk(int cout) {
     return 16;
 }
 
+// The largest multiple of 16 below `below` that divides cout (16 if none).
+int largest_nblk_below(int cout, int below) {
+    for (int d = below - 16; d >= 16; d -= 16)
+        if (cout % d == 0) return d;
+    return 16;
+}
+
 }  // namespace
 
 std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, bool* unsupported) {
@@ -235,16 +242,23 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 blocks += (int64_t)ceil_div(cr.h(), MAFAT_BLK_ROWS) * ceil_div(cr.w(), MAFAT_BLK_COLS);
             }
             blocks *= cfg.batch;
-            // Output-channel block (MMA N): as wide as possible, narrowed while the stage
-            // would have fewer items than CTAs (short stages then spread over more SMs).
-            // The MMA N must be a multiple of 16: pad with zero weights, store only cout channels.
-            // Output-channel block (MMA N): as wide as possible (up to 256).  Narrower
-            // blocks would spread short stages over more SMs, but every item then streams
-            // the same activations and more weight pieces; measured, the widest block is
-            // fastest.  The MMA N must be a multiple of 16: pad with zero weights, store
-            // only cout channels.
+            // Output-channel block (MMA N, a multiple of 16 dividing the padded cout; zero
+            // weights pad it, only cout channels are stored): the widest block that still
+            // gives every CTA an item, but not below 64 channels.  Wide blocks reuse each A
+            // operand for more output channels; a stage with few M blocks (the small maps
+            // after the cut) needs narrower ones to spread over the SMs, which measured
+            // faster down to N = 64 and slower at N = 32 (the MMA's A read then dominates).
             const int cout_pad = (L.c_out + 15) / 16 * 16;
-            s.n_blk = cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0 ? cfg.fixed_nblk : largest_nblk(cout_pad);
+            if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
+                s.n_blk = cfg.fixed_nblk;
+            } else {
+                s.n_blk = largest_nblk(cout_pad);
+                while (s.n_blk > 64 && blocks * (cout_pad / s.n_blk) < n_ctas) {
+                    const int next = largest_nblk_below(cout_pad, s.n_blk);
+                    if (next < 64) break;
+                    s.n_blk = next;
+                }
+            }
             s.n_nblk = cout_pad / s.n_blk;
             // Blocks per item (stacked along rows, one accumulator each, sharing every
             // weight blob): grow while the stage keeps at least one item per CTA.
