@@ -287,6 +287,11 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&h);
 }
+__device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
+    __nv_bfloat162 x = *reinterpret_cast<__nv_bfloat162*>(&a), y = *reinterpret_cast<__nv_bfloat162*>(&b);
+    __nv_bfloat162 m = __hmax2(x, y);
+    return *reinterpret_cast<uint32_t*>(&m);
+}
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
@@ -331,8 +336,9 @@ struct EpiDst {
 };
 
 // Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1) of one
-// pixel per thread: folded BN, leaky ReLU 0.1, optional 2x2 max over the quad
-// lanes {l, l^1, l^8, l^9}, bf16 (nearest-even) and 16-byte stores per octet.
+// pixel per thread: folded BN, leaky ReLU 0.1, bf16 (nearest-even), optional 2x2 max
+// over the quad lanes {l, l^1, l^8, l^9} on the packed bf16 pairs (rounding is
+// monotonic, so the max of rounded values is the rounded max), 16-byte stores per octet.
 template <int NC>
 __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const float* bi, int ch0,
                                           const EpiDst& d) {
@@ -343,23 +349,26 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         tmem_ld32(taddr, raw);
     else
         tmem_ld16(taddr, raw);
-    float v[NC];
+    uint32_t pk[NC / 2];
 #pragma unroll
     for (int i = 0; i < NC; i += 4) {
         const float4 s4 = __ldg(reinterpret_cast<const float4*>(sc + i));
         const float4 b4 = __ldg(reinterpret_cast<const float4*>(bi + i));
         const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+        float v[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const float z = sv[u] * __uint_as_float(raw[i + u]) + bv[u];
-            v[i + u] = z > 0.f ? z : 0.1f * z;
+            v[u] = z > 0.f ? z : 0.1f * z;
         }
+        pk[i / 2] = pack_bf16x2(v[0], v[1]);
+        pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
     }
     if (d.pool) {
 #pragma unroll
-        for (int i = 0; i < NC; ++i) {
-            v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 1));
-            v[i] = fmaxf(v[i], __shfl_xor_sync(0xffffffffu, v[i], 8));
+        for (int i = 0; i < NC / 2; ++i) {
+            pk[i] = max_bf16x2(pk[i], __shfl_xor_sync(0xffffffffu, pk[i], 1));
+            pk[i] = max_bf16x2(pk[i], __shfl_xor_sync(0xffffffffu, pk[i], 8));
         }
     }
     if (!d.store) return;
@@ -367,11 +376,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
     for (int o = 0; o < NC / 8; ++o) {
         const int ch = ch0 + 8 * o;
         if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
-        uint4 w;
-        w.x = pack_bf16x2(v[8 * o + 0], v[8 * o + 1]);
-        w.y = pack_bf16x2(v[8 * o + 2], v[8 * o + 3]);
-        w.z = pack_bf16x2(v[8 * o + 4], v[8 * o + 5]);
-        w.w = pack_bf16x2(v[8 * o + 6], v[8 * o + 7]);
+        const uint4 w = make_uint4(pk[4 * o], pk[4 * o + 1], pk[4 * o + 2], pk[4 * o + 3]);
         __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
         *reinterpret_cast<uint4*>(p) = w;
     }
@@ -821,8 +826,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             mbar_arrive(bar(kBarAccEmpty + buf));
             ++acc_cnt;
+            // Every epilogue thread's stores are ordered before the barrier; thread 0 then
+            // publishes with a gpu-scope fence and release (cumulative over the barrier), so
+            // no thread needs a gpu-scope fence of its own.  The proxy fence orders the stores
+            // (generic proxy) with later TMA reads (async proxy) of the same memory.
             mafat_dev::fence_proxy_async_global();
-            __threadfence();
             asm volatile("bar.sync 1, %0;" ::"r"(kEpiThreads) : "memory");
             if (threadIdx.x == 0) {
                 mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
