@@ -64,6 +64,16 @@ def dist_env():
     return ws, rank, local
 
 
+def reduce_max(pg, values, device):
+    """Max over ranks of each value (the slowest rank's times); the values themselves at N = 1."""
+    if pg is None:
+        return [float(v) for v in values]
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
 def aggregate(units_per_rank, seconds_per_rank):
     """Whole-job throughput of independent replicas: all units over the slowest rank's time."""
     return float(sum(units_per_rank)) / float(max(seconds_per_rank))
@@ -85,9 +95,15 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.QUERY, "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
+            # nvidia-smi takes a while to start: wait (bounded) for its first line so that
+            # the samples cover the timed region rather than the time after it
+            t0 = time.time()
+            while not self.lines and time.time() - t0 < 5.0 and self.proc.poll() is None:
+                time.sleep(0.01)
+            self.n_before = len(self.lines)
         except Exception:
             self.proc = None
 
@@ -105,7 +121,8 @@ class ClockSampler:
             self.proc.kill()
         sm, smax, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        # the samples taken after the timed region started (the first line predates it)
+        for ln in self.lines[self.n_before:] or self.lines[-1:]:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 9:
                 continue
@@ -179,7 +196,7 @@ def run_reference(args, wl):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mafat", choices=["mafat", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
@@ -258,12 +275,7 @@ def main():
         plan.run_host(xh, oh, stream=stream)
     e2e_s = time.perf_counter() - t0
 
-    if pg:
-        t = torch.tensor([dev_s, e2e_s], dtype=torch.float64, device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        dev_s_max, e2e_s_max = float(t[0]), float(t[1])
-    else:
-        dev_s_max, e2e_s_max = dev_s, e2e_s
+    dev_s_max, e2e_s_max = reduce_max(pg, [dev_s, e2e_s], dev)
     if rank != 0:
         if pg:
             pg.destroy_process_group()
