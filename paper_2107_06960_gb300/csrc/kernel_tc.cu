@@ -590,11 +590,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             // dependency counters already seen at (or above) a target: items of one task
             // usually follow each other, so most items skip the round trip to L2
             int ok_idx0 = -1, ok_idx1 = -1, ok_tgt0 = 0, ok_tgt1 = 0;
-            // the next ticket is taken one item ahead, hiding the atomic's latency
+            // The next ticket is taken one item ahead, and its item record is loaded with it,
+            // hiding the latency of the atomic and of the load behind the current item.
             int next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+            MafatItemDev it_next;
+            if (next < p.n_items) it_next = p.items[next];
             while (true) {
                 const int ticket = next < p.n_items ? next : -1;
-                if (ticket >= 0) next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                const MafatItemDev it = it_next;
+                if (ticket >= 0) {
+                    next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                    if (next < p.n_items) it_next = p.items[next];
+                }
                 if (ticket >= 0 && p.trace) {
                     mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
@@ -605,7 +612,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(bar(kBarQFull + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
-                const MafatItemDev it = p.items[ticket];
                 const MafatTaskDev tk = p.tasks[it.task];
                 const MafatStageDev st = p.stages[tk.stage];
                 const int key = tk.stage * 256 + it.nb;
