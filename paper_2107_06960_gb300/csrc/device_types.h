@@ -24,6 +24,7 @@
 #define MAFAT_BLK_ROWS 16   // conv output rows of one M block
 #define MAFAT_BLK_COLS 8    // conv output columns of one M block (M = 128)
 #define MAFAT_MAX_MB 4      // M blocks per work item
+#define MAFAT_MAX_MB_PAIRED 8  // M blocks per work item of a paired-tap (8-input-channel) layer
 #define MAFAT_MAX_NBLK 256  // output channels of one item (MMA N)
 #define MAFAT_A_STAGE_BYTES 36864   // shared-memory A halo stage of the tensor-core kernel (x2)
 #define MAFAT_B_PIECE_BYTES 75776   // one of the two shared-memory weight buffers (x2)

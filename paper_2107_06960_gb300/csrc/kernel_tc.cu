@@ -29,8 +29,8 @@
 //    of TMA time however small it is, so copies are large and few).
 //
 // Warp roles (320 threads): warps 0-7 epilogue (warp w reads TMEM lanes
-// 32(w%4)..+31 = conv rows 4(w%4)..+3 of a block; the two warpgroups split an
-// item's blocks or columns), warp 8 scheduler + TMA producer, warp 9 TMEM
+// 32(w%4)..+31 = conv rows 4(w%4)..+3 of a block; the two warpgroups take units
+// of one block x 32 columns in turn), warp 8 scheduler + TMA producer, warp 9 TMEM
 // allocator + MMA issuer.  Shared memory: 2 A halo stages, 2 weight buffers and
 // a 4-deep queue of item indices; TMEM: 2 accumulators of 256 columns (the
 // epilogue of one item overlaps the MMAs of the next).
@@ -50,7 +50,8 @@
 
 namespace {
 
-constexpr int kEpiWarps = 8;            // two warpgroups over the 128 TMEM lanes
+constexpr int kEpiGroups = 2;           // epilogue warpgroups, each over all 128 TMEM lanes
+constexpr int kEpiWarps = 4 * kEpiGroups;
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kProducerWarp = kEpiWarps;
 constexpr int kMmaWarp = kEpiWarps + 1;
@@ -416,6 +417,20 @@ struct WeightBufs {
     }
 };
 
+// L2 prefetch of this CTA's 1/gridDim share of a buffer (16-byte aligned base), in
+// bulk prefetches of at most 64 KB; the tail below 16 bytes is left out.
+__device__ __forceinline__ void prefetch_l2_share(const void* base, int64_t bytes) {
+    if (base == nullptr || bytes <= 0) return;
+    const int64_t per = ((bytes + gridDim.x - 1) / gridDim.x + 15) & ~(int64_t)15;
+    int64_t off = (int64_t)blockIdx.x * per;
+    const int64_t end = min(bytes, off + per);
+    for (; off < end; off += 65536) {
+        const uint32_t n = (uint32_t)min((int64_t)65536, end - off) & ~15u;
+        if (n == 0) break;
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"((const char*)base + off), "r"(n) : "memory");
+    }
+}
+
 // Byte offset of tap t inside an A halo buffer.
 __device__ __forceinline__ uint32_t tap_off(int t, int k, int cols) {
     return (uint32_t)(((t / k) * cols + (t % k)) * 16);
@@ -585,6 +600,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ scheduler + TMA producer
         if (lane == 0) {
+            // The input, the weights, the work tables and scale / bias are read from DRAM
+            // once per run, mostly by loads that wait for them (the first layer's halos, the
+            // first use of every weight set and table entry on each SM); fetching them into
+            // L2 at once, spread over all CTAs, overlaps those DRAM latencies instead of
+            // paying them item by item.
+            for (int r = 0; r < MAFAT_PF_REGIONS; ++r) prefetch_l2_share(p.pf_ptr[r], p.pf_bytes[r]);
             uint32_t a_cnt = 0, q_cnt = 0;
             WeightBufs wb;
             // dependency counters already seen at (or above) a target: items of one task
@@ -744,6 +765,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     MAFAT_MMA_CASE(0, 2, 1) MAFAT_MMA_CASE(0, 2, 2) MAFAT_MMA_CASE(0, 2, 3) MAFAT_MMA_CASE(0, 2, 4)
                     MAFAT_MMA_CASE(0, 1, 1) MAFAT_MMA_CASE(0, 1, 2) MAFAT_MMA_CASE(0, 1, 3) MAFAT_MMA_CASE(0, 1, 4)
                     MAFAT_MMA_CASE(1, 1, 1) MAFAT_MMA_CASE(1, 1, 2) MAFAT_MMA_CASE(1, 1, 3) MAFAT_MMA_CASE(1, 1, 4)
+                    MAFAT_MMA_CASE(1, 1, 5) MAFAT_MMA_CASE(1, 1, 6) MAFAT_MMA_CASE(1, 1, 7) MAFAT_MMA_CASE(1, 1, 8)
 #undef MAFAT_MMA_CASE
                     default:  // a shape the planner never makes: fail loudly, never compute silently wrong
                         mafat_dev::record_status(p.ctr, MAFAT_DEV_PIPE);
@@ -771,7 +793,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Warp w reads TMEM lanes 32*(w%4) .. +31 (conv rows 4*(w%4) .. +3 of a block);
         // the two warpgroups (h = w/4) split an item's blocks, or a single block's columns.
         uint32_t q_cnt = 0, acc_cnt = 0;
-        const int wq = warp & 3, h = warp >> 2;
+        const int wq = warp & 3, h = warp >> 2;  // lane quarter, warpgroup
         const int r = wq * 4 + (lane >> 3);  // conv row within the block
         const int cc = lane & 7;             // conv column within the block
         while (true) {
@@ -798,11 +820,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float* sc = p.scale + st.sb_off + it.nb * st.n_blk;
             const float* bi = p.bias + st.sb_off + it.nb * st.n_blk;
             const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
-            // work split between the warpgroups: blocks when there are several, else columns
-            const bool split_blocks = it.nbk > 1;
-            const int col_lo = split_blocks ? 0 : (st.n_blk >= 32 ? h * (st.n_blk / 2) : 0);
-            const int col_hi = split_blocks ? st.n_blk : (st.n_blk >= 32 ? col_lo + st.n_blk / 2 : (h ? 0 : st.n_blk));
-            for (int b = split_blocks ? h : 0; b < it.nbk; b += split_blocks ? 2 : 1) {
+            // Work split between the warpgroups in units of one block x 32 output columns
+            // (16 when N is an odd multiple of 16), dealt round-robin.
+            const int uw = (st.n_blk % 32 == 0) ? 32 : 16;
+            const int upb = st.n_blk / uw;  // units per block
+            const int ch_base = it.nb * st.n_blk;
+            for (int u = h; u < it.nbk * upb; u += kEpiGroups) {
+                const int b = u / upb, q = (u - b * upb) * uw;
                 const int Y = tk.cy0 + (it.by + b) * MAFAT_BLK_ROWS + r;
                 const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
                 bool store = valid;
@@ -822,12 +846,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 dst.store = store;
                 dst.pool = st.pool;
                 const uint32_t taddr = tmem_base + ((uint32_t)(wq * 32) << 16) +
-                                       (uint32_t)(buf * kAccStride + b * st.n_blk);
-                const int ch_base = it.nb * st.n_blk;
-                int q = col_lo;
-                for (; q + 64 <= col_hi; q += 64) epi_chunk<64>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
-                for (; q + 32 <= col_hi; q += 32) epi_chunk<32>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
-                for (; q + 16 <= col_hi; q += 16) epi_chunk<16>(taddr + (uint32_t)q, sc + q, bi + q, ch_base + q, dst);
+                                       (uint32_t)(buf * kAccStride + b * st.n_blk + q);
+                if (uw == 32)
+                    epi_chunk<32>(taddr, sc + q, bi + q, ch_base + q, dst);
+                else
+                    epi_chunk<16>(taddr, sc + q, bi + q, ch_base + q, dst);
             }
             tc_fence_before();
             mbar_arrive(bar(kBarAccEmpty + buf));

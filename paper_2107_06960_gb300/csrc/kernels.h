@@ -6,6 +6,8 @@
 
 #include "device_types.h"
 
+#define MAFAT_PF_REGIONS 8
+
 struct MafatKParams {
     const MafatStageDev* stages;
     const MafatTaskDev* tasks;
@@ -28,6 +30,10 @@ struct MafatKParams {
     int32_t pad2;
     int64_t timeout_ns;
     unsigned long long* trace;    // per-item timestamps (null: off)
+    // Regions every CTA warms into L2 (its 1/grid share of each) at start: the input, the
+    // packed weights, the work tables and the scale / bias arrays (bytes 0: unused slot).
+    const void* pf_ptr[MAFAT_PF_REGIONS];
+    int64_t pf_bytes[MAFAT_PF_REGIONS];
 };
 
 // bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.

@@ -269,7 +269,10 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 while (s.mb * 2 * s.n_blk <= 256 && blocks * s.n_nblk / (s.mb * 2) >= n_ctas) s.mb *= 2;
             }
             if (s.mb * s.n_blk > 256) s.mb = std::max(1, 256 / s.n_blk);
-            s.mb = std::min(s.mb, MAFAT_MAX_MB);  // the kernel has MMA code for 1..4 blocks per item
+            // the kernel has MMA code for 1..4 blocks per item, and 1..8 for the paired-tap
+            // form of 8-input-channel layers (narrow N, many small items: their epilogue's
+            // fixed cost per item dominates)
+            s.mb = std::min(s.mb, s.cin8 == 1 ? MAFAT_MAX_MB_PAIRED : MAFAT_MAX_MB);
             s.cols_box = MAFAT_BLK_COLS + L.k - 1;
             // input octets per A chunk: the largest that fits the A stage with mb blocks
             for (;;) {
@@ -577,7 +580,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
             return "weight blobs outside the packed weights";
         if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
-        if (s.mb < 1 || s.mb > MAFAT_MAX_MB) return "blocks per item out of range";
+        if (s.mb < 1 || s.mb > (s.paired ? MAFAT_MAX_MB_PAIRED : MAFAT_MAX_MB)) return "blocks per item out of range";
         if (!(s.kst == 1 || s.kst == 2 || s.kst == 4) || (s.paired && s.kst != 1))
             return "K steps per blob must be 1, 2 or 4 (1 when taps are paired)";
         if (s.b_swz && (s.kst != 4 || s.paired || (s.blob_elems * 2) % 1024 != 0))

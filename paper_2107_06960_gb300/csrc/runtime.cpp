@@ -156,6 +156,16 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
     kp.timeout_ns = p->timeout_ns;
     kp.trace = p->d_trace;
     if (p->dtype == MAFAT_BF16) {
+        const void* pf[] = {input, p->d_w, p->d_items, p->d_tasks, p->d_stages, p->d_scale, p->d_bias};
+        const int64_t pb[] = {(int64_t)p->in_bytes, (int64_t)p->t.weight_elems * 2,
+                              (int64_t)(p->t.items.size() * sizeof(MafatItemDev)),
+                              (int64_t)(p->t.tasks.size() * sizeof(MafatTaskDev)),
+                              (int64_t)(p->t.stages.size() * sizeof(MafatStageDev)), (int64_t)p->t.sb_elems * 4,
+                              (int64_t)p->t.sb_elems * 4};
+        for (int i = 0; i < 7; ++i) {
+            kp.pf_ptr[i] = pf[i];
+            kp.pf_bytes[i] = pb[i];
+        }
         if (p->in_map_ptr != input) {
             std::string err;
             const mafat::Layer& L0 = p->shapes.layers[0];
