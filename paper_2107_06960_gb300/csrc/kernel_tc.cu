@@ -611,18 +611,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             // dependency counters already seen at (or above) a target: items of one task
             // usually follow each other, so most items skip the round trip to L2
             int ok_idx0 = -1, ok_idx1 = -1, ok_tgt0 = 0, ok_tgt1 = 0;
-            // The next ticket is taken one item ahead, and its item record is loaded with it,
-            // hiding the latency of the atomic and of the load behind the current item.
+            // A ticket is taken (and its item record loaded) at the end of the previous item,
+            // once the A stage the new item will use is about to free: early enough to hide
+            // the new item's loads behind the current MMAs, late enough that a CTA busy with a
+            // long item does not hold work another CTA could start now.
             int next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
             MafatItemDev it_next;
             if (next < p.n_items) it_next = p.items[next];
             while (true) {
                 const int ticket = next < p.n_items ? next : -1;
                 const MafatItemDev it = it_next;
-                if (ticket >= 0) {
-                    next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
-                    if (next < p.n_items) it_next = p.items[next];
-                }
                 if (ticket >= 0 && p.trace) {
                     mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
@@ -690,6 +688,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
                 }
 #undef MAFAT_LOAD_PIECE
+                mbar_wait(bar(kBarAEmpty + (int)(a_cnt % kAStages)), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr,
+                          pipe_limit, broken, 64);
+                next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                if (next < p.n_items) it_next = p.items[next];
             }
             // Drain: every copy issued has landed before the CTA may exit.
             for (uint32_t i = 0; i < kAStages && i < a_cnt; ++i) {
