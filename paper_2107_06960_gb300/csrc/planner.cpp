@@ -165,13 +165,6 @@ int largest_nblk(int cout) {
     return 16;
 }
 
-// The largest multiple of 16 below `below` that divides cout (16 if none).
-int largest_nblk_below(int cout, int below) {
-    for (int d = below - 16; d >= 16; d -= 16)
-        if (cout % d == 0) return d;
-    return 16;
-}
-
 }  // namespace
 
 std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, bool* unsupported) {
@@ -243,20 +236,23 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             }
             blocks *= cfg.batch;
             // Output-channel block (MMA N, a multiple of 16 dividing the padded cout; zero
-            // weights pad it, only cout channels are stored): the widest block that still
-            // gives every CTA an item, but not below 64 channels.  Wide blocks reuse each A
-            // operand for more output channels; a stage with few M blocks (the small maps
-            // after the cut) needs narrower ones to spread over the SMs, which measured
-            // faster down to N = 64 and slower at N = 32 (the MMA's A read then dominates).
+            // weights pad it, only cout channels are stored): the narrowest block of at least
+            // 64 channels whose items fit one wave of CTAs, else the widest.  A stage with few
+            // M blocks (the small maps after the cut) then spreads over the SMs without a
+            // second wave, which its successor would wait for; below N = 64 the MMA's A read
+            // dominates.  Stages with more blocks than CTAs keep the widest block, which
+            // reuses every A operand for the most output channels.
             const int cout_pad = (L.c_out + 15) / 16 * 16;
             if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
                 s.n_blk = cfg.fixed_nblk;
             } else {
                 s.n_blk = largest_nblk(cout_pad);
-                while (s.n_blk > 64 && blocks * (cout_pad / s.n_blk) < n_ctas) {
-                    const int next = largest_nblk_below(cout_pad, s.n_blk);
-                    if (next < 64) break;
-                    s.n_blk = next;
+                for (int nb = std::min(64, cout_pad); nb <= std::min(cout_pad, MAFAT_MAX_NBLK); nb += 16) {
+                    if (cout_pad % nb != 0) continue;
+                    if (blocks * (cout_pad / nb) <= n_ctas) {
+                        s.n_blk = nb;
+                        break;
+                    }
                 }
             }
             s.n_nblk = cout_pad / s.n_blk;
