@@ -508,14 +508,18 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         const MafatTaskDev& tk = t.tasks[ti];
         const MafatStageDev& st = t.stages[tk.stage];
         const TaskDep& d = deps[ti];
-        // channel-block major: consecutive items share a resident weight set
+        // channel-block major: consecutive items share a resident weight set; a task's block
+        // rows are split evenly over ceil(nby / mb) items (9 rows at mb = 8 give 5 + 4, not
+        // 8 + 1, whose 1-block item would pay a whole item's fixed cost for little work)
+        const int n_rows = ceil_div(tk.nby, st.mb);
         for (int nb = 0; nb < st.n_nblk; ++nb)
-            for (int by = 0; by < tk.nby; by += st.mb)
+            for (int ri = 0; ri < n_rows; ++ri)
                 for (int bx = 0; bx < tk.nbx; ++bx) {
+                    const int by = ri * tk.nby / n_rows, by_end = (ri + 1) * tk.nby / n_rows;
                     MafatItemDev it{};
                     it.task = ti;
                     it.by = (int16_t)by;
-                    it.nbk = (int16_t)std::min(st.mb, tk.nby - by);
+                    it.nbk = (int16_t)(by_end - by);
                     it.bx = (int16_t)bx;
                     it.nb = (int16_t)nb;
                     it.flags = (ti == cfg.unpublished_task) ? 1 : 0;
