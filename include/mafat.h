@@ -166,10 +166,14 @@ mafat_status mafat_run(const mafat_plan_t* plan, const void* input, void* output
 mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* cut_out,
                              void* output, void* stream);
 
-/* End-to-end call on HOST buffers (same layouts as mafat_run): copies the input
- * to plan-owned device memory, runs, copies the output back and synchronises
- * `stream`; returns the device status as mafat_sync_status does.  Pinned host
- * memory gives asynchronous copies. */
+/* End-to-end call on HOST buffers.  input_host is the image batch as it comes,
+ * NHWC [batch][H][W][C] in the plan's dtype (C = the net's input channels, no
+ * padding); output_host is NHWC [batch][H_out][W_out][C_out] as for mafat_run.
+ * Copies the input to plan-owned device memory, converts it there to the
+ * octet-planar layout mafat_run reads (one small kernel), runs, copies the
+ * output back and synchronises `stream`; returns the device status as
+ * mafat_sync_status does.  Pinned host memory gives asynchronous copies.
+ * Allocates the plan's staging buffers on its first call. */
 mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, void* output_host,
                             void* stream);
 

@@ -229,6 +229,8 @@ class Plan:
         _check(lib.mafat_run_fp32_noalloc(self.handle, _ptr(inp), _ptr(out), _stream(stream, inp)))
 
     def run_host(self, inp_host, out_host, stream=None):
+        """End to end on host tensors: inp_host NHWC [B][H][W][C] (the image batch as it
+        comes, pinned for asynchronous copies), out_host NHWC; synchronises the stream."""
         _check(lib.mafat_run_host(self.handle, _ptr(inp_host), _ptr(out_host), _stream(stream)))
 
     def sync_status(self, stream=None, like=None):

@@ -118,6 +118,55 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
 
 }  // namespace
 
+namespace {
+// One thread per (frame, octet, y, x), x fastest, so that the 8-element writes of a
+// warp are contiguous; channels at or above c are written as zero.
+template <typename T>
+__global__ void __launch_bounds__(256) to_planar_kernel(const T* __restrict__ in, T* __restrict__ out, int frames,
+                                                        int h, int w, int c, int c8) {
+    const int64_t total = (int64_t)frames * c8 * h * w;
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int x = (int)(idx % w);
+    int64_t r = idx / w;
+    const int y = (int)(r % h);
+    r /= h;
+    const int o = (int)(r % c8);
+    const int f = (int)(r / c8);
+    const T* src = in + (((int64_t)f * h + y) * w + x) * c;
+    T v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int ch = o * 8 + k;
+        v[k] = ch < c ? src[ch] : T(0);
+    }
+    T* dst = out + idx * 8;  // [f][o][y][x][8] in idx order, 16-byte aligned
+    if constexpr (sizeof(T) == 2) {
+        uint4 q;
+        q.x = (uint32_t)v[0] | ((uint32_t)v[1] << 16);
+        q.y = (uint32_t)v[2] | ((uint32_t)v[3] << 16);
+        q.z = (uint32_t)v[4] | ((uint32_t)v[5] << 16);
+        q.w = (uint32_t)v[6] | ((uint32_t)v[7] << 16);
+        *reinterpret_cast<uint4*>(dst) = q;
+    } else {
+        reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+        reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    }
+}
+}  // namespace
+
+cudaError_t mafat_launch_to_planar(const void* nhwc, void* planar, int frames, int h, int w, int c, int c8,
+                                   int elem_bytes, cudaStream_t s) {
+    const int64_t total = (int64_t)frames * c8 * h * w;
+    if (total <= 0) return cudaSuccess;
+    const unsigned grid = (unsigned)((total + 255) / 256);
+    if (elem_bytes == 2)
+        to_planar_kernel<uint16_t><<<grid, 256, 0, s>>>((const uint16_t*)nhwc, (uint16_t*)planar, frames, h, w, c, c8);
+    else
+        to_planar_kernel<float><<<grid, 256, 0, s>>>((const float*)nhwc, (float*)planar, frames, h, w, c, c8);
+    return cudaGetLastError();
+}
+
 cudaError_t mafat_launch_fp32(const MafatKParams& p, int grid, cudaStream_t s) {
     mafat_fp32_kernel<<<grid, 128, 0, s>>>(p);
     return cudaGetLastError();

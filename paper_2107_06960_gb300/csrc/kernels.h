@@ -41,6 +41,10 @@ cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, in
 size_t mafat_tc_smem_bytes();
 // fp32 CUDA-core check kernel: same work list, same scheduler.
 cudaError_t mafat_launch_fp32(const MafatKParams& p, int grid, cudaStream_t s);
+// NHWC [frames][h][w][c] -> octet-planar [frames][c8][h][w][8] (padded channels zero),
+// for element sizes of 2 (bf16) or 4 (fp32) bytes.
+cudaError_t mafat_launch_to_planar(const void* nhwc, void* planar, int frames, int h, int w, int c, int c8,
+                                   int elem_bytes, cudaStream_t s);
 // Diagnostic single-MMA kernel.
 cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int lbo_is_k,
                                    cudaStream_t s);

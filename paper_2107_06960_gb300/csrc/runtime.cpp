@@ -50,6 +50,7 @@ struct mafat_plan_s {
     // staging for mafat_run_host
     void* d_in_stage = nullptr;
     void* d_out_stage = nullptr;
+    void* d_in_nhwc = nullptr;   // the NHWC image batch as copied from the host
     std::mutex mu;
 };
 
@@ -113,7 +114,8 @@ void free_plan_memory(mafat_plan_s* p) {
     p->allocs.clear();
     if (p->d_in_stage) cudaFree(p->d_in_stage);
     if (p->d_out_stage) cudaFree(p->d_out_stage);
-    p->d_in_stage = p->d_out_stage = nullptr;
+    if (p->d_in_nhwc) cudaFree(p->d_in_nhwc);
+    p->d_in_stage = p->d_out_stage = p->d_in_nhwc = nullptr;
 }
 
 template <class T>
@@ -463,12 +465,18 @@ mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, vo
     {
         std::lock_guard<std::mutex> lk(p->mu);
         cudaError_t e;
+        const mafat::Layer& L0 = p->shapes.layers[0];
+        const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
         if (!p->d_in_stage) {
             if ((e = cudaMalloc(&p->d_in_stage, p->in_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
             if ((e = cudaMalloc(&p->d_out_stage, p->out_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+            if ((e = cudaMalloc(&p->d_in_nhwc, nhwc_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
         }
-        if ((e = cudaMemcpyAsync(p->d_in_stage, input_host, p->in_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        if ((e = cudaMemcpyAsync(p->d_in_nhwc, input_host, nhwc_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
             return cuda_fail(e, "cudaMemcpyAsync");
+        if ((e = mafat_launch_to_planar(p->d_in_nhwc, p->d_in_stage, p->t.cfg.batch, L0.h_in, L0.w_in, L0.c_in,
+                                        p->t.in_c8, (int)p->esz, s)) != cudaSuccess)
+            return cuda_fail(e, "layout conversion launch");
         mafat_status st = launch(p, p->d_in_stage, p->d_out_stage, s);
         if (st != MAFAT_OK) return st;
         if ((e = cudaMemcpyAsync(output_host, p->d_out_stage, p->out_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)

@@ -210,8 +210,29 @@ def test_run_host_matches_device_run(mf):
     out_dev = torch.empty((1, 38, 38, 256), dtype=torch.bfloat16, device="cuda")
     plan.run(xin.cuda(), out_dev)
     plan.sync_status(like=out_dev)
-    xh = xin.pin_memory()
+    # the host call takes the image as it comes (NHWC, 3 channels) and converts on the device
+    xh = torch.from_numpy(wl["input"]).to(torch.bfloat16).pin_memory()
     oh = torch.empty((1, 38, 38, 256), dtype=torch.bfloat16).pin_memory()
+    plan.run_host(xh, oh)
+    assert torch.equal(oh, out_dev.cpu())
+    plan.run_host(xh, oh)  # staging buffers reused
+    assert torch.equal(oh, out_dev.cpu())
+
+
+def test_run_host_fp32_matches_device_run(mf):
+    import torch
+    from tests.gpu_util import to_planar
+    wl = synth.workload("tiny3_64_fp32")
+    net = mf.Net(wl["layers"], wl["h"], wl["w"], 3)
+    net.set_params(wl["params"])
+    plan = mf.Plan(net, wl["cut"], wl["grids"], batch=wl["batch"], dtype=mf.FP32)
+    sh = net.shape(len(wl["layers"]) - 1)
+    xin = torch.from_numpy(to_planar(wl["input"])).float()
+    out_dev = torch.empty((wl["batch"], sh[3], sh[4], sh[5]), dtype=torch.float32, device="cuda")
+    plan.run(xin.cuda(), out_dev)
+    plan.sync_status(like=out_dev)
+    xh = torch.from_numpy(wl["input"]).float().contiguous()
+    oh = torch.empty(out_dev.shape, dtype=torch.float32)
     plan.run_host(xh, oh)
     assert torch.equal(oh, out_dev.cpu())
 
