@@ -263,19 +263,31 @@ def main():
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     dev_s = sum(step_ms) / 1e3
 
-    # end to end through the C ABI on pinned host buffers (copies inside the timed region)
+    # End to end through the C ABI on pinned host buffers, every step's upload of its
+    # input and read-back of its output inside the timed region.  Streamed the way a
+    # serving loop would (mafat_run_host_async: the upload of one frame overlaps the run
+    # of the previous one); the synchronous call's rate is reported beside it.
     xh = torch.from_numpy(wl["input"]).to(tdt).pin_memory()   # NHWC image batch as it comes
-    oh = torch.empty(out.shape, dtype=tdt).pin_memory()
+    ohs = [torch.empty(out.shape, dtype=tdt).pin_memory() for _ in range(2)]
+    oh = ohs[0]
+    for i in range(4):
+        plan.run_host_async(xh, ohs[i % 2], stream=stream)
+    plan.run_host_wait()
+    e2e_steps = max(5, min(args.steps, 200))
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        plan.run_host_async(xh, ohs[i % 2], stream=stream)
+    plan.run_host_wait()
+    e2e_s = time.perf_counter() - t0
     for _ in range(2):
         plan.run_host(xh, oh, stream=stream)
-    torch.cuda.synchronize()
-    e2e_steps = max(5, min(args.steps, 50))
+    sync_steps = max(5, min(args.steps, 50))
     t0 = time.perf_counter()
-    for _ in range(e2e_steps):
+    for _ in range(sync_steps):
         plan.run_host(xh, oh, stream=stream)
-    e2e_s = time.perf_counter() - t0
+    sync_s = time.perf_counter() - t0
 
-    dev_s_max, e2e_s_max = reduce_max(pg, [dev_s, e2e_s], dev)
+    dev_s_max, e2e_s_max, sync_s_max = reduce_max(pg, [dev_s, e2e_s, sync_s], dev)
     if rank != 0:
         if pg:
             pg.destroy_process_group()
@@ -310,6 +322,7 @@ def main():
             "workload": args.workload, "input": "%dx%dx3" % (H, W), "batch": B,
             "cut": wl["cut"], "grids": "/".join("%dx%d" % tuple(gd) for gd in wl["grids"]),
             "l2": "flushed before every timed step (256 MiB write, not timed)",
+            "e2e_l2": "not flushed between streamed frames (a serving loop keeps the 6.9 MB of weights in L2)",
             "useful_gflop_per_frame": st["useful_flops"] / B / 1e9,
             "executed_gflop_per_frame": st["executed_flops"] / B / 1e9,
             "halo_recompute": st["executed_flops"] / st["useful_flops"] - 1.0,
@@ -325,7 +338,9 @@ def main():
                      "kernel": "mafat_tc_kernel", "flops": "useful (unfused network) per launch",
                      "peak_source": "%s dense bf16 burst" % peak_src},
         "e2e": {"value": e2e_value, "unit": "frames/s", "h2d_bytes_per_step": int(xh.numel() * xh.element_size()),
-                "d2h_bytes_per_step": int(oh.numel() * oh.element_size())},
+                "d2h_bytes_per_step": int(oh.numel() * oh.element_size()),
+                "mode": "mafat_run_host_async, two frames in flight, copies in the timed region",
+                "sync_call_value": aggregate([B * sync_steps] * ws, [sync_s_max])},
         "gpu_launches": args.steps * plan.launches_per_run(),
         "clocks": clk,
     }

@@ -177,6 +177,22 @@ mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* 
 mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, void* output_host,
                             void* stream);
 
+/* Frames in flight on HOST buffers: the asynchronous form of mafat_run_host
+ * (same layouts).  Enqueues the input upload on a plan-owned copy stream, the
+ * layout conversion and the run on `stream`, and the read-back of the output on a
+ * second plan-owned copy stream, then returns; two staging slots alternate, so
+ * the upload of one frame overlaps the run of the one before.  input_host must
+ * stay unchanged, and output_host unread, until mafat_run_host_wait returns (or
+ * until the frame after next has been enqueued, for the input).  Runs on one plan
+ * still execute one after another.  Allocates the slots, streams and events on
+ * its first call.  Launch errors only; device status via mafat_run_host_wait. */
+mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_host, void* output_host,
+                                  void* stream);
+
+/* Wait until every frame enqueued by mafat_run_host_async has its output in host
+ * memory; returns the device status as mafat_sync_status does. */
+mafat_status mafat_run_host_wait(const mafat_plan_t* plan);
+
 /* Synchronise `stream` and read (and clear) the plan's device status word:
  * MAFAT_OK, MAFAT_ETIMEOUT (a tile waited on another that never finished) or
  * MAFAT_EDEVICE. */

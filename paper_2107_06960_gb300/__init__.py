@@ -56,6 +56,8 @@ _SIGNATURES = [
     ("mafat_run", i32, [vp, vp, vp, vp]),
     ("mafat_run_debug", i32, [vp, vp, vp, vp, vp]),
     ("mafat_run_host", i32, [vp, vp, vp, vp]),
+    ("mafat_run_host_async", i32, [vp, vp, vp, vp]),
+    ("mafat_run_host_wait", i32, [vp]),
     ("mafat_sync_status", i32, [vp, vp]),
     ("mafat_tile_region", i32, [vp, i32, i32, i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_net_tile_region", i32, [vp, i32, i32, i32, i32, i32, i32, i32, ctypes.POINTER(i32),
@@ -232,6 +234,15 @@ class Plan:
         """End to end on host tensors: inp_host NHWC [B][H][W][C] (the image batch as it
         comes, pinned for asynchronous copies), out_host NHWC; synchronises the stream."""
         _check(lib.mafat_run_host(self.handle, _ptr(inp_host), _ptr(out_host), _stream(stream)))
+
+    def run_host_async(self, inp_host, out_host, stream=None):
+        """Enqueue one frame on host tensors (two frames in flight); inp_host must stay
+        unchanged and out_host unread until run_host_wait returns."""
+        _check(lib.mafat_run_host_async(self.handle, _ptr(inp_host), _ptr(out_host), _stream(stream)))
+
+    def run_host_wait(self):
+        """Wait for every enqueued frame's output to reach host memory; raises on device errors."""
+        _check(lib.mafat_run_host_wait(self.handle))
 
     def sync_status(self, stream=None, like=None):
         """Raises MafatError (ETIMEOUT / EDEVICE) if a device-side wait ran out."""

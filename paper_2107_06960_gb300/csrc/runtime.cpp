@@ -51,6 +51,16 @@ struct mafat_plan_s {
     void* d_in_stage = nullptr;
     void* d_out_stage = nullptr;
     void* d_in_nhwc = nullptr;   // the NHWC image batch as copied from the host
+    // two staging slots of mafat_run_host_async (frames in flight), its copy streams
+    struct HostSlot {
+        void* d_nhwc = nullptr;
+        void* d_planar = nullptr;
+        void* d_out = nullptr;
+        cudaEvent_t h2d_done = nullptr, compute_done = nullptr, d2h_done = nullptr;
+        bool used = false;
+    } hs[2];
+    int hs_next = 0, hs_last = -1;
+    cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
     std::mutex mu;
 };
 
@@ -116,6 +126,19 @@ void free_plan_memory(mafat_plan_s* p) {
     if (p->d_out_stage) cudaFree(p->d_out_stage);
     if (p->d_in_nhwc) cudaFree(p->d_in_nhwc);
     p->d_in_stage = p->d_out_stage = p->d_in_nhwc = nullptr;
+    for (auto& h : p->hs) {
+        if (h.d_nhwc) cudaFree(h.d_nhwc);
+        if (h.d_planar) cudaFree(h.d_planar);
+        if (h.d_out) cudaFree(h.d_out);
+        if (h.h2d_done) cudaEventDestroy(h.h2d_done);
+        if (h.compute_done) cudaEventDestroy(h.compute_done);
+        if (h.d2h_done) cudaEventDestroy(h.d2h_done);
+        h = mafat_plan_s::HostSlot{};
+    }
+    if (p->s_h2d) cudaStreamDestroy(p->s_h2d);
+    if (p->s_d2h) cudaStreamDestroy(p->s_d2h);
+    p->s_h2d = p->s_d2h = nullptr;
+    p->hs_last = -1;
 }
 
 template <class T>
@@ -440,6 +463,74 @@ mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* 
         if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
     }
     return MAFAT_OK;
+}
+
+mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_host, void* output_host,
+                                  void* stream) {
+    if (!plan || !input_host || !output_host) return fail(MAFAT_EINVAL, "null argument");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    cudaStream_t s = (cudaStream_t)stream;
+    std::lock_guard<std::mutex> lk(p->mu);
+    cudaError_t e;
+    const mafat::Layer& L0 = p->shapes.layers[0];
+    const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
+    if (!p->s_h2d) {
+        if ((e = cudaStreamCreateWithFlags(&p->s_h2d, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaStreamCreateWithFlags(&p->s_d2h, cudaStreamNonBlocking)) != cudaSuccess)
+            return cuda_fail(e, "cudaStreamCreate");
+        for (auto& h : p->hs) {
+            if ((e = cudaMalloc(&h.d_nhwc, nhwc_bytes)) != cudaSuccess ||
+                (e = cudaMalloc(&h.d_planar, p->in_bytes)) != cudaSuccess ||
+                (e = cudaMalloc(&h.d_out, p->out_bytes)) != cudaSuccess)
+                return cuda_fail(e, "cudaMalloc");
+            if ((e = cudaEventCreateWithFlags(&h.h2d_done, cudaEventDisableTiming)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&h.compute_done, cudaEventDisableTiming)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&h.d2h_done, cudaEventDisableTiming)) != cudaSuccess)
+                return cuda_fail(e, "cudaEventCreate");
+        }
+    }
+    const int k = p->hs_next;
+    mafat_plan_s::HostSlot& h = p->hs[k];
+    // upload into slot k once the run that last read it is done
+    if (h.used && (e = cudaStreamWaitEvent(p->s_h2d, h.compute_done, 0)) != cudaSuccess)
+        return cuda_fail(e, "cudaStreamWaitEvent");
+    if ((e = cudaMemcpyAsync(h.d_nhwc, input_host, nhwc_bytes, cudaMemcpyHostToDevice, p->s_h2d)) != cudaSuccess ||
+        (e = cudaEventRecord(h.h2d_done, p->s_h2d)) != cudaSuccess)
+        return cuda_fail(e, "upload");
+    // run on the caller's stream once the upload landed and slot k's last result was read back
+    if ((e = cudaStreamWaitEvent(s, h.h2d_done, 0)) != cudaSuccess ||
+        (h.used && (e = cudaStreamWaitEvent(s, h.d2h_done, 0)) != cudaSuccess))
+        return cuda_fail(e, "cudaStreamWaitEvent");
+    if ((e = mafat_launch_to_planar(h.d_nhwc, h.d_planar, p->t.cfg.batch, L0.h_in, L0.w_in, L0.c_in, p->t.in_c8,
+                                    (int)p->esz, s)) != cudaSuccess)
+        return cuda_fail(e, "layout conversion launch");
+    mafat_status st = launch(p, h.d_planar, h.d_out, s);
+    if (st != MAFAT_OK) return st;
+    if ((e = cudaEventRecord(h.compute_done, s)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    // read the result back on its own stream
+    if ((e = cudaStreamWaitEvent(p->s_d2h, h.compute_done, 0)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(output_host, h.d_out, p->out_bytes, cudaMemcpyDeviceToHost, p->s_d2h)) != cudaSuccess ||
+        (e = cudaEventRecord(h.d2h_done, p->s_d2h)) != cudaSuccess)
+        return cuda_fail(e, "download");
+    h.used = true;
+    p->hs_last = k;
+    p->hs_next = k ^ 1;
+    return MAFAT_OK;
+}
+
+mafat_status mafat_run_host_wait(const mafat_plan_t* plan) {
+    if (!plan) return fail(MAFAT_EINVAL, "null plan");
+    mafat_plan_s* p = const_cast<mafat_plan_s*>(plan);
+    if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
+    {
+        std::lock_guard<std::mutex> lk(p->mu);
+        if (p->hs_last < 0) return MAFAT_OK;
+        // read-backs run in order on one stream: the last one done means all are
+        cudaError_t e = cudaEventSynchronize(p->hs[p->hs_last].d2h_done);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+    }
+    return mafat_sync_status(plan, p->s_d2h);
 }
 
 mafat_status mafat_sync_status(const mafat_plan_t* plan, void* stream) {

@@ -219,6 +219,30 @@ def test_run_host_matches_device_run(mf):
     assert torch.equal(oh, out_dev.cpu())
 
 
+def test_run_host_async_frames_in_flight_match_device_runs(mf):
+    import torch
+    from tests.gpu_util import to_planar
+    wl = synth.workload("yolo16_416_1x3x3")
+    net = mf.Net(wl["layers"], 416, 416, 3)
+    net.set_params(wl["params"])
+    plan = mf.Plan(net, None, wl["grids"], batch=1, dtype=mf.BF16)
+    frames = [synth.make_input(1, 416, 416, 3, 100 + i) for i in range(3)]
+    ref = []
+    for x in frames:
+        out = torch.empty((1, 26, 26, 256), dtype=torch.bfloat16, device="cuda")
+        plan.run(torch.from_numpy(to_planar(x)).to(torch.bfloat16).cuda(), out)
+        plan.sync_status(like=out)
+        ref.append(out.cpu())
+    xh = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in frames]
+    oh = [torch.empty((1, 26, 26, 256), dtype=torch.bfloat16).pin_memory() for _ in frames]
+    for i in range(3):  # three frames enqueued back to back over the two staging slots
+        plan.run_host_async(xh[i], oh[i])
+    plan.run_host_wait()
+    for i in range(3):
+        assert torch.equal(oh[i], ref[i]), i
+    plan.run_host_wait()  # nothing in flight: returns at once
+
+
 def test_run_host_fp32_matches_device_run(mf):
     import torch
     from tests.gpu_util import to_planar
