@@ -147,6 +147,21 @@ def test_bf16_yolo16_96_batch2(mf, cut, grids):
     _check_groups(c, out, refs, cut, TOL_BF16)
 
 
+@pytest.mark.parametrize("cut,grids", [(8, [(3, 3), (2, 2)]), (4, [(2, 2), (2, 1)]), (None, [(2, 2)])])
+def test_bf16_smallest_map_batch3(mf, cut, grids):
+    # 32x32 input: the 16-layer net ends at 2x2, group 1 at cut 8 ends at 4x4, so tiles
+    # shrink to one or two pixels; three frames in one launch
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, synth.SEED_BASE + 80, "bf16")
+    x = synth.make_input(3, 32, 32, 3, synth.SEED_BASE + 80, "bf16")
+    c, out = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
+    for f in range(3):
+        refs = oracle.group_outputs(layers, params, x[f], cut)
+        assert rel_err(out[f], refs[-1]) <= TOL_BF16
+        if cut is not None:
+            assert rel_err(c[f], refs[0]) <= TOL_BF16
+
+
 @pytest.mark.parametrize("name", ["yolo16_416_1x3x3", "yolo16_608_5x5_c8_2x2"])
 def test_bf16_full_size(mf, name):
     wl = synth.workload(name)
