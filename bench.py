@@ -193,6 +193,66 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """Plans of the 608x608 network over cut points and per-group grids (the paper's
+    configuration space, Sec. 4 and Table 1): device-timed frames/s with L2 flushed before
+    every step, Algorithm 1's prediction, the plan's intermediate bytes (tile scratch ring
+    plus cut tensor) and the halo recompute, one JSON line each."""
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    import paper_2107_06960_gb300 as mf
+    torch.cuda.set_device(0)
+    wl = synth.workload(DEFAULT_WORKLOAD)
+    H, W = wl["h"], wl["w"]
+    net = mf.Net(wl["layers"], H, W, 3)
+    net.set_params(wl["params"])
+    xin = torch.from_numpy(mf.to_planar(wl["input"])).to(torch.bfloat16).cuda()
+    sh = net.shape(len(wl["layers"]) - 1)
+    out = torch.empty((1, sh[3], sh[4], sh[5]), dtype=torch.bfloat16, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device="cuda")
+    configs = [(None, [(t, t)]) for t in synth.SWEEP_GRIDS]
+    configs += [(cut, [(t1, t1), (t2, t2)]) for cut in synth.SWEEP_CUTS
+                for t1 in synth.SWEEP_GRIDS for t2 in synth.SWEEP_GRIDS]
+    steps = max(20, min(args.steps, 200))
+    best = None
+    for cut, grids in configs:
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
+        plan = mf.Plan(net, cut, grids, batch=1, dtype=mf.BF16)
+        st = plan.stats()
+        torch.cuda.synchronize()
+        plan_bytes = free0 - torch.cuda.mem_get_info()[0]
+        for _ in range(3):
+            plan.run(xin, out)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in ev:
+            flush.fill_(1)
+            a.record()
+            plan.run(xin, out)
+            b.record()
+        torch.cuda.synchronize()
+        plan.sync_status(like=out)
+        times = [a.elapsed_time(b) for a, b in ev]
+        ms = statistics.fmean(times)
+        cut_bytes = 0
+        if cut is not None:
+            c = net.shape(cut - 1)
+            cut_bytes = (c[5] + 7) // 8 * 8 * c[3] * c[4] * 2
+        line = {"sweep": True, "cut": cut, "grids": "/".join("%dx%d" % gd for gd in grids),
+                "frames_per_s": 1e3 / ms, "ms_mean": ms, "ms_median": statistics.median(times), "steps": steps,
+                "predicted_mib_alg1": st["predicted_mib"],
+                "intermediate_mb": (st["scratch_bytes"] + cut_bytes) / 1e6,
+                "plan_device_mb": plan_bytes / 1e6,
+                "executed_gflop": st["executed_flops"] / 1e9,
+                "halo_recompute": st["executed_flops"] / st["useful_flops"] - 1.0, "work_items": st["n_items"]}
+        print(json.dumps(line), flush=True)
+        if best is None or ms < best["ms_mean"]:
+            best = line
+        plan.close()
+    print(json.dumps({"sweep_best": best}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -201,6 +261,9 @@ def main():
     ap.add_argument("--impl", default="mafat", choices=["mafat", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time every plan of the 608x608 net over cuts {none, 2, 4, 8, 12} x grids 1..5 per "
+                         "group (one JSON line per plan, then the fastest), instead of the benchmark line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -208,6 +271,9 @@ def main():
 
     if args.impl == "reference":
         run_reference(args, wl)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
 
     import torch

@@ -200,14 +200,23 @@ def test_bf16_608_plan_sweep_is_plan_independent(mf):
                 assert np.array_equal(out, base), "plan %d/%dx%d/%dx%d differs" % (cut, t1, t1, t2, t2)
 
 
-@pytest.mark.parametrize("cut,t1,t2", [(2, 1, 2), (4, 3, 3), (8, 5, 2), (8, 2, 5), (12, 4, 1), (12, 5, 5)])
-def test_bf16_608_sweep_default_shapes(mf, cut, t1, t2):
-    # the default per-stage MMA shapes depend on the plan; results stay within tolerance
+def test_bf16_608_every_sweep_plan_default_shapes(mf):
+    # every plan the benchmark's sweep times (one group with grids 1..5, and cut after
+    # layer 1, 3, 7, 11 x per-group grids 1..5), with the MMA shapes the planner picks for
+    # it: the cut tensor and the output within tolerance of one layer-by-layer oracle pass
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     layers, params, x = wl["layers"], wl["params"], wl["input"]
-    refs = _oracle_groups(layers, params, x, 8, "yolo16_608_5x5_c8_2x2")
-    _, out = run_plan(mf, layers, params, x, cut, [(t1, t1), (t2, t2)], mf.BF16)
-    assert rel_err(out[0], refs[0][-1]) <= TOL_BF16
+    outs = oracle.forward(layers, params, x[0])
+    plans = [(None, [(t, t)]) for t in synth.SWEEP_GRIDS]
+    plans += [(cut, [(t1, t1), (t2, t2)]) for cut in synth.SWEEP_CUTS
+              for t1 in synth.SWEEP_GRIDS for t2 in synth.SWEEP_GRIDS]
+    for cut, grids in plans:
+        c, out = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
+        e = rel_err(out[0], outs[-1])
+        assert e <= TOL_BF16, "plan %s %s output: rel err %.3g" % (cut, grids, e)
+        if cut is not None:
+            e = rel_err(c[0], outs[cut - 1])
+            assert e <= TOL_BF16, "plan %s %s cut tensor: rel err %.3g" % (cut, grids, e)
 
 
 # ---------------------------------------------------------------------------
