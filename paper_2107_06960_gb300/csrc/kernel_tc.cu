@@ -28,12 +28,17 @@
 //    it, larger sets stream piece by piece (every copy costs a few hundred cycles
 //    of TMA time however small it is, so copies are large and few).
 //
-// Warp roles (320 threads): warps 0-7 epilogue (warp w reads TMEM lanes
+// Warp roles (352 threads): warps 0-7 epilogue (warp w reads TMEM lanes
 // 32(w%4)..+31 = conv rows 4(w%4)..+3 of a block; the two warpgroups take units
 // of one block x 32 columns in turn), warp 8 scheduler + TMA producer, warp 9 TMEM
-// allocator + MMA issuer.  Shared memory: 2 A halo stages, 2 weight buffers and
-// a 4-deep queue of item indices; TMEM: 2 accumulators of 256 columns (the
-// epilogue of one item overlaps the MMAs of the next).
+// allocator + MMA issuer, warp 10 publisher (bumps an item's completion counter
+// once all epilogue threads have stored it, so that the epilogue warps never wait
+// for their stores to reach L2).  Shared memory: 2 A halo stages, 2 weight
+// buffers, a 4-deep queue of items with the record the epilogue needs (written by
+// the producer, so the epilogue reads no work table from global memory), and one
+// scale / bias slot per accumulator (copied in by the MMA warp and landing on the
+// accumulator's full barrier); TMEM: 2 accumulators of 256 columns (the epilogue
+// of one item overlaps the MMAs of the next).
 //
 // Epilogue: y = leaky_0.1(scale[n] * acc + bias[n]); for a fused 2x2/s2
 // max-pool the quad of pixels {(r, c), (r, c+1), (r+1, c), (r+1, c+1)} are lanes
@@ -55,7 +60,8 @@ constexpr int kEpiWarps = 4 * kEpiGroups;
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kProducerWarp = kEpiWarps;
 constexpr int kMmaWarp = kEpiWarps + 1;
-constexpr int kThreads = (kEpiWarps + 2) * 32;
+constexpr int kPubWarp = kEpiWarps + 2;
+constexpr int kThreads = (kEpiWarps + 3) * 32;
 constexpr int kAStages = 2;
 constexpr int kQDepth = 4;
 constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;   // one A halo box, multiple of 1024
@@ -73,15 +79,22 @@ constexpr int kBarAccEmpty = kBarAccFull + 2;
 constexpr int kBarQFull = kBarAccEmpty + 2;
 constexpr int kBarQEmpty = kBarQFull + kQDepth;
 constexpr int kBarDone = kBarQEmpty + kQDepth;
-constexpr int kNumBars = kBarDone + 1;
-constexpr int kOffQItems = 512;
+constexpr int kBarEpiDone = kBarDone + 1;          // every epilogue thread has stored item e (slot e % 2)
+constexpr int kBarPubDone = kBarEpiDone + 2;       // the publisher has published item e (slot e % 2)
+constexpr int kNumBars = kBarPubDone + 2;
+constexpr int kOffRec = 256;                        // kQDepth epilogue records
+constexpr int kRecStride = 128;
+constexpr int kOffQItems = kOffRec + kQDepth * kRecStride;
 constexpr int kOffTmem = kOffQItems + 4 * kQDepth;
 constexpr int kOffBroken = kOffTmem + 4;
 constexpr int kOffA = 1024;
 constexpr int kOffB = kOffA + kAStages * kAStageBytes;
-constexpr int kSmemUsed = kOffB + 2 * kBPieceBytes;
+constexpr int kSbSlotBytes = 2 * MAFAT_MAX_NBLK * 4;  // scale then bias of one item's channels
+constexpr int kOffSb = kOffB + 2 * kBPieceBytes;
+constexpr int kSmemUsed = kOffSb + 2 * kSbSlotBytes;
 constexpr int kSmemBytes = kSmemUsed + 1024;  // slack for aligning the base
-static_assert(kNumBars * 8 <= kOffQItems, "barrier area");
+static_assert(kNumBars * 8 <= kOffRec, "barrier area");
+static_assert(kOffBroken + 4 <= kOffA, "queue area");
 static_assert(kSmemBytes <= 232448, "shared memory");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -94,6 +107,11 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Adds bytes to the current phase's expected transactions without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
@@ -307,28 +325,34 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&v)[64]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
-        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, "
-        "%36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, "
-        "%57, %58, %59, %60, %61, %62, %63}, [%64];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
-          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
-          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31]),
-          "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]), "=r"(v[37]), "=r"(v[38]), "=r"(v[39]),
-          "=r"(v[40]), "=r"(v[41]), "=r"(v[42]), "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]),
-          "=r"(v[48]), "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]), "=r"(v[55]),
-          "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]), "=r"(v[61]), "=r"(v[62]), "=r"(v[63])
-        : "r"(taddr)
-        : "memory");
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
 // Where one thread's epilogue results go: its pixel's element offset in the
 // output buffer (octet-planar: offset inside an 8-channel plane; NHWC: offset
 // of channel 0), the plane stride, and whether this lane stores at all.
+// What the MMA issuer needs of an item (all small).
+struct MmaRec {
+    int16_t k, cols_box, rows_box, n_chunks, n_bsteps, bpp, n_pieces, kst, paired, b_swz, nbk, pad;
+    int32_t key;         // stage * 256 + channel block: identifies a resident weight set
+    int32_t blob_elems;  // elements of one weight blob
+    int32_t sb;          // offset of the item's first channel in the scale / bias arrays
+};
+
+// What the MMA issuer, the epilogue and the publisher need of an item, written into its
+// queue slot by the producer (which has the work tables in registers anyway), so that
+// none of them reads a work table from global memory on its critical path.
+struct EpiRec {
+    __nv_bfloat16* out;      // output buffer of the task (frame and tile offset applied)
+    int32_t x0, xlim;        // conv column of the item's block column; end of the task's columns
+    int32_t y0, ylim;        // conv row of the item's first block row; end of the task's rows
+    int32_t out_y0, out_x0;  // map position of output buffer pixel (0, 0)
+    int32_t out_w, out_h;    // output buffer extent (pixels, after pooling)
+    int32_t nbk, n_blk;      // blocks of the item; output channels per item (accumulator columns per block)
+    int32_t cout, ch_base;   // channels of the layer; first channel of the item
+    int32_t flags;           // bit 0: fused max-pool, bit 1: NHWC output, bit 2: never published (test hook)
+    int32_t done_ctr, extra_ctr;
+    MmaRec mma;
+};
+static_assert(sizeof(EpiRec) <= kRecStride, "item record");
+
 struct EpiDst {
     __nv_bfloat16* out;
     size_t pix, plane;
@@ -336,50 +360,86 @@ struct EpiDst {
     bool store;
 };
 
-// Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1) of one
-// pixel per thread: folded BN, leaky ReLU 0.1, bf16 (nearest-even), optional 2x2 max
-// over the quad lanes {l, l^1, l^8, l^9} on the packed bf16 pairs (rounding is
-// monotonic, so the max of rounded values is the rounded max), 16-byte stores per octet.
+// Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1, NC = 16 or 32)
+// of one pixel per thread: folded BN, leaky ReLU 0.1 (as max(z, 0.1 z), the same value),
+// bf16 (nearest-even), 16-byte stores per octet of channels.
+//
+// A fused 2x2 max-pool reduces the window {(r, c), (r, c+1), (r+1, c), (r+1, c+1)},
+// lanes {l, l^1, l^8, l^9}, on packed bf16 pairs (rounding is monotonic, so the max of
+// rounded values is the rounded max) in two exchange rounds that each halve the octets a
+// lane holds: with the partner lane^1, a lane keeps octets 2m + (l & 1) and sends the
+// others; with lane^8, it keeps every other remaining octet.  Every shuffle carries data
+// both lanes need, and each lane of the window ends with its own octet(s) of the pooled
+// pixel to store (two octets: both lanes l and l^8 end with the same one; one stores).
 template <int NC>
 __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const float* bi, int ch0,
-                                          const EpiDst& d) {
+                                          const EpiDst& d, int lane) {
+    static_assert(NC == 16 || NC == 32, "unit width");
+    constexpr int NO = NC / 8;  // octets
     uint32_t raw[NC];
-    if constexpr (NC == 64)
-        tmem_ld64(taddr, raw);
-    else if constexpr (NC == 32)
+    if constexpr (NC == 32)
         tmem_ld32(taddr, raw);
     else
         tmem_ld16(taddr, raw);
     uint32_t pk[NC / 2];
 #pragma unroll
     for (int i = 0; i < NC; i += 4) {
-        const float4 s4 = __ldg(reinterpret_cast<const float4*>(sc + i));
-        const float4 b4 = __ldg(reinterpret_cast<const float4*>(bi + i));
+        const float4 s4 = *reinterpret_cast<const float4*>(sc + i);  // shared memory, same address
+        const float4 b4 = *reinterpret_cast<const float4*>(bi + i);  // for the whole warp
         const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
         float v[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            const float z = sv[u] * __uint_as_float(raw[i + u]) + bv[u];
-            v[u] = z > 0.f ? z : 0.1f * z;
+            const float z = fmaf(sv[u], __uint_as_float(raw[i + u]), bv[u]);
+            v[u] = fmaxf(z, 0.1f * z);
         }
         pk[i / 2] = pack_bf16x2(v[0], v[1]);
         pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
     }
-    if (d.pool) {
+    if (!d.pool) {
+        if (!d.store) return;
 #pragma unroll
-        for (int i = 0; i < NC / 2; ++i) {
-            pk[i] = max_bf16x2(pk[i], __shfl_xor_sync(0xffffffffu, pk[i], 1));
-            pk[i] = max_bf16x2(pk[i], __shfl_xor_sync(0xffffffffu, pk[i], 8));
+        for (int o = 0; o < NO; ++o) {
+            const int ch = ch0 + 8 * o;
+            if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
+            const uint4 w = make_uint4(pk[4 * o], pk[4 * o + 1], pk[4 * o + 2], pk[4 * o + 3]);
+            __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+            *reinterpret_cast<uint4*>(p) = w;
         }
+        return;
     }
-    if (!d.store) return;
+    const bool h0 = (lane & 1) != 0, h3 = (lane & 8) != 0;
+    // round 1, partner lane ^ 1: keep octet 2m + h0 of each pair (2m, 2m + 1)
+    uint32_t r1[NC / 4];
 #pragma unroll
-    for (int o = 0; o < NC / 8; ++o) {
-        const int ch = ch0 + 8 * o;
-        if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
-        const uint4 w = make_uint4(pk[4 * o], pk[4 * o + 1], pk[4 * o + 2], pk[4 * o + 3]);
+    for (int m = 0; m < NO / 2; ++m)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t lo = pk[8 * m + j], hi = pk[8 * m + 4 + j];
+            const uint32_t got = __shfl_xor_sync(0xffffffffu, h0 ? lo : hi, 1);
+            r1[4 * m + j] = max_bf16x2(h0 ? hi : lo, got);
+        }
+    if constexpr (NO == 4) {
+        // round 2, partner lane ^ 8: keep octet 2 * h3 + h0
+        uint32_t r2[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t lo = r1[j], hi = r1[4 + j];
+            const uint32_t got = __shfl_xor_sync(0xffffffffu, h3 ? lo : hi, 8);
+            r2[j] = max_bf16x2(h3 ? hi : lo, got);
+        }
+        const int ch = ch0 + 8 * (2 * (int)h3 + (int)h0);
+        if (!d.store || ch >= d.cout) return;
         __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
-        *reinterpret_cast<uint4*>(p) = w;
+        *reinterpret_cast<uint4*>(p) = make_uint4(r2[0], r2[1], r2[2], r2[3]);
+    } else {
+        // two octets: round 2 is a plain max with lane ^ 8, and lanes with h3 set leave the store
+#pragma unroll
+        for (int j = 0; j < 4; ++j) r1[j] = max_bf16x2(r1[j], __shfl_xor_sync(0xffffffffu, r1[j], 8));
+        const int ch = ch0 + 8 * (int)h0;
+        if (!d.store || h3 || ch >= d.cout) return;
+        __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+        *reinterpret_cast<uint4*>(p) = make_uint4(r1[0], r1[1], r1[2], r1[3]);
     }
 }
 
@@ -478,7 +538,9 @@ __device__ __forceinline__ void mma_begin_piece(MmaState& s, MmaJob& j) {
 // B operand) and the paired-tap form (8 input channels, two taps per K step).  One
 // instance per shape keeps every blob's KST x NBK MMAs one straight run of code: on
 // GB300, MMAs separated by a runtime loop or a branch per MMA, or by a jump per blob into
-// a large switch, issued at half the tensor core's rate or worse.
+// a large switch, issued at half the tensor core's rate or worse; so does an MMA that
+// is issued predicated off (measured: a block-count-generic instance with absent
+// blocks' MMAs predicated off doubled the MMA time of one-block items).
 template <int KST, int NBK, bool PAIRED>
 __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     uint32_t accumulate = 0;
@@ -557,6 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int* q_items = reinterpret_cast<volatile int*>(smem + kOffQItems);
     volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + kOffTmem);
     volatile int* broken = reinterpret_cast<volatile int*>(smem + kOffBroken);
+    EpiRec* recs = reinterpret_cast<EpiRec*>(smem + kOffRec);
     auto bar = [&](int i) { return sbase + (uint32_t)(i * 8); };
 
     const int warp = threadIdx.x >> 5;
@@ -578,9 +641,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < kQDepth; ++i) {
             mbar_init(bar(kBarQFull + i), 1);
-            mbar_init(bar(kBarQEmpty + i), kEpiWarps + 1);
+            mbar_init(bar(kBarQEmpty + i), kEpiWarps + 2);  // epilogue warps, MMA warp, publisher
         }
         mbar_init(bar(kBarDone), 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(kBarEpiDone + i), kEpiThreads);
+            mbar_init(bar(kBarPubDone + i), 1);
+        }
         *broken = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -625,14 +692,54 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
                 }
+                MafatTaskDev tk;
+                MafatStageDev st;
+                if (ticket >= 0) {
+                    tk = p.tasks[it.task];
+                    st = p.stages[tk.stage];
+                }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                 q_items[qs] = ticket;
-                mbar_arrive(bar(kBarQFull + qs));
+                if (ticket >= 0) {
+                    EpiRec& rc = recs[qs];
+                    rc.out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
+                                              : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
+                                                                                : p.scratch) +
+                             tk.out_off;
+                    rc.x0 = tk.cx0 + it.bx * MAFAT_BLK_COLS;
+                    rc.xlim = tk.cx0 + tk.cw;
+                    rc.y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS;
+                    rc.ylim = tk.cy0 + tk.ch;
+                    rc.out_y0 = tk.out_y0;
+                    rc.out_x0 = tk.out_x0;
+                    rc.out_w = tk.out_w;
+                    rc.out_h = tk.out_h;
+                    rc.nbk = it.nbk;
+                    rc.n_blk = st.n_blk;
+                    rc.cout = st.cout;
+                    rc.ch_base = it.nb * st.n_blk;
+                    rc.flags = (st.pool ? 1 : 0) | (tk.out_nhwc ? 2 : 0) | ((it.flags & 1) ? 4 : 0);
+                    rc.done_ctr = tk.done_ctr;
+                    rc.extra_ctr = it.extra_ctr;
+                    rc.mma.k = (int16_t)st.k;
+                    rc.mma.cols_box = (int16_t)st.cols_box;
+                    rc.mma.rows_box = (int16_t)st.rows_box;
+                    rc.mma.n_chunks = (int16_t)st.n_chunks;
+                    rc.mma.n_bsteps = (int16_t)st.n_bsteps;
+                    rc.mma.bpp = (int16_t)st.bpp;
+                    rc.mma.n_pieces = (int16_t)st.n_pieces;
+                    rc.mma.kst = (int16_t)st.kst;
+                    rc.mma.paired = (int16_t)st.paired;
+                    rc.mma.b_swz = (int16_t)st.b_swz;
+                    rc.mma.nbk = it.nbk;
+                    rc.mma.key = tk.stage * 256 + it.nb;
+                    rc.mma.blob_elems = st.blob_elems;
+                    rc.mma.sb = st.sb_off + it.nb * st.n_blk;
+                }
+                mbar_arrive(bar(kBarQFull + qs));  // release: the record is visible to the consumers
                 ++q_cnt;
                 if (ticket < 0) break;
-                const MafatTaskDev tk = p.tasks[it.task];
-                const MafatStageDev st = p.stages[tk.stage];
                 const int key = tk.stage * 256 + it.nb;
                 const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
                 const uint32_t blob_bytes = (uint32_t)(st.blob_elems * 2);
@@ -722,32 +829,50 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait_mma(ms.bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
                 const int ticket = wu(q_items[qs]);
-                mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
+                MmaRec mr;
+                int n_blk = 0;
+                if (ticket >= 0) {
+                    mr = recs[qs].mma;
+                    n_blk = recs[qs].n_blk;
+                }
+                mbar_arrive_elect(ms.bar(kBarQEmpty + qs));  // release: the record has been read
                 ++q_cnt;
                 if (ticket < 0) break;
-                const MafatItemDev& it = p.items[ticket];
-                const MafatTaskDev& tk = p.tasks[it.task];
-                const MafatStageDev& st = p.stages[tk.stage];
                 MmaJob j;
                 j.ticket = ticket;
-                j.k = wu(st.k);
-                j.cols_box = wu(st.cols_box);
-                j.n_blk = (uint32_t)wu(st.n_blk);
-                j.n_chunks = wu(st.n_chunks);
-                j.n_bsteps = wu(st.n_bsteps);
-                j.bpp = wu(st.bpp);
-                j.P = wu(st.n_pieces);
+                j.k = wu(mr.k);
+                j.cols_box = wu(mr.cols_box);
+                j.n_blk = (uint32_t)wu(n_blk);
+                j.n_chunks = wu(mr.n_chunks);
+                j.n_bsteps = wu(mr.n_bsteps);
+                j.bpp = wu(mr.bpp);
+                j.P = wu(mr.n_pieces);
                 j.G = j.n_chunks * j.n_bsteps;
-                j.key = wu(tk.stage * 256 + it.nb);
-                j.blob_bytes = (uint32_t)wu(st.blob_elems * 2);
-                j.a_plane = (uint32_t)wu(st.rows_box * st.cols_box * 16);
-                j.bswz = wu(st.b_swz) != 0;
-                const int kst = wu(st.kst), nbk = wu(it.nbk), paired = wu(st.paired);
+                j.key = wu(mr.key);
+                j.blob_bytes = (uint32_t)wu(mr.blob_elems * 2);
+                j.a_plane = (uint32_t)wu(mr.rows_box * mr.cols_box * 16);
+                j.bswz = wu(mr.b_swz) != 0;
+                const int kst = wu(mr.kst), nbk = wu(mr.nbk), paired = wu(mr.paired);
+                const int sb = wu(mr.sb);
                 j.cur_b = j.P == 1 ? ms.wb.resident(j.key) : -1;
                 if (j.cur_b < 0) mma_begin_piece(ms, j);
                 const int buf = (int)(acc_cnt & 1u);
                 mbar_wait_mma(ms.bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
                 tc_fence_after();
+                {
+                    // the item's scale and bias go into the accumulator's slot (the epilogue of
+                    // the slot's previous item is past it); the accumulator's full barrier then
+                    // completes only once they have landed as well
+                    const uint32_t sb_bytes = j.n_blk * 4u;
+                    if (lane == 0) {
+                        const uint32_t fb = ms.bar(kBarAccFull + buf);
+                        const uint32_t slot = ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes);
+                        mbar_expect_tx(fb, 2u * sb_bytes);
+                        bulk_load(slot, p.scale + sb, sb_bytes, fb);
+                        bulk_load(slot + (uint32_t)(kSbSlotBytes / 2), p.bias + sb, sb_bytes, fb);
+                    }
+                    __syncwarp();
+                }
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
                 j.idesc = instr_desc_bf16((int)j.n_blk, 128);
                 j.a_row = (uint32_t)(j.cols_box * 16);
@@ -790,10 +915,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         __syncwarp();
+    } else if (warp == kPubWarp) {
+        // ------------------------------------------------------------ publisher (warp 10)
+        // An item is done once every epilogue thread has stored its share and fenced it
+        // for the async proxy, then arrived on the item's EpiDone slot (release, CTA
+        // scope).  The publisher's gpu-scope release reduction is cumulative over those
+        // arrivals, so a consumer that acquires the counter sees every store; waiting for
+        // the stores to reach L2 is this warp's job, not the epilogue warps'.
+        if (lane == 0) {
+            uint32_t q_cnt = 0, e_cnt = 0;
+            while (true) {
+                const int qs = (int)(q_cnt % kQDepth);
+                mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
+                const int ticket = q_items[qs];
+                int done_ctr = 0, extra_ctr = -1, flags = 0;
+                if (ticket >= 0) {
+                    done_ctr = recs[qs].done_ctr;
+                    extra_ctr = recs[qs].extra_ctr;
+                    flags = recs[qs].flags;
+                }
+                mbar_arrive(bar(kBarQEmpty + qs));
+                ++q_cnt;
+                if (ticket < 0) break;
+                const int es = (int)(e_cnt & 1u);
+                mbar_wait(bar(kBarEpiDone + es), (e_cnt >> 1) & 1u, p.ctr, pipe_limit, broken, 32);
+                if (!(flags & 4)) mafat_dev::publish_counters(p.ctr, done_ctr, extra_ctr);
+                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 3, mafat_dev::globaltimer_ns());
+                mbar_arrive(bar(kBarPubDone + es));
+                ++e_cnt;
+            }
+        }
+        __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue (warps 0-7)
         // Warp w reads TMEM lanes 32*(w%4) .. +31 (conv rows 4*(w%4) .. +3 of a block);
-        // the two warpgroups (h = w/4) split an item's blocks, or a single block's columns.
+        // the two warpgroups (h = w/4) take units of one block x 32 columns in turn.
         uint32_t q_cnt = 0, acc_cnt = 0;
         const int wq = warp & 3, h = warp >> 2;  // lane quarter, warpgroup
         const int r = wq * 4 + (lane >> 3);  // conv row within the block
@@ -802,71 +958,65 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int qs = (int)(q_cnt % kQDepth);
             mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
             const int ticket = q_items[qs];
+            EpiRec rc;
+            if (ticket >= 0) rc = recs[qs];
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
             ++q_cnt;
             if (ticket < 0) break;
-            const MafatItemDev it = p.items[ticket];
-            const MafatTaskDev tk = p.tasks[it.task];
-            const MafatStageDev st = p.stages[tk.stage];
             const int buf = (int)(acc_cnt & 1u);
+            // completes once the item's MMAs are done and its scale / bias have landed
             mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken, 128);
             if (p.trace && threadIdx.x == 0) mafat_dev::trace_put(p.trace, ticket, 2, mafat_dev::globaltimer_ns());
             __syncwarp();
             tc_fence_after();
 
-            __nv_bfloat16* out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
-                                                  : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
-                                                                                    : p.scratch) +
-                                 tk.out_off;
-            const float* sc = p.scale + st.sb_off + it.nb * st.n_blk;
-            const float* bi = p.bias + st.sb_off + it.nb * st.n_blk;
-            const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + cc;
+            const float* sc = reinterpret_cast<const float*>(smem + kOffSb + buf * kSbSlotBytes);
+            const float* bi = sc + MAFAT_MAX_NBLK;
+            const int X = rc.x0 + cc;
+            const bool pool = (rc.flags & 1) != 0, nhwc = (rc.flags & 2) != 0;
             // Work split between the warpgroups in units of one block x 32 output columns
             // (16 when N is an odd multiple of 16), dealt round-robin.
-            const int uw = (st.n_blk % 32 == 0) ? 32 : 16;
-            const int upb = st.n_blk / uw;  // units per block
-            const int ch_base = it.nb * st.n_blk;
-            for (int u = h; u < it.nbk * upb; u += kEpiGroups) {
+            const int uw = (rc.n_blk % 32 == 0) ? 32 : 16;
+            const int upb = rc.n_blk / uw;  // units per block
+            for (int u = h; u < rc.nbk * upb; u += kEpiGroups) {
                 const int b = u / upb, q = (u - b * upb) * uw;
-                const int Y = tk.cy0 + (it.by + b) * MAFAT_BLK_ROWS + r;
-                const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
-                bool store = valid;
+                const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
+                const bool valid = (Y < rc.ylim) && (X < rc.xlim);
+                // a pooled stage's conv region starts on even rows and columns and has even
+                // extents, so a window's four lanes agree on valid
+                const bool store = valid;
                 int oy = Y, ox = X;
-                if (st.pool) {
-                    store = valid && ((r & 1) == 0) && ((cc & 1) == 0);
+                if (pool) {
                     oy = Y >> 1;
                     ox = X >> 1;
                 }
+                const size_t pix = (size_t)(oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0);
                 EpiDst dst;
-                dst.out = out;
-                dst.nhwc = tk.out_nhwc;
-                dst.pix = tk.out_nhwc ? ((size_t)(oy - tk.out_y0) * tk.out_w + (ox - tk.out_x0)) * st.cout
-                                      : ((size_t)(oy - tk.out_y0) * tk.out_w + (ox - tk.out_x0)) * 8;
-                dst.plane = (size_t)tk.out_h * tk.out_w * 8;
-                dst.cout = st.cout;
+                dst.out = rc.out;
+                dst.nhwc = nhwc;
+                dst.pix = nhwc ? pix * rc.cout : pix * 8;
+                dst.plane = (size_t)rc.out_h * rc.out_w * 8;
+                dst.cout = rc.cout;
                 dst.store = store;
-                dst.pool = st.pool;
+                dst.pool = pool;
                 const uint32_t taddr = tmem_base + ((uint32_t)(wq * 32) << 16) +
-                                       (uint32_t)(buf * kAccStride + b * st.n_blk + q);
+                                       (uint32_t)(buf * kAccStride + b * rc.n_blk + q);
                 if (uw == 32)
-                    epi_chunk<32>(taddr, sc + q, bi + q, ch_base + q, dst);
+                    epi_chunk<32>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
                 else
-                    epi_chunk<16>(taddr, sc + q, bi + q, ch_base + q, dst);
+                    epi_chunk<16>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
             }
             tc_fence_before();
-            mbar_arrive(bar(kBarAccEmpty + buf));
-            ++acc_cnt;
-            // Every epilogue thread's stores are ordered before the barrier; thread 0 then
-            // publishes with a gpu-scope fence and release (cumulative over the barrier), so
-            // no thread needs a gpu-scope fence of its own.  The proxy fence orders the stores
-            // (generic proxy) with later TMA reads (async proxy) of the same memory.
+            mbar_arrive(bar(kBarAccEmpty + buf));  // also frees the scale / bias slot
+            // Hand the item to the publisher: the stores are fenced for the async proxy (TMA
+            // reads of them by later items), then every thread arrives on the item's EpiDone
+            // slot.  A slot is reused two items later, once the publisher is past it.
             mafat_dev::fence_proxy_async_global();
-            asm volatile("bar.sync 1, %0;" ::"r"(kEpiThreads) : "memory");
-            if (threadIdx.x == 0) {
-                mafat_dev::publish_item(p.ctr, it, tk.done_ctr);
-                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 3, mafat_dev::globaltimer_ns());
-            }
+            if (acc_cnt >= 2)
+                mbar_wait(bar(kBarPubDone + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 32);
+            mbar_arrive(bar(kBarEpiDone + buf));
+            ++acc_cnt;
         }
     }
 

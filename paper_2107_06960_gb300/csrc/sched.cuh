@@ -72,13 +72,17 @@ __device__ __forceinline__ void wait_item_deps(uint32_t* ctr, const MafatItemDev
 
 // Publish completion of an item (call once, after all of its stores are
 // ordered before this thread by a CTA-level barrier).
+// A release at gpu scope orders every write this thread has observed before it,
+// including the other threads' writes ordered before it by a CTA barrier or an
+// mbarrier (releases are cumulative), so no separate fence is needed.
+__device__ __forceinline__ void publish_counters(uint32_t* ctr, int done_ctr, int extra_ctr) {
+    red_release_add(ctr + done_ctr, 1u);
+    if (extra_ctr >= 0) red_release_add(ctr + extra_ctr, 1u);
+}
+
 __device__ __forceinline__ void publish_item(uint32_t* ctr, const MafatItemDev& it, int done_ctr) {
     if (it.flags & 1) return;  // test hook: never published
-    // A release at gpu scope orders every write this thread has observed before it,
-    // including the other threads' writes ordered by the CTA barrier (releases are
-    // cumulative), so no separate fence is needed.
-    red_release_add(ctr + done_ctr, 1u);
-    if (it.extra_ctr >= 0) red_release_add(ctr + it.extra_ctr, 1u);
+    publish_counters(ctr, done_ctr, it.extra_ctr);
 }
 
 __device__ __forceinline__ uint32_t smid() {
