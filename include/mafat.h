@@ -89,7 +89,12 @@ typedef struct {
     int32_t trace;              /* 1: record per-item timestamps on every run (mafat_plan_trace) */
     int32_t force_nblk;         /* output channels per work item for every stage (0: chosen per stage) */
     int32_t force_mb;           /* 16x8 pixel blocks per work item for every stage (0: chosen per stage) */
-    int32_t reserved[3];
+    int32_t lookahead_items;    /* a stage with at least this many work items (all tiles and frames)
+                                   takes each CTA's next item before the CTA's input buffer for it
+                                   is free, hiding the hand-out latency; smaller stages take it
+                                   only then, so that a busy CTA holds no item an idle one could
+                                   start (0: 5/4 of the CTAs; < 0: never) */
+    int32_t reserved[2];
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */

@@ -33,7 +33,7 @@ class LayerDesc(ctypes.Structure):
 class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
-                ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("reserved", i32 * 3)]
+                ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32), ("reserved", i32 * 2)]
 
 
 class PlanStats(ctypes.Structure):
@@ -196,7 +196,7 @@ class Plan:
 
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
-                 force_nblk=0, force_mb=0):
+                 force_nblk=0, force_mb=0, lookahead_items=0):
         self.net = net
         n_groups = 1 if cut is None else 2
         grids = list(grids)[:n_groups]
@@ -211,6 +211,7 @@ class Plan:
         opt.dry_run = 1 if dry_run else 0
         opt.trace = 1 if trace else 0
         opt.force_nblk, opt.force_mb = force_nblk, force_mb
+        opt.lookahead_items = lookahead_items
         h = vp()
         _check(lib.mafat_plan_ex(net.handle, n_groups, cuts, gn, gm, batch, dtype, ctypes.byref(opt),
                                  ctypes.byref(h)))

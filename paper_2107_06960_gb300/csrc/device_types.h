@@ -54,6 +54,7 @@ struct MafatStageDev {
     int32_t bpp;          // blobs per weight piece (a piece fills at most one shared-memory buffer)
     int32_t n_pieces;     // pieces per channel block (1: the set stays resident across items)
     int32_t sb_off;       // offset into the scale / bias arrays
+    int32_t lookahead;    // 1: a CTA takes its next item as soon as this stage's item is loaded
     int64_t w32_off;      // element offset of the fp32 weights [cout][cin][k][k]
 };
 
@@ -85,7 +86,7 @@ struct MafatItemDev {
     int16_t nb;           // output-channel block
     int16_t nbk;          // M blocks of this item (rows by .. by+nbk-1)
     int16_t flags;        // bit 0: do not publish completion (test hook)
-    int16_t pad;
+    int16_t stage;        // the task's stage (lets the task and stage records load in parallel)
     int32_t dep0, dep0_target;  // counter index (-1: none) and value to wait for
     int32_t dep1, dep1_target;
     int32_t extra_ctr;    // second counter bumped on completion (-1: none)

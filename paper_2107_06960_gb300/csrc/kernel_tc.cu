@@ -681,7 +681,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // A ticket is taken (and its item record loaded) at the end of the previous item,
             // once the A stage the new item will use is about to free: early enough to hide
             // the new item's loads behind the current MMAs, late enough that a CTA busy with a
-            // long item does not hold work another CTA could start now.
+            // long item does not hold work another CTA could start now.  After an item of a
+            // stage with many items (lookahead) it is taken at once: every CTA has work then,
+            // and the hand-out latency (atomic, record loads) is hidden behind the A stage's
+            // release instead of added to it.
             int next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
             MafatItemDev it_next;
             if (next < p.n_items) it_next = p.items[next];
@@ -694,9 +697,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 MafatTaskDev tk;
                 MafatStageDev st;
-                if (ticket >= 0) {
+                if (ticket >= 0) {  // two independent loads (the item names its stage)
                     tk = p.tasks[it.task];
-                    st = p.stages[tk.stage];
+                    st = p.stages[it.stage];
                 }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
@@ -795,8 +798,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
                 }
 #undef MAFAT_LOAD_PIECE
-                mbar_wait(bar(kBarAEmpty + (int)(a_cnt % kAStages)), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr,
-                          pipe_limit, broken, 64);
+                if (!st.lookahead)
+                    mbar_wait(bar(kBarAEmpty + (int)(a_cnt % kAStages)), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr,
+                              pipe_limit, broken, 64);
                 next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
                 if (next < p.n_items) it_next = p.items[next];
             }

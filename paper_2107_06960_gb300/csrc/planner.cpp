@@ -518,6 +518,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                     const int by = ri * tk.nby / n_rows, by_end = (ri + 1) * tk.nby / n_rows;
                     MafatItemDev it{};
                     it.task = ti;
+                    it.stage = (int16_t)tk.stage;
                     it.by = (int16_t)by;
                     it.nbk = (int16_t)(by_end - by);
                     it.bx = (int16_t)bx;
@@ -539,6 +540,17 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 }
     }
     if (t.items.size() > (size_t)0x7fffffff) return "too many work items";
+    // Stages with many items (all tiles and frames) keep every CTA busy whatever it holds,
+    // so their CTAs take the next ticket early; stages with about a wave of items or fewer
+    // take it only when the CTA can start it, so that no idle CTA waits for a busy one.
+    {
+        const int n_ctas = cfg.n_ctas > 0 ? cfg.n_ctas : 152;
+        const int64_t thr = cfg.lookahead_items > 0 ? cfg.lookahead_items : (int64_t)n_ctas * 5 / 4;
+        std::vector<int64_t> stage_items(t.stages.size(), 0);
+        for (const MafatTaskDev& tk : t.tasks) stage_items[tk.stage] += tk.n_items;
+        for (size_t s = 0; s < t.stages.size(); ++s)
+            t.stages[s].lookahead = (cfg.lookahead_items >= 0 && stage_items[s] >= thr) ? 1 : 0;
+    }
 
     // ---- statistics
     for (int l = 0; l < n; ++l) {
@@ -590,6 +602,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     for (size_t i = 0; i < t.items.size(); ++i) {
         int tk = t.items[i].task;
         if (tk < 0 || tk >= n_tasks) return "item with a bad task";
+        if (t.items[i].stage != t.tasks[tk].stage) return "item names another stage than its task";
         if (first_item[tk] < 0) first_item[tk] = (int)i;
         last_item[tk] = (int)i;
     }

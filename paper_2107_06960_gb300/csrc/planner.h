@@ -68,6 +68,7 @@ struct PlanConfig {
     int n_ctas = 0;           // persistent CTAs (shapes items; 0: 152)
     int fixed_nblk = 0;       // force the output-channel block of every stage (0: choose)
     int fixed_mb = 0;         // force blocks per item (0: choose)
+    int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
 };
 
 // A tensor-map request for a task whose input is a scratch region buffer.

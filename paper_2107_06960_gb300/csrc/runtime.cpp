@@ -322,6 +322,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.unpublished_task = o.test_unpublished_task;
     cfg.fixed_nblk = o.force_nblk;
     cfg.fixed_mb = o.force_mb;
+    cfg.lookahead_items = o.lookahead_items;
     int sms = 0;
     if (!o.dry_run) {
         int dev = 0;
