@@ -109,9 +109,21 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-// Adds bytes to the current phase's expected transactions without arriving.
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+// One elected lane of the converged warp adds 2 x bytes to the current phase of bar's
+// expected transactions (without arriving) and copies bytes of scale and of bias into
+// the slot (bias at slot + MAFAT_MAX_NBLK floats), completing on bar.  No branch on the
+// lane: the MMA warp stays converged.
+__device__ __forceinline__ void sb_load_elect(uint32_t bar, uint32_t slot, const float* scale, const float* bias,
+                                              uint32_t bytes) {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t.reg .b32 tx;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "add.u32 tx, %4, %4;\n\t"
+        "@e mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], tx;\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%1], [%2], %4, [%0];\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%5], [%3], %4, [%0];\n\t}" ::"r"(bar),
+        "r"(slot), "l"(scale), "l"(bias), "r"(bytes), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4))
+        : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
@@ -867,15 +879,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // the item's scale and bias go into the accumulator's slot (the epilogue of
                     // the slot's previous item is past it); the accumulator's full barrier then
                     // completes only once they have landed as well
-                    const uint32_t sb_bytes = j.n_blk * 4u;
-                    if (lane == 0) {
-                        const uint32_t fb = ms.bar(kBarAccFull + buf);
-                        const uint32_t slot = ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes);
-                        mbar_expect_tx(fb, 2u * sb_bytes);
-                        bulk_load(slot, p.scale + sb, sb_bytes, fb);
-                        bulk_load(slot + (uint32_t)(kSbSlotBytes / 2), p.bias + sb, sb_bytes, fb);
-                    }
-                    __syncwarp();
+                    sb_load_elect(ms.bar(kBarAccFull + buf), ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes),
+                                  p.scale + sb, p.bias + sb, j.n_blk * 4u);
                 }
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
                 j.idesc = instr_desc_bf16((int)j.n_blk, 128);
