@@ -251,6 +251,15 @@ def run_sweep(args):
             best = line
         plan.close()
     print(json.dumps({"sweep_best": best}), flush=True)
+    # the same space through the library's measured search: candidates whose intermediates
+    # exceed the L2 are refused, the rest timed on the device
+    cands, bi = net.search_measured(cuts=synth.SWEEP_CUTS, max_grid=max(synth.SWEEP_GRIDS), runs=steps)
+    timed = [c for c in cands if c["us_per_run"] is not None]
+    print(json.dumps({"search_measured": {
+        "candidates": len(cands), "timed": len(timed), "refused_over_l2": sum(c["status"] == mf.ENOFIT for c in cands),
+        "best": cands[bi] if bi >= 0 else None,
+        "benchmark_plan": next((c for c in cands if c["cut"] == 8 and c["grids"] == [(5, 5), (2, 2)]), None)}}),
+        flush=True)
 
 
 def main():

@@ -233,6 +233,52 @@ mafat_status mafat_predict_mem(const mafat_net_t* net, int32_t cut, int32_t n1, 
 mafat_status mafat_search(const mafat_net_t* net, double limit_mib, double bias_mib,
                           int32_t* top_tile, int32_t* cut, int32_t* bottom_tile);
 
+/* Measured plan search: Algorithm 2 (Sec. 4.1) re-targeted at the GPU.  Algorithm 2
+ * looks for the cut and tilings of lowest latency whose predicted memory fits the
+ * device; here the memory that matters is the L2 that a plan's intermediates (tile
+ * scratch ring and cut tensor) should stay in, and latency is measured rather than
+ * predicted: every candidate within budget_bytes is planned and timed on the device,
+ * and the fastest is reported.  Candidates, in this order: one layer group (if
+ * include_one_group), then two groups at each cut of cuts[0..n_cuts-1] (the first
+ * layer of group 2), every group tiled N x M for N, M in 1..max_grid (N == M when
+ * square_only, else |N - M| <= 1), group 1's tiling outer. */
+typedef struct {
+    int32_t struct_size;        /* sizeof(mafat_search_options) */
+    int32_t batch;              /* images per run (0: 1) */
+    int32_t dtype;              /* MAFAT_BF16 or MAFAT_FP32 */
+    int32_t include_one_group;
+    int32_t n_cuts;
+    const int32_t* cuts;        /* n_cuts candidate cuts (may be NULL when n_cuts == 0) */
+    int32_t max_grid;           /* tiles per axis 1..max_grid (0: 5) */
+    int32_t square_only;
+    int64_t budget_bytes;       /* intermediate bytes allowed (0: the device's L2 size, or 128 MiB for a
+                                   dry run; < 0: no limit) */
+    int32_t runs;               /* timed runs per candidate, median reported (0: 10) */
+    int32_t flush_l2;           /* 1: write 256 MiB before each timed run (every run starts with a cold L2) */
+    int32_t dry_run;            /* 1: enumerate and size the candidates only; needs no GPU */
+    int32_t reserved[3];
+} mafat_search_options;
+
+typedef struct {
+    int32_t n_groups, cut;      /* cut is 0 for one group */
+    int32_t grid_n[2], grid_m[2];
+    int64_t intermediate_bytes; /* tile scratch ring + cut tensor of the plan */
+    double predicted_mib;       /* Algorithm 1 (literal reading, 31 MiB bias) for the configuration */
+    double executed_flops;      /* per run, halo recompute included */
+    double us_per_run;          /* median device time of a run; < 0 if not timed */
+    int32_t status;             /* MAFAT_OK if timed; MAFAT_ENOFIT over budget; else the plan's error */
+    int32_t reserved;
+} mafat_search_candidate;
+
+/* Runs the measured search on `stream` (the net's weights must be set; the input is
+ * synthetic, since a run's time does not depend on the data).  Writes the first
+ * max_out candidates to out (may be NULL), their total number to *n_out and the
+ * index of the fastest timed one to *best (-1 if none was timed).  Allocates device
+ * memory; not for use during stream capture. */
+mafat_status mafat_search_measured(const mafat_net_t* net, const mafat_search_options* opt, void* stream,
+                                   mafat_search_candidate* out, int32_t max_out, int32_t* n_out,
+                                   int32_t* best);
+
 /* Plan statistics (struct_size must be set by the caller). */
 mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out);
 

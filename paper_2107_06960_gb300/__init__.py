@@ -22,6 +22,7 @@ MAFAT_CONV, MAFAT_MAXPOOL = 0, 1
 BF16, FP32 = 0, 1
 STATUS = {0: "OK", 1: "EINVAL", 2: "EUNSUPPORTED", 3: "ENOMEM", 4: "ECUDA", 5: "ETIMEOUT", 6: "ENOFIT",
           7: "EDEVICE"}
+OK, EINVAL, EUNSUPPORTED, ENOMEM, ECUDA, ETIMEOUT, ENOFIT, EDEVICE = range(8)
 
 i32, i64, dbl, vp = ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_void_p
 
@@ -42,6 +43,19 @@ class PlanStats(ctypes.Structure):
                 ("predicted_mib", dbl), ("group_io_bytes", i64), ("weight_bytes", i64),
                 ("scratch_bytes", i64), ("workspace_bytes", i64), ("smem_bytes_per_cta", i64),
                 ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32), ("dtype", i32)]
+
+
+class SearchOptions(ctypes.Structure):
+    _fields_ = [("struct_size", i32), ("batch", i32), ("dtype", i32), ("include_one_group", i32),
+                ("n_cuts", i32), ("cuts", ctypes.POINTER(i32)), ("max_grid", i32), ("square_only", i32),
+                ("budget_bytes", i64), ("runs", i32), ("flush_l2", i32), ("dry_run", i32),
+                ("reserved", i32 * 3)]
+
+
+class SearchCandidate(ctypes.Structure):
+    _fields_ = [("n_groups", i32), ("cut", i32), ("grid_n", i32 * 2), ("grid_m", i32 * 2),
+                ("intermediate_bytes", i64), ("predicted_mib", dbl), ("executed_flops", dbl),
+                ("us_per_run", dbl), ("status", i32), ("reserved", i32)]
 
 
 # (name, restype, argtypes) of every entry point of include/mafat.h
@@ -66,6 +80,8 @@ _SIGNATURES = [
     ("mafat_predict_mem", i32, [vp, i32, i32, i32, i32, i32, dbl, ctypes.POINTER(dbl)]),
     ("mafat_search", i32, [vp, dbl, dbl, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_plan_stats_get", i32, [vp, ctypes.POINTER(PlanStats)]),
+    ("mafat_search_measured", i32, [vp, ctypes.POINTER(SearchOptions), vp, ctypes.POINTER(SearchCandidate), i32,
+                                    ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_launches_per_run", i32, [vp]),
     ("mafat_plan_trace", i32, [vp, vp, i64, vp]),
     ("mafat_plan_destroy", None, [vp]),
@@ -178,6 +194,34 @@ class Net:
         a, c, b = i32(), i32(), i32()
         _check(lib.mafat_search(self.handle, limit_mib, bias_mib, ctypes.byref(a), ctypes.byref(c), ctypes.byref(b)))
         return a.value, b.value, c.value  # (top_tile, bottom_tile, cut)
+
+    def search_measured(self, cuts=(2, 4, 8, 12), include_one_group=True, max_grid=5, square_only=True,
+                        budget_bytes=0, runs=10, flush_l2=True, dry_run=False, batch=1, dtype=BF16, stream=None):
+        """Measured plan search (mafat_search_measured): returns (candidates, best index), each
+        candidate a dict with n_groups, cut (None for one group), grids [(n, m), ...],
+        intermediate_bytes, predicted_mib, executed_flops, us_per_run (None if not timed) and
+        status."""
+        opt = SearchOptions()
+        opt.struct_size = ctypes.sizeof(SearchOptions)
+        opt.batch, opt.dtype, opt.include_one_group = batch, dtype, int(include_one_group)
+        cut_arr = (i32 * max(1, len(cuts)))(*cuts)
+        opt.n_cuts, opt.cuts = len(cuts), ctypes.cast(cut_arr, ctypes.POINTER(i32))
+        opt.max_grid, opt.square_only, opt.budget_bytes = max_grid, int(square_only), budget_bytes
+        opt.runs, opt.flush_l2, opt.dry_run = runs, int(flush_l2), int(dry_run)
+        cap = 4096
+        out = (SearchCandidate * cap)()
+        n, best = i32(), i32()
+        _check(lib.mafat_search_measured(self.handle, ctypes.byref(opt), _stream(stream), out, cap,
+                                         ctypes.byref(n), ctypes.byref(best)))
+        res = []
+        for c in out[:min(n.value, cap)]:
+            g = c.n_groups
+            res.append({"n_groups": g, "cut": c.cut if g == 2 else None,
+                        "grids": [(c.grid_n[i], c.grid_m[i]) for i in range(g)],
+                        "intermediate_bytes": c.intermediate_bytes, "predicted_mib": c.predicted_mib,
+                        "executed_flops": c.executed_flops,
+                        "us_per_run": c.us_per_run if c.us_per_run >= 0 else None, "status": c.status})
+        return res, best.value
 
     def close(self):
         if getattr(self, "handle", None):

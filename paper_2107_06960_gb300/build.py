@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmafat.so")
-SOURCES = ["planner.cpp", "runtime.cpp", "kernel_fp32.cu", "kernel_tc.cu", "noalloc.cu"]
+SOURCES = ["planner.cpp", "runtime.cpp", "search.cpp", "kernel_fp32.cu", "kernel_tc.cu", "noalloc.cu"]
 HEADERS = ["planner.h", "device_types.h", "kernels.h", "sched.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

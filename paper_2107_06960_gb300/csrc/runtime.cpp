@@ -239,6 +239,8 @@ mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* 
 }
 
 mafat_status mafat_internal_fail(mafat_status s, const char* msg) { return fail(s, msg); }
+int32_t mafat_internal_net_layers(const mafat_net_t* net) { return net ? (int32_t)net->net.layers.size() : 0; }
+void mafat_internal_clear_error() { g_err.clear(); }
 
 extern "C" {
 

@@ -219,6 +219,30 @@ def test_bf16_608_every_sweep_plan_default_shapes(mf):
             assert e <= TOL_BF16, "plan %s %s cut tensor: rel err %.3g" % (cut, grids, e)
 
 
+def test_measured_search_picks_the_fastest_timed_plan(mf):
+    # Algorithm 2 re-targeted at the GPU: candidates whose intermediates fit the L2 are timed,
+    # the others refused; the fastest is reported, and it computes the network correctly
+    import torch
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    layers, params, x = wl["layers"], wl["params"], wl["input"]
+    net = mf.Net(layers, 608, 608, 3)
+    net.set_params(params)
+    cands, best = net.search_measured(cuts=(8, 12), max_grid=3, runs=5)
+    assert len(cands) == 3 + 2 * 9
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    for c in cands:
+        if c["intermediate_bytes"] > l2:
+            assert c["status"] == mf.ENOFIT and c["us_per_run"] is None
+        else:
+            assert c["status"] == mf.OK and c["us_per_run"] > 0
+    timed = [i for i, c in enumerate(cands) if c["us_per_run"] is not None]
+    assert best in timed
+    assert cands[best]["us_per_run"] == min(cands[i]["us_per_run"] for i in timed)
+    b = cands[best]
+    _, out = run_plan(mf, layers, params, x, b["cut"], b["grids"], mf.BF16)
+    assert rel_err(out[0], oracle.forward(layers, params, x[0])[-1]) <= TOL_BF16
+
+
 # ---------------------------------------------------------------------------
 # Run paths: host buffers, CUDA graphs, repeated runs
 # ---------------------------------------------------------------------------

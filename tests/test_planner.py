@@ -145,3 +145,36 @@ def test_grid_finer_than_output_skips_empty_tiles(mf):
     # group 1 output at cut 12 is 4x4; a 5x5 grid has empty rows/columns of tiles
     st = mf.Plan(net, 12, [(5, 5), (3, 3)], dry_run=True).stats()
     assert st["n_tiles"] == 4 * 4 + 3 * 3
+
+
+def test_measured_search_dry_run_candidates(mf):
+    # the candidate list of the measured search (Algorithm 2 re-targeted at the GPU): order,
+    # sizes, the L2 budget rule and the non-square grids, all on the host
+    net = _net(mf, synth.YOLO16, 608)
+    cands, best = net.search_measured(dry_run=True, budget_bytes=-1)
+    assert best == -1
+    assert len(cands) == 5 + 4 * 25
+    assert [c["grids"] for c in cands[:5]] == [[(t, t)] for t in range(1, 6)]
+    assert all(c["n_groups"] == 1 and c["cut"] is None for c in cands[:5])
+    assert [c["cut"] for c in cands[5:]] == [cut for cut in (2, 4, 8, 12) for _ in range(25)]
+    assert [c["grids"] for c in cands[5:30]] == [[(a, a), (b, b)] for a in range(1, 6) for b in range(1, 6)]
+    for c in cands[::7]:
+        st = mf.Plan(net, c["cut"], c["grids"], dry_run=True).stats()
+        cut_bytes = 0
+        if c["cut"] is not None:
+            sh = net.shape(c["cut"] - 1)
+            cut_bytes = (sh[5] + 7) // 8 * 8 * sh[3] * sh[4] * 2
+        assert c["intermediate_bytes"] == st["scratch_bytes"] + cut_bytes
+        assert c["predicted_mib"] == st["predicted_mib"]
+        assert c["executed_flops"] == st["executed_flops"]
+        assert c["status"] == 0 and c["us_per_run"] is None
+    # with a budget, exactly the candidates above it are refused (MAFAT_ENOFIT)
+    budget = sorted(c["intermediate_bytes"] for c in cands)[len(cands) // 2]
+    capped, _ = net.search_measured(dry_run=True, budget_bytes=budget)
+    assert [c["status"] for c in capped] == [
+        mf.ENOFIT if c["intermediate_bytes"] > budget else 0 for c in cands]
+    # non-square tilings: N x M with |N - M| <= 1, 13 per group
+    ns, _ = net.search_measured(dry_run=True, square_only=False, cuts=(8,), budget_bytes=-1)
+    assert len(ns) == 13 + 13 * 13
+    assert all(abs(n - m) <= 1 for c in ns for n, m in c["grids"])
+    assert (5, 4) in [c["grids"][0] for c in ns[:13]]
