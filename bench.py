@@ -34,6 +34,15 @@ import numpy as np  # noqa: E402
 import synth  # noqa: E402
 
 METRIC = "frames/s (YOLOv2 first 16 layers, 608x608, bf16, fused tiles)"
+
+
+def metric_of(name):
+    """The metric line of a workload (the headline one for the default workload)."""
+    wl = synth.WORKLOADS[name]
+    if name == DEFAULT_WORKLOAD:
+        return METRIC
+    net = "YOLOv2 first 16 layers" if wl["layers"] == synth.YOLO16 else "YOLOv2 trunk, %d layers" % len(wl["layers"])
+    return "frames/s (%s, %dx%d, %s, fused tiles)" % (net, wl["h"], wl["w"], wl["dtype"])
 DEFAULT_WORKLOAD = "yolo16_608_5x5_c8_2x2"
 L2_FLUSH_BYTES = 256 << 20
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -182,7 +191,7 @@ def run_reference(args, wl):
     value = frac * args.steps / el
     sample = "%dx%d crop per step (%.4f of a frame's FLOPs), unfused fp64 forward" % (side, side, frac)
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": ws,
+        "impl": "reference", "metric": metric_of(args.workload), "value": value, "unit": "frames/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": args.workload, "input": "%dx%dx3" % (wl["h"], wl["w"]), "batch": wl["batch"]},
@@ -390,14 +399,15 @@ def main():
         cpu = {"value": v, "unit": "frames/s", "cores": cores, "kind": "oracle", "sample": sample}
 
     line = {
-        "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": ws, "steps": args.steps,
+        "metric": metric_of(args.workload), "value": value, "unit": "frames/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if dt == mf.BF16 else "f32", "data": "synthetic",
         "config": {
             "workload": args.workload, "input": "%dx%dx3" % (H, W), "batch": B,
             "cut": wl["cut"], "grids": "/".join("%dx%d" % tuple(gd) for gd in wl["grids"]),
             "l2": "flushed before every timed step (256 MiB write, not timed)",
-            "e2e_l2": "not flushed between streamed frames (a serving loop keeps the 6.9 MB of weights in L2)",
+            "e2e_l2": "not flushed between streamed frames (a serving loop keeps the %.1f MB of weights in L2)"
+                      % (st["weight_bytes"] / 1e6),
             "useful_gflop_per_frame": st["useful_flops"] / B / 1e9,
             "executed_gflop_per_frame": st["executed_flops"] / B / 1e9,
             "halo_recompute": st["executed_flops"] / st["useful_flops"] - 1.0,

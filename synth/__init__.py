@@ -39,6 +39,21 @@ YOLO16 = [
     (CONV, 1, 1, 0, 256),
 ]
 
+# The rest of the YOLOv2 trunk up to its route layer: conv 3x3 512, max-pool, then at 1/32
+# resolution conv 3x3 1024, 1x1 512, 3x3 1024, 1x1 512, 3x3 1024 and two detection-head
+# 3x3 1024 convolutions (25 layers in all; every later layer is a route, reorg or concat).
+YOLO25 = YOLO16 + [
+    (CONV, 3, 1, 1, 512),
+    (MAX, 2, 2, 0, 0),
+    (CONV, 3, 1, 1, 1024),
+    (CONV, 1, 1, 0, 512),
+    (CONV, 3, 1, 1, 1024),
+    (CONV, 1, 1, 0, 512),
+    (CONV, 3, 1, 1, 1024),
+    (CONV, 3, 1, 1, 1024),
+    (CONV, 3, 1, 1, 1024),
+]
+
 # Tiny three-layer stack used for fp32 parity.
 TINY3 = [
     (CONV, 3, 1, 1, 8),
@@ -60,6 +75,11 @@ WORKLOADS = {
                                   cut=8, grids=[(5, 5), (2, 2)], seed=SEED_BASE + 2),
     "yolo16_1216_b8_8x8_c8_4x4": dict(layers=YOLO16, h=1216, w=1216, c=3, batch=8, dtype="bf16",
                                       cut=8, grids=[(8, 8), (4, 4)], seed=SEED_BASE + 4),
+    # a second workload: the whole YOLOv2 trunk (weight-heavy 1024-channel layers at 19x19)
+    "yolo25_96_2x2_c8_1x1": dict(layers=YOLO25, h=96, w=96, c=3, batch=2, dtype="bf16",
+                                 cut=8, grids=[(2, 2), (1, 1)], seed=SEED_BASE + 5),
+    "yolo25_608_5x5_c8_2x2": dict(layers=YOLO25, h=608, w=608, c=3, batch=1, dtype="bf16",
+                                  cut=8, grids=[(5, 5), (2, 2)], seed=SEED_BASE + 6),
 }
 # The sweep: cut after layer 1, 3, 7, 11 (paper cut 2, 4, 8, 12) x grids 1..5 per group.
 SWEEP_CUTS = [2, 4, 8, 12]

@@ -170,6 +170,24 @@ def test_bf16_full_size(mf, name):
     _check_groups(c, out, refs, wl["cut"], TOL_BF16)
 
 
+@pytest.mark.parametrize("name", ["yolo25_96_2x2_c8_1x1", "yolo25_608_5x5_c8_2x2"])
+def test_bf16_yolov2_trunk(mf, name):
+    # a second workload: the whole YOLOv2 trunk, 1024-channel 3x3 layers (16 input chunks,
+    # 1.2 MB of weights streamed per work item) after the fifth pooling
+    wl = synth.workload(name)
+    c, out = run_plan(mf, wl["layers"], wl["params"], wl["input"], wl["cut"], wl["grids"], mf.BF16)
+    refs = _oracle_groups(wl["layers"], wl["params"], wl["input"], wl["cut"], name)
+    _check_groups(c, out, refs, wl["cut"], TOL_BF16)
+
+
+def test_fp32_yolov2_trunk_96(mf):
+    layers = synth.YOLO25
+    params = synth.make_params(layers, 3, 51, "fp32")
+    x = synth.make_input(1, 96, 96, 3, 52, "fp32")
+    c, out = run_plan(mf, layers, params, x, 8, [(2, 2), (1, 1)], mf.FP32)
+    _check_groups(c, out, _oracle_groups(layers, params, x, 8), 8, TOL_FP32)
+
+
 def test_bf16_1216_batch8_stress(mf):
     wl = synth.workload("yolo16_1216_b8_8x8_c8_4x4")
     c, out = run_plan(mf, wl["layers"], wl["params"], wl["input"], wl["cut"], wl["grids"], mf.BF16)

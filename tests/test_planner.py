@@ -92,7 +92,8 @@ def _region_flops(layers, size, cut, grids, batch):
     return tot * batch
 
 
-@pytest.mark.parametrize("name", ["yolo16_416_1x3x3", "yolo16_608_5x5_c8_2x2", "yolo16_1216_b8_8x8_c8_4x4"])
+@pytest.mark.parametrize("name", ["yolo16_416_1x3x3", "yolo16_608_5x5_c8_2x2", "yolo16_1216_b8_8x8_c8_4x4",
+                                  "yolo25_608_5x5_c8_2x2"])
 def test_plan_statistics(mf, name):
     wl = synth.WORKLOADS[name]
     layers, size, batch = wl["layers"], wl["h"], wl["batch"]
