@@ -94,7 +94,9 @@ typedef struct {
                                    is free, hiding the hand-out latency; smaller stages take it
                                    only then, so that a busy CTA holds no item an idle one could
                                    start (0: 5/4 of the CTAs; < 0: never) */
-    int32_t reserved[2];
+    const int32_t* tile_bounds; /* non-uniform tiling (NULL: the even N x M grid): for each group, its
+                                   grid_n + 1 row bounds then its grid_m + 1 column bounds on the
+                                   group's last-layer output, 0 = b[0] < b[1] < ... < b[n] = size */
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */
@@ -226,6 +228,15 @@ mafat_status mafat_predict_layer_group(const mafat_net_t* net, int32_t first, in
  * configuration (cut, n1 x m1 top tiling, n2 x m2 bottom tiling), MiB. */
 mafat_status mafat_predict_mem(const mafat_net_t* net, int32_t cut, int32_t n1, int32_t m1,
                                int32_t n2, int32_t m2, double bias_mib, double* out_mib);
+
+/* Work-balanced non-uniform tile bounds for layers first..last: n + 1 row bounds and
+ * m + 1 column bounds on the last layer's output, chosen per axis so that the largest
+ * part's executed work (its regions traced back through every convolution of the
+ * group, halo included, the other axis whole) is as small as possible.  Edge tiles need
+ * less halo, so they come out larger than interior ones.  Pass them as
+ * mafat_plan_options.tile_bounds.  Host only. */
+mafat_status mafat_balanced_bounds(const mafat_net_t* net, int32_t first, int32_t last, int32_t n, int32_t m,
+                                   int32_t* row_bounds, int32_t* col_bounds);
 
 /* Algorithm 2: search cut in {n (no cut), 12, 8} x square top tilings 1..5
  * with a 2x2 bottom tiling, returning the first configuration predicted

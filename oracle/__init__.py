@@ -119,17 +119,26 @@ def _back(rng, k, s, p, size_in):
     return (max(lo, 0), min(hi, size_in))
 
 
-def tile_regions(layers, shapes, group, n, m, i, j):
+def tile_regions(layers, shapes, group, n, m, i, j, bounds=None):
     """The ``Grid`` traversal: for tile (i, j) of an n x m grid on the group's
     last-layer output, the output and input rectangle of every layer of the
-    group, walking from the last layer back to the first.
+    group, walking from the last layer back to the first.  ``bounds`` = (row
+    bounds, column bounds) gives a non-uniform grid (n + 1 and m + 1 increasing
+    values from 0 to the map size); None means the even grid.
 
     Returns {layer: (out_rect, in_rect)} with rect = (y0, y1, x0, x1), half-open.
     """
     first, last = group
     sh = shapes[last]
-    rows = grid_bounds(sh["h_out"], n)[i]
-    cols = grid_bounds(sh["w_out"], m)[j]
+    if bounds is None:
+        rows = grid_bounds(sh["h_out"], n)[i]
+        cols = grid_bounds(sh["w_out"], m)[j]
+    else:
+        rb, cb = bounds
+        for b, size, parts in ((rb, sh["h_out"], n), (cb, sh["w_out"], m)):
+            if len(b) != parts + 1 or b[0] != 0 or b[-1] != size or any(x >= y for x, y in zip(b, b[1:])):
+                raise ValueError("tile bounds do not partition the group output")
+        rows, cols = (rb[i], rb[i + 1]), (cb[j], cb[j + 1])
     out = {}
     for l in range(last, first - 1, -1):
         t, k, s, p, f = layers[l]
@@ -307,26 +316,28 @@ def _region_layer(layer, prm, buf, in_rect, map_hw, out_rect):
     return out
 
 
-def forward_tiled(layers, params, x, cut, grids):
+def forward_tiled(layers, params, x, cut, grids, bounds=None):
     """Fused tile partitioning with up to two layer groups (Sec. 3, Sec. 4).
 
     Each group's last-layer output is split into an N x M grid; every tile
     runs all layers of its group on its own regions (recomputing the overlap),
     and writes its rectangle of the group output.  Group 2 re-tiles the merged
-    cut tensor.  Returns the group outputs; raises if the tiles do not cover
-    the group output exactly once.
+    cut tensor.  ``bounds`` (one (row bounds, column bounds) pair per group, or
+    None) gives non-uniform grids.  Returns the group outputs; raises if the
+    tiles do not cover the group output exactly once.
     """
     shapes = layer_shapes(layers, x.shape[0], x.shape[1], x.shape[2])
     gin = np.asarray(x, dtype=np.float64)
     results = []
-    for g, (n, m) in zip(groups_of(len(layers), cut), grids):
+    for gi, (g, (n, m)) in enumerate(zip(groups_of(len(layers), cut), grids)):
+        gb = None if bounds is None else bounds[gi]
         first, last = g
         sh = shapes[last]
         gout = np.zeros((sh["h_out"], sh["w_out"], sh["c_out"]), dtype=np.float64)
         cover = np.zeros((sh["h_out"], sh["w_out"]), dtype=np.int64)
         for i in range(n):
             for j in range(m):
-                regs = tile_regions(layers, shapes, g, n, m, i, j)
+                regs = tile_regions(layers, shapes, g, n, m, i, j, gb)
                 out_rect_last = regs[last][0]
                 if out_rect_last[1] <= out_rect_last[0] or out_rect_last[3] <= out_rect_last[2]:
                     continue

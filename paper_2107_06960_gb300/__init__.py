@@ -34,7 +34,8 @@ class LayerDesc(ctypes.Structure):
 class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
-                ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32), ("reserved", i32 * 2)]
+                ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32),
+                ("tile_bounds", ctypes.POINTER(i32))]
 
 
 class PlanStats(ctypes.Structure):
@@ -79,6 +80,7 @@ _SIGNATURES = [
     ("mafat_predict_layer_group", i32, [vp, i32, i32, i32, i32, dbl, i32, ctypes.POINTER(dbl)]),
     ("mafat_predict_mem", i32, [vp, i32, i32, i32, i32, i32, dbl, ctypes.POINTER(dbl)]),
     ("mafat_search", i32, [vp, dbl, dbl, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)]),
+    ("mafat_balanced_bounds", i32, [vp, i32, i32, i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_plan_stats_get", i32, [vp, ctypes.POINTER(PlanStats)]),
     ("mafat_search_measured", i32, [vp, ctypes.POINTER(SearchOptions), vp, ctypes.POINTER(SearchCandidate), i32,
                                     ctypes.POINTER(i32), ctypes.POINTER(i32)]),
@@ -195,6 +197,13 @@ class Net:
         _check(lib.mafat_search(self.handle, limit_mib, bias_mib, ctypes.byref(a), ctypes.byref(c), ctypes.byref(b)))
         return a.value, b.value, c.value  # (top_tile, bottom_tile, cut)
 
+    def balanced_bounds(self, first, last, n, m):
+        """Work-balanced non-uniform tile bounds (rows, cols) of an n x m grid on the output of
+        layers first..last (mafat_balanced_bounds)."""
+        r, c = (i32 * (n + 1))(), (i32 * (m + 1))()
+        _check(lib.mafat_balanced_bounds(self.handle, first, last, n, m, r, c))
+        return list(r), list(c)
+
     def search_measured(self, cuts=(2, 4, 8, 12), include_one_group=True, max_grid=5, square_only=True,
                         budget_bytes=0, runs=10, flush_l2=True, dry_run=False, batch=1, dtype=BF16, stream=None):
         """Measured plan search (mafat_search_measured): returns (candidates, best index), each
@@ -240,7 +249,7 @@ class Plan:
 
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
-                 force_nblk=0, force_mb=0, lookahead_items=0):
+                 force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None):
         self.net = net
         n_groups = 1 if cut is None else 2
         grids = list(grids)[:n_groups]
@@ -256,6 +265,11 @@ class Plan:
         opt.trace = 1 if trace else 0
         opt.force_nblk, opt.force_mb = force_nblk, force_mb
         opt.lookahead_items = lookahead_items
+        if tile_bounds is not None:
+            # per group (rows, cols): the non-uniform tiling; kept alive with the plan
+            flat = [v for rows, cols in list(tile_bounds)[:n_groups] for v in list(rows) + list(cols)]
+            self._bounds = (i32 * len(flat))(*flat)
+            opt.tile_bounds = ctypes.cast(self._bounds, ctypes.POINTER(i32))
         h = vp()
         _check(lib.mafat_plan_ex(net.handle, n_groups, cuts, gn, gm, batch, dtype, ctypes.byref(opt),
                                  ctypes.byref(h)))

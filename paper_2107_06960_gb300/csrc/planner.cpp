@@ -78,6 +78,70 @@ void tile_regions(const Net& net, int first, int last, int n, int m, int i, int 
     r.y1 = grid_bound(Ll.h_out, n, i + 1);
     r.x0 = grid_bound(Ll.w_out, m, j);
     r.x1 = grid_bound(Ll.w_out, m, j + 1);
+    rect_regions(net, first, last, r, out_rects, in_rects);
+}
+
+std::vector<int> axis_bounds(int len, int n, const std::vector<int>& given) {
+    if (!given.empty()) return given;
+    std::vector<int> b(n + 1);
+    for (int i = 0; i <= n; ++i) b[i] = grid_bound(len, n, i);
+    return b;
+}
+
+std::string check_bounds(const std::vector<int>& b, int len, int n) {
+    if ((int)b.size() != n + 1) return "tile bounds: need n + 1 values per axis";
+    if (b[0] != 0 || b[n] != len) return "tile bounds must start at 0 and end at the map size";
+    for (int i = 0; i < n; ++i)
+        if (b[i + 1] <= b[i]) return "tile bounds must increase strictly";
+    return "";
+}
+
+std::vector<int> balanced_bounds(const Net& net, int first, int last, int n, int axis) {
+    const Layer& Ll = net.layers[last];
+    const int len = axis == 0 ? Ll.h_out : Ll.w_out;
+    n = std::max(1, std::min(n, len));
+    // work[a][b]: MACs of the part [a, b) with the other axis whole
+    std::vector<double> work((size_t)(len + 1) * (len + 1), 0.0);
+    for (int a = 0; a < len; ++a)
+        for (int b = a + 1; b <= len; ++b) {
+            int lo = a, hi = b;
+            double w = 0.0;
+            for (int l = last; l >= first; --l) {
+                const Layer& L = net.layers[l];
+                int ilo, ihi;
+                back_interval(lo, hi, L.k, L.stride, L.pad, axis == 0 ? L.h_in : L.w_in, &ilo, &ihi);
+                if (L.type == L_CONV)
+                    w += (double)(hi - lo) * (axis == 0 ? L.w_out : L.h_out) * L.c_out * (double)L.c_in * L.k * L.k;
+                lo = ilo;
+                hi = ihi;
+            }
+            work[(size_t)a * (len + 1) + b] = w;
+        }
+    // best[k][b]: smallest possible largest part when [0, b) is cut into k parts
+    const double inf = 1e300;
+    std::vector<double> best((size_t)(n + 1) * (len + 1), inf);
+    std::vector<int> from((size_t)(n + 1) * (len + 1), -1);
+    best[0] = 0.0;
+    for (int k = 1; k <= n; ++k)
+        for (int b = k; b <= len; ++b)
+            for (int a = k - 1; a < b; ++a) {
+                const double prev = best[(size_t)(k - 1) * (len + 1) + a];
+                if (prev >= inf) continue;
+                const double v = std::max(prev, work[(size_t)a * (len + 1) + b]);
+                if (v < best[(size_t)k * (len + 1) + b]) {
+                    best[(size_t)k * (len + 1) + b] = v;
+                    from[(size_t)k * (len + 1) + b] = a;
+                }
+            }
+    std::vector<int> bounds(n + 1);
+    bounds[n] = len;
+    for (int k = n; k > 0; --k) bounds[k - 1] = from[(size_t)k * (len + 1) + bounds[k]];
+    return bounds;
+}
+
+void rect_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
+                  std::vector<Rect>& in_rects) {
+    Rect r = out_last;
     if ((int)out_rects.size() < (int)net.layers.size()) out_rects.resize(net.layers.size());
     if ((int)in_rects.size() < (int)net.layers.size()) in_rects.resize(net.layers.size());
     for (int l = last; l >= first; --l) {
@@ -186,17 +250,29 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         t.groups[1][1] = n - 1;
     }
 
-    // ---- tiles of every group (non-empty only)
+    // ---- tiles of every group (non-empty only), on the even grid or the given bounds
     std::vector<std::vector<TileInfo>> tiles(G);
     int max_tiles = 1;
     for (int g = 0; g < G; ++g) {
+        const Layer& Lg = net.layers[t.groups[g][1]];
+        if (!cfg.row_bounds[g].empty() || !cfg.col_bounds[g].empty()) {
+            std::string e = check_bounds(cfg.row_bounds[g], Lg.h_out, cfg.grid_n[g]);
+            if (e.empty()) e = check_bounds(cfg.col_bounds[g], Lg.w_out, cfg.grid_m[g]);
+            if (!e.empty()) return "group " + std::to_string(g + 1) + ": " + e;
+        }
+        t.rows[g] = axis_bounds(Lg.h_out, cfg.grid_n[g], cfg.row_bounds[g]);
+        t.cols[g] = axis_bounds(Lg.w_out, cfg.grid_m[g], cfg.col_bounds[g]);
         for (int i = 0; i < cfg.grid_n[g]; ++i)
             for (int j = 0; j < cfg.grid_m[g]; ++j) {
                 TileInfo ti;
                 ti.i = i;
                 ti.j = j;
-                tile_regions(net, t.groups[g][0], t.groups[g][1], cfg.grid_n[g], cfg.grid_m[g], i, j,
-                             ti.outs, ti.ins);
+                Rect r;
+                r.y0 = t.rows[g][i];
+                r.y1 = t.rows[g][i + 1];
+                r.x0 = t.cols[g][j];
+                r.x1 = t.cols[g][j + 1];
+                rect_regions(net, t.groups[g][0], t.groups[g][1], r, ti.outs, ti.ins);
                 if (ti.outs[t.groups[g][1]].empty()) continue;
                 tiles[g].push_back(std::move(ti));
             }

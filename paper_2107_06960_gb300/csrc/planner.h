@@ -44,9 +44,25 @@ inline int grid_bound(int len, int n, int i) { return (int)((int64_t)i * len / n
 void back_interval(int a, int b, int k, int s, int p, int size_in, int* lo, int* hi);
 
 // Grid traversal: out_rects[l] / in_rects[l] for every layer l of first..last
-// (vectors indexed by layer; entries outside the group untouched).
+// (vectors indexed by layer; entries outside the group untouched), for tile (i, j)
+// of the even n x m grid on layer last's output.
 void tile_regions(const Net& net, int first, int last, int n, int m, int i, int j,
                   std::vector<Rect>& out_rects, std::vector<Rect>& in_rects);
+// The same traversal from any output rectangle of layer last.
+void rect_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
+                  std::vector<Rect>& in_rects);
+
+// Tile bounds of a group along one axis: n + 1 increasing values from 0 to len.
+// Empty `given` means the even partition.
+std::vector<int> axis_bounds(int len, int n, const std::vector<int>& given);
+// "" if `b` is a valid bounds vector for n parts of len (0 = b[0] < ... < b[n] = len).
+std::string check_bounds(const std::vector<int>& b, int len, int n);
+
+// Work-balanced bounds along one axis of group first..last (the non-uniform tiling of
+// Sec. 6): n parts of the last layer's output such that the largest part's executed
+// MACs (its regions back-traversed through every conv of the group, the other axis
+// taken whole) is as small as possible.  axis 0: rows, 1: columns.
+std::vector<int> balanced_bounds(const Net& net, int first, int last, int n, int axis);
 
 // Algorithm 1 (literal reading), MiB.
 double predict_layer_group(const Net& net, int first, int last, int n, int m, double bias_mib,
@@ -69,6 +85,8 @@ struct PlanConfig {
     int fixed_nblk = 0;       // force the output-channel block of every stage (0: choose)
     int fixed_mb = 0;         // force blocks per item (0: choose)
     int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
+    // explicit tile bounds per group (empty: even): rows[g] has grid_n[g] + 1 entries, cols[g] grid_m[g] + 1
+    std::vector<int> row_bounds[2], col_bounds[2];
 };
 
 // A tensor-map request for a task whose input is a scratch region buffer.
@@ -82,6 +100,7 @@ struct TmapReq {
 struct PlanTables {
     PlanConfig cfg;
     int groups[2][2];         // [g] = {first, last} layer
+    std::vector<int> rows[2], cols[2];   // tile bounds of each group on its last layer's output
     int stage_first[2], stage_last[2];   // stage index range per group
     std::vector<MafatStageDev> stages;
     std::vector<MafatTaskDev> tasks;

@@ -325,6 +325,16 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.fixed_nblk = o.force_nblk;
     cfg.fixed_mb = o.force_mb;
     cfg.lookahead_items = o.lookahead_items;
+    if (o.tile_bounds) {
+        // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
+        const int32_t* b = o.tile_bounds;
+        for (int g = 0; g < n_groups; ++g) {
+            cfg.row_bounds[g].assign(b, b + grid_n[g] + 1);
+            b += grid_n[g] + 1;
+            cfg.col_bounds[g].assign(b, b + grid_m[g] + 1);
+            b += grid_m[g] + 1;
+        }
+    }
     int sms = 0;
     if (!o.dry_run) {
         int dev = 0;
@@ -588,8 +598,12 @@ mafat_status mafat_tile_region(const mafat_plan_t* plan, int32_t group, int32_t 
         return fail(MAFAT_EINVAL, "tile out of range");
     if (layer < t.groups[group][0] || layer > t.groups[group][1]) return fail(MAFAT_EINVAL, "layer not in group");
     std::vector<mafat::Rect> outs, ins;
-    mafat::tile_regions(plan->shapes, t.groups[group][0], t.groups[group][1], t.cfg.grid_n[group],
-                        t.cfg.grid_m[group], ti, tj, outs, ins);
+    mafat::Rect r;
+    r.y0 = t.rows[group][ti];
+    r.y1 = t.rows[group][ti + 1];
+    r.x0 = t.cols[group][tj];
+    r.x1 = t.cols[group][tj + 1];
+    mafat::rect_regions(plan->shapes, t.groups[group][0], t.groups[group][1], r, outs, ins);
     const mafat::Rect& i = ins[layer];
     const mafat::Rect& o = outs[layer];
     in_rect[0] = i.y0; in_rect[1] = i.y1; in_rect[2] = i.x0; in_rect[3] = i.x1;
@@ -627,6 +641,20 @@ mafat_status mafat_predict_mem(const mafat_net_t* net, int32_t cut, int32_t n1, 
     if (!net || !out_mib) return fail(MAFAT_EINVAL, "null argument");
     if (n1 <= 0 || m1 <= 0 || n2 <= 0 || m2 <= 0) return fail(MAFAT_EINVAL, "grid sizes must be positive");
     *out_mib = mafat::predict_mem(net->net, cut, n1, m1, n2, m2, bias_mib);
+    return MAFAT_OK;
+}
+
+mafat_status mafat_balanced_bounds(const mafat_net_t* net, int32_t first, int32_t last, int32_t n, int32_t m,
+                                   int32_t* row_bounds, int32_t* col_bounds) {
+    if (!net || !row_bounds || !col_bounds) return fail(MAFAT_EINVAL, "null argument");
+    const int nl = (int)net->net.layers.size();
+    if (first < 0 || last >= nl || first > last) return fail(MAFAT_EINVAL, "bad layer range");
+    const mafat::Layer& L = net->net.layers[last];
+    if (n <= 0 || m <= 0 || n > L.h_out || m > L.w_out) return fail(MAFAT_EINVAL, "bad grid size");
+    const std::vector<int> r = mafat::balanced_bounds(net->net, first, last, n, 0);
+    const std::vector<int> c = mafat::balanced_bounds(net->net, first, last, m, 1);
+    std::copy(r.begin(), r.end(), row_bounds);
+    std::copy(c.begin(), c.end(), col_bounds);
     return MAFAT_OK;
 }
 

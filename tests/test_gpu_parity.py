@@ -237,6 +237,21 @@ def test_bf16_608_every_sweep_plan_default_shapes(mf):
             assert e <= TOL_BF16, "plan %s %s cut tensor: rel err %.3g" % (cut, grids, e)
 
 
+def test_bf16_608_nonuniform_tiling(mf):
+    # non-uniform tile bounds: the output equals the oracle's, and with the MMA shapes held
+    # fixed it is bit-identical to the even grid's
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    layers, params, x = wl["layers"], wl["params"], wl["input"]
+    bounds = [([0, 20, 30, 45, 60, 76], [0, 12, 30, 50, 64, 76]), ([0, 15, 38], [0, 24, 38])]
+    outs = oracle.forward(layers, params, x[0])
+    c, out = run_plan(mf, layers, params, x, 8, [(5, 5), (2, 2)], mf.BF16, plan_kwargs=dict(tile_bounds=bounds))
+    assert rel_err(out[0], outs[-1]) <= TOL_BF16 and rel_err(c[0], outs[7]) <= TOL_BF16
+    fixed = dict(force_nblk=32, force_mb=1)
+    _, a = run_plan(mf, layers, params, x, 8, [(5, 5), (2, 2)], mf.BF16, plan_kwargs=dict(tile_bounds=bounds, **fixed))
+    _, b = run_plan(mf, layers, params, x, 8, [(5, 5), (2, 2)], mf.BF16, plan_kwargs=fixed)
+    assert np.array_equal(a, b)
+
+
 def test_measured_search_picks_the_fastest_timed_plan(mf):
     # Algorithm 2 re-targeted at the GPU: candidates whose intermediates fit the L2 are timed,
     # the others refused; the fastest is reported, and it computes the network correctly

@@ -186,6 +186,23 @@ def test_yolo16_tiled_is_bit_identical_to_unfused(cut, t1, t2):
         assert np.array_equal(a, b)
 
 
+@pytest.mark.parametrize("cut,bounds", [
+    (8, [([0, 1, 5, 8], [0, 3, 4, 8]), ([0, 3, 4], [0, 1, 4])]),   # 64x64: group 1 ends at 8x8, group 2 at 4x4
+    (None, [([0, 2, 3, 4], [0, 1, 4])]),                           # one group, 3 x 2 uneven tiles of the 4x4 output
+    (12, [([0, 1, 4], [0, 1, 2, 3, 4]), ([0, 4], [0, 3, 4])]),  # both groups end at 4x4
+])
+def test_yolo16_uneven_tiling_is_bit_identical_to_unfused(cut, bounds):
+    # non-uniform grids (Sec. 6): any partition of the group outputs gives the unfused result
+    layers = synth.YOLO16
+    x = synth.make_input(1, 64, 64, 3, 23, "fp32")[0]
+    params = _params(layers, 3, 24)
+    grids = [(len(r) - 1, len(c) - 1) for r, c in bounds]
+    ref = oracle.group_outputs(layers, params, x, cut)
+    got = oracle.forward_tiled(layers, params, x, cut, grids, bounds)
+    for a, b in zip(got, ref):
+        assert np.array_equal(a, b)
+
+
 def test_region_that_misses_halo_is_rejected():
     # A region one row short of the receptive field must be refused, not silently padded.
     layers = [_conv_layer(3, 2)]

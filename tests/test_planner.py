@@ -179,3 +179,65 @@ def test_measured_search_dry_run_candidates(mf):
     assert len(ns) == 13 + 13 * 13
     assert all(abs(n - m) <= 1 for c in ns for n, m in c["grids"])
     assert (5, 4) in [c["grids"][0] for c in ns[:13]]
+
+
+def test_tile_regions_with_explicit_bounds_match_oracle(mf):
+    # a non-uniform tiling passed as tile bounds: every tile's regions equal the oracle's
+    layers = synth.YOLO16
+    net = _net(mf, layers, 608)
+    shapes = oracle.layer_shapes(layers, 608, 608, 3)
+    bounds = [([0, 20, 30, 45, 60, 76], [0, 12, 30, 50, 64, 76]), ([0, 15, 38], [0, 24, 38])]
+    plan = mf.Plan(net, 8, [(5, 5), (2, 2)], dry_run=True, tile_bounds=bounds)
+    for gi, g in enumerate(oracle.groups_of(len(layers), 8)):
+        rb, cb = bounds[gi]
+        for i in range(len(rb) - 1):
+            for j in range(len(cb) - 1):
+                ref = oracle.tile_regions(layers, shapes, g, len(rb) - 1, len(cb) - 1, i, j, (rb, cb))
+                for l in range(g[0], g[1] + 1):
+                    assert plan.tile_region(gi, i, j, l) == ref[l], (gi, i, j, l)
+    with pytest.raises(mf.MafatError):   # bounds must increase strictly and cover the map
+        mf.Plan(net, 8, [(5, 5), (2, 2)], dry_run=True,
+                tile_bounds=[([0, 20, 20, 45, 60, 76], bounds[0][1]), bounds[1]])
+    with pytest.raises(mf.MafatError):
+        mf.Plan(net, 8, [(5, 5), (2, 2)], dry_run=True, tile_bounds=[([0, 20, 30, 45, 76], bounds[0][1]), bounds[1]])
+
+
+def _band_work(layers, shapes, group, axis, lo, hi):
+    """Executed MACs of the band [lo, hi) of the group's output along `axis`, the other
+    axis whole, through the oracle's Grid traversal."""
+    first, last = group
+    sh = shapes[last]
+    size = sh["h_out"] if axis == 0 else sh["w_out"]
+    band = sorted({0, lo, hi, size})          # a partition with [lo, hi) as one of its parts
+    k = band.index(lo)
+    whole = [0, sh["w_out"] if axis == 0 else sh["h_out"]]
+    b = (band, whole) if axis == 0 else (whole, band)
+    n, m = (len(band) - 1, 1) if axis == 0 else (1, len(band) - 1)
+    regs = oracle.tile_regions(layers, shapes, group, n, m, *((k, 0) if axis == 0 else (0, k)), b)
+    w = 0
+    for l in range(first, last + 1):
+        t, k, s, p, f = layers[l]
+        if t == oracle.CONV:
+            (y0, y1, x0, x1), _ = regs[l]
+            w += (y1 - y0) * (x1 - x0) * shapes[l]["c_out"] * shapes[l]["c_in"] * k * k
+    return w
+
+
+@pytest.mark.parametrize("group,n", [((8, 15), 4), ((0, 15), 5), ((0, 7), 3), ((4, 11), 3)])
+def test_balanced_bounds_minimise_the_largest_part(mf, group, n):
+    # the work-balanced non-uniform tiling against exhaustive search over every partition
+    import itertools
+    layers = synth.YOLO16
+    net = _net(mf, layers, 608)
+    shapes = oracle.layer_shapes(layers, 608, 608, 3)
+    length = shapes[group[1]]["h_out"]
+    rows, cols = net.balanced_bounds(group[0], group[1], n, n)
+    assert rows == cols  # square map, same rule per axis
+    assert rows[0] == 0 and rows[-1] == length and all(a < b for a, b in zip(rows, rows[1:]))
+    work = {(a, b): _band_work(layers, shapes, group, 0, a, b) for a in range(length) for b in range(a + 1, length + 1)}
+    got = max(work[(a, b)] for a, b in zip(rows, rows[1:]))
+    best = min(max(work[(a, b)] for a, b in zip((0,) + cuts, cuts + (length,)))
+               for cuts in itertools.combinations(range(1, length), n - 1))
+    assert got == best
+    even = oracle.grid_bounds(length, n)
+    assert got <= max(work[r] for r in even)
