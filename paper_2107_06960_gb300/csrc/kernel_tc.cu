@@ -489,11 +489,11 @@ struct WeightBufs {
     }
 };
 
-// L2 prefetch of this CTA's 1/gridDim share of a buffer (16-byte aligned base), in
-// bulk prefetches of at most 64 KB; the tail below 16 bytes is left out.
-__device__ __forceinline__ void prefetch_l2_share(const void* base, int64_t bytes) {
+// L2 prefetch of this CTA's share (per bytes, computed on the host) of a buffer
+// (16-byte aligned base), in bulk prefetches of at most 64 KB; the tail below 16 bytes
+// is left out.
+__device__ __forceinline__ void prefetch_l2_share(const void* base, int64_t bytes, int64_t per) {
     if (base == nullptr || bytes <= 0) return;
-    const int64_t per = ((bytes + gridDim.x - 1) / gridDim.x + 15) & ~(int64_t)15;
     int64_t off = (int64_t)blockIdx.x * per;
     const int64_t end = min(bytes, off + per);
     for (; off < end; off += 65536) {
@@ -637,6 +637,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int64_t pipe_limit = 4 * p.timeout_ns + 1000000000LL;
+    // the producer's first item record, in flight while the CTA sets up
+    MafatItemDev it_first{};
+    if (warp == kProducerWarp && lane == 0 && (int)blockIdx.x < p.n_items) it_first = p.items[blockIdx.x];
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kAStages; ++i) {
@@ -684,7 +687,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // first use of every weight set and table entry on each SM); fetching them into
             // L2 at once, spread over all CTAs, overlaps those DRAM latencies instead of
             // paying them item by item.
-            for (int r = 0; r < MAFAT_PF_REGIONS; ++r) prefetch_l2_share(p.pf_ptr[r], p.pf_bytes[r]);
+            for (int r = 0; r < MAFAT_PF_REGIONS; ++r) prefetch_l2_share(p.pf_ptr[r], p.pf_bytes[r], p.pf_per[r]);
             uint32_t a_cnt = 0, q_cnt = 0;
             WeightBufs wb;
             // dependency counters already seen at (or above) a target: items of one task
@@ -697,9 +700,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             // stage with many items (lookahead) it is taken at once: every CTA has work then,
             // and the hand-out latency (atomic, record loads) is hidden behind the A stage's
             // release instead of added to it.
-            int next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
-            MafatItemDev it_next;
-            if (next < p.n_items) it_next = p.items[next];
+            // The first ticket is the CTA's index (the first gridDim.x items go out at once
+            // anyway), its record loaded during the setup; later tickets come from the atomic
+            // counter, offset by gridDim.x.
+            int next = (int)blockIdx.x;
+            MafatItemDev it_next = it_first;
             while (true) {
                 const int ticket = next < p.n_items ? next : -1;
                 const MafatItemDev it = it_next;
@@ -813,7 +818,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!st.lookahead)
                     mbar_wait(bar(kBarAEmpty + (int)(a_cnt % kAStages)), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr,
                               pipe_limit, broken, 64);
-                next = (int)atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u);
+                next = (int)(atomicAdd(&p.ctr[MAFAT_CTR_TICKET], 1u) + gridDim.x);
                 if (next < p.n_items) it_next = p.items[next];
             }
             // Drain: every copy issued has landed before the CTA may exit.

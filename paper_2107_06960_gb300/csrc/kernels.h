@@ -34,6 +34,7 @@ struct MafatKParams {
     // packed weights, the work tables and the scale / bias arrays (bytes 0: unused slot).
     const void* pf_ptr[MAFAT_PF_REGIONS];
     int64_t pf_bytes[MAFAT_PF_REGIONS];
+    int64_t pf_per[MAFAT_PF_REGIONS];   // each CTA's share of region r (bytes, multiple of 16)
 };
 
 // bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.

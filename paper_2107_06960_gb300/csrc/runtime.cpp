@@ -190,6 +190,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
         for (int i = 0; i < 7; ++i) {
             kp.pf_ptr[i] = pf[i];
             kp.pf_bytes[i] = pb[i];
+            kp.pf_per[i] = ((pb[i] + p->grid - 1) / p->grid + 15) & ~(int64_t)15;
         }
         if (p->in_map_ptr != input) {
             std::string err;

@@ -110,14 +110,10 @@ __device__ __forceinline__ void finish_cta(uint32_t* ctr, int n_ctr) {
     }
     __syncthreads();
     if (!s_last) return;
+    // the next launch on the stream starts after this one has completed, so these stores
+    // need no fence of their own
     for (int i = threadIdx.x; i < n_ctr; i += blockDim.x)
-        if (i != MAFAT_CTR_STATUS && i != MAFAT_CTR_EXIT) ctr[i] = 0u;
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        ctr[MAFAT_CTR_EXIT] = 0u;
-        __threadfence();
-    }
+        if (i != MAFAT_CTR_STATUS) ctr[i] = 0u;
 }
 
 }  // namespace mafat_dev
