@@ -97,6 +97,12 @@ typedef struct {
     const int32_t* tile_bounds; /* non-uniform tiling (NULL: the even N x M grid): for each group, its
                                    grid_n + 1 row bounds then its grid_m + 1 column bounds on the
                                    group's last-layer output, 0 = b[0] < b[1] < ... < b[n] = size */
+    int32_t halo_reuse;         /* 1: inter-tile reuse instead of halo recompute: a tile computes only
+                                   its own part of every layer, into whole layer maps on the device,
+                                   and reads the halo its next layer needs from its neighbours' parts
+                                   (each layer waits for those neighbours); 0: the fused tiles of
+                                   Sec. 3-4, every tile recomputing its halo */
+    int32_t reserved;
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */
@@ -206,7 +212,9 @@ mafat_status mafat_run_host_wait(const mafat_plan_t* plan);
 mafat_status mafat_sync_status(const mafat_plan_t* plan, void* stream);
 
 /* Host-side query of the Grid traversal (Sec. 4.1): input and output
- * rectangle of layer `layer` for tile (ti, tj) of group `group`. */
+ * rectangle of layer `layer` for tile (ti, tj) of group `group`.  With halo reuse
+ * the output rectangle is the part of the layer the tile computes (owns) and the
+ * input rectangle what that part reads (its neighbours' parts included). */
 mafat_status mafat_tile_region(const mafat_plan_t* plan, int32_t group, int32_t ti, int32_t tj,
                                int32_t layer, int32_t in_rect[4], int32_t out_rect[4]);
 

@@ -35,7 +35,7 @@ class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
                 ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32),
-                ("tile_bounds", ctypes.POINTER(i32))]
+                ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("reserved", i32)]
 
 
 class PlanStats(ctypes.Structure):
@@ -249,7 +249,7 @@ class Plan:
 
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
-                 force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None):
+                 force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False):
         self.net = net
         n_groups = 1 if cut is None else 2
         grids = list(grids)[:n_groups]
@@ -265,6 +265,7 @@ class Plan:
         opt.trace = 1 if trace else 0
         opt.force_nblk, opt.force_mb = force_nblk, force_mb
         opt.lookahead_items = lookahead_items
+        opt.halo_reuse = int(halo_reuse)
         if tile_bounds is not None:
             # per group (rows, cols): the non-uniform tiling; kept alive with the plan
             flat = [v for rows, cols in list(tile_bounds)[:n_groups] for v in list(rows) + list(cols)]

@@ -29,7 +29,15 @@
 #define MAFAT_A_STAGE_BYTES 36864   // shared-memory A halo stage of the tensor-core kernel (x2)
 #define MAFAT_B_PIECE_BYTES 75776   // one of the two shared-memory weight buffers (x2)
 
-enum { MAFAT_BUF_USER_IN = 0, MAFAT_BUF_CUT = 1, MAFAT_BUF_SCRATCH = 2, MAFAT_BUF_USER_OUT = 3 };
+// SCRATCH: a tile's own region buffer in the scratch ring (frame in the offset); MAP: a
+// whole layer-output map of every frame in the scratch allocation (halo reuse: tiles
+// read their neighbours' results from it; frame as the tensor map's fourth coordinate).
+enum { MAFAT_BUF_USER_IN = 0, MAFAT_BUF_CUT = 1, MAFAT_BUF_SCRATCH = 2, MAFAT_BUF_USER_OUT = 3, MAFAT_BUF_MAP = 4 };
+
+// One entry of a task's dependency list: wait until counter ctr reaches target.
+struct MafatDepDev {
+    int32_t ctr, target;
+};
 
 struct MafatStageDev {
     int32_t layer;        // network layer index of the conv
@@ -78,6 +86,7 @@ struct MafatTaskDev {
     int32_t out_y0, out_x0; // map position of buffer pixel (0, 0) (pooled map)
     int32_t done_ctr;     // counter bumped once per finished item
     int32_t n_items;
+    int32_t dep_first, dep_count;  // the task's own dependency list in the plan's list (halo reuse)
 };
 
 struct MafatItemDev {

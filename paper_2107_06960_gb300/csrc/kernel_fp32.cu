@@ -17,7 +17,8 @@ __device__ __forceinline__ const float* buf_ptr(const MafatKParams& p, int kind)
     switch (kind) {
         case MAFAT_BUF_USER_IN: return (const float*)p.user_in;
         case MAFAT_BUF_CUT: return (const float*)p.cut;
-        case MAFAT_BUF_SCRATCH: return (const float*)p.scratch;
+        case MAFAT_BUF_SCRATCH:
+        case MAFAT_BUF_MAP: return (const float*)p.scratch;
         default: return (const float*)p.user_out;
     }
 }
@@ -40,6 +41,7 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
                 mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
             }
             mafat_dev::wait_item_deps(p.ctr, it, p.timeout_ns);
+            if (tk.dep_count > 0) mafat_dev::wait_dep_list(p.ctr, p.deps, tk.dep_first, tk.dep_count, p.timeout_ns);
             if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
         }
         __syncthreads();

@@ -693,6 +693,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // dependency counters already seen at (or above) a target: items of one task
             // usually follow each other, so most items skip the round trip to L2
             int ok_idx0 = -1, ok_idx1 = -1, ok_tgt0 = 0, ok_tgt1 = 0;
+            int ok_task = -1;  // the last task whose dependency list was found complete
             // A ticket is taken (and its item record loaded) at the end of the previous item,
             // once the A stage the new item will use is about to free: early enough to hide
             // the new item's loads behind the current MMAs, late enough that a CTA busy with a
@@ -799,6 +800,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::wait_counter(p.ctr, it.dep1, it.dep1_target, p.timeout_ns);
                     ok_idx1 = it.dep1;
                     ok_tgt1 = it.dep1_target;
+                    waited = true;
+                }
+                if (tk.dep_count > 0 && it.task != ok_task) {
+                    mafat_dev::wait_dep_list(p.ctr, p.deps, tk.dep_first, tk.dep_count, p.timeout_ns);
+                    ok_task = it.task;
                     waited = true;
                 }
                 if (waited) mafat_dev::fence_proxy_async_global();

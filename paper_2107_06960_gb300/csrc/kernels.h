@@ -35,6 +35,7 @@ struct MafatKParams {
     const void* pf_ptr[MAFAT_PF_REGIONS];
     int64_t pf_bytes[MAFAT_PF_REGIONS];
     int64_t pf_per[MAFAT_PF_REGIONS];   // each CTA's share of region r (bytes, multiple of 16)
+    const MafatDepDev* deps;            // task dependency lists (halo reuse)
 };
 
 // bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.

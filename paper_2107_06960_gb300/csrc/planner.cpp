@@ -139,6 +139,27 @@ std::vector<int> balanced_bounds(const Net& net, int first, int last, int n, int
     return bounds;
 }
 
+// Halo reuse: the part of every layer's output a tile owns (its group-output rectangle
+// scaled through the max-pools, never grown by a convolution's halo: stride-1 convs keep
+// the map size), and the input region each layer reads for it (halo included, computed
+// by the neighbours that own it).
+void owned_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
+                   std::vector<Rect>& in_rects) {
+    Rect r = out_last;
+    if ((int)out_rects.size() < (int)net.layers.size()) out_rects.resize(net.layers.size());
+    if ((int)in_rects.size() < (int)net.layers.size()) in_rects.resize(net.layers.size());
+    for (int l = last; l >= first; --l) {
+        const Layer& L = net.layers[l];
+        Rect in;
+        back_interval(r.y0, r.y1, L.k, L.stride, L.pad, L.h_in, &in.y0, &in.y1);
+        back_interval(r.x0, r.x1, L.k, L.stride, L.pad, L.w_in, &in.x0, &in.x1);
+        if (r.empty()) in = Rect{};
+        out_rects[l] = r;
+        in_rects[l] = in;
+        if (L.type == L_MAXPOOL) r = Rect{2 * r.y0, 2 * r.y1, 2 * r.x0, 2 * r.x1};
+    }
+}
+
 void rect_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
                   std::vector<Rect>& in_rects) {
     Rect r = out_last;
@@ -272,7 +293,10 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 r.y1 = t.rows[g][i + 1];
                 r.x0 = t.cols[g][j];
                 r.x1 = t.cols[g][j + 1];
-                rect_regions(net, t.groups[g][0], t.groups[g][1], r, ti.outs, ti.ins);
+                if (cfg.halo_reuse)
+                    owned_regions(net, t.groups[g][0], t.groups[g][1], r, ti.outs, ti.ins);
+                else
+                    rect_regions(net, t.groups[g][0], t.groups[g][1], r, ti.outs, ti.ins);
                 if (ti.outs[t.groups[g][1]].empty()) continue;
                 tiles[g].push_back(std::move(ti));
             }
@@ -431,7 +455,12 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
 
     int S = cfg.ring_slots > 0 ? cfg.ring_slots : std::min(max_tiles, 64);
     int W = cfg.wave_tiles > 0 ? std::min(cfg.wave_tiles, S) : S;
-    t.ring_slots = S;
+    if (cfg.halo_reuse) {
+        // a layer's tasks read their neighbours' previous layer, so every tile of a group
+        // goes out stage by stage in one wave; there is no ring
+        S = W = max_tiles;
+    }
+    t.ring_slots = cfg.halo_reuse ? 0 : S;
     t.wave_tiles = W;
 
     // ---- scratch buffer size: largest non-final stage output of any tile
@@ -445,6 +474,41 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 buf = std::max(buf, (int64_t)r.h() * r.w() * ceil_div(st.cout, 8) * 8);
             }
     t.slot_buf_elems = (buf + 127) / 128 * 128;  // 256-byte aligned for bf16, 512 for fp32
+    t.scratch_elems = (int64_t)S * 2 * t.slot_buf_elems;
+    // halo reuse: one whole output map per non-final stage, every frame, instead of the ring
+    std::vector<int64_t> map_off(t.stages.size(), -1), map_frame(t.stages.size(), 0);
+    std::vector<int> map_h(t.stages.size(), 0), map_w(t.stages.size(), 0), stage_tmap(t.stages.size(), -1);
+    if (cfg.halo_reuse) {
+        int64_t off = 0;
+        for (int g = 0; g < G; ++g)
+            for (int s = t.stage_first[g]; s < t.stage_last[g]; ++s) {
+                const MafatStageDev& st = t.stages[s];
+                const Layer& Lo = net.layers[stage_pool_layer[s] >= 0 ? stage_pool_layer[s] : st.layer];
+                map_h[s] = Lo.h_out;
+                map_w[s] = Lo.w_out;
+                map_frame[s] = (int64_t)ceil_div(st.cout, 8) * 8 * Lo.h_out * Lo.w_out;
+                map_off[s] = off;
+                off += (map_frame[s] * cfg.batch + 127) / 128 * 128;
+            }
+        t.scratch_elems = std::max<int64_t>(off, 128);
+        t.slot_buf_elems = 0;
+        for (int g = 0; g < G; ++g)
+            for (int s = t.stage_first[g] + 1; s <= t.stage_last[g]; ++s) {
+                const MafatStageDev& st = t.stages[s];
+                TmapReq req{};
+                req.task = -1;
+                req.elem_off = map_off[s - 1];
+                req.h = map_h[s - 1];
+                req.w = map_w[s - 1];
+                req.c8 = st.cin8;
+                req.frames = cfg.batch;
+                req.rows_box = st.rows_box;
+                req.cols_box = st.cols_box;
+                req.chunk8 = st.chunk8;
+                stage_tmap[s] = (int)t.tmaps.size();
+                t.tmaps.push_back(req);
+            }
+    }
 
     // ---- tasks in hand-out order, with their dependencies expressed as task indices
     struct TaskDep {
@@ -464,6 +528,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 for (int s = t.stage_first[g]; s <= t.stage_last[g]; ++s) {
                     const MafatStageDev& st = t.stages[s];
                     const Layer& Lc = net.layers[st.layer];
+                    const std::vector<int> prev_stage_task = prev_of_tile;  // stage s - 1's task of each tile
                     for (size_t q = w0; q < w1; ++q) {
                         const TileInfo& ti = tl[q];
                         int tseq = seq + (int)(q - w0);
@@ -496,6 +561,14 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             tk.in_w = Lc.w_in;
                             tk.in_y0 = 0;
                             tk.in_x0 = 0;
+                        } else if (cfg.halo_reuse) {
+                            tk.in_kind = MAFAT_BUF_MAP;
+                            tk.in_off = map_off[s - 1] + f * map_frame[s - 1];
+                            tk.in_h = map_h[s - 1];
+                            tk.in_w = map_w[s - 1];
+                            tk.in_y0 = 0;
+                            tk.in_x0 = 0;
+                            tk.in_tmap = stage_tmap[s];
                         } else {
                             int b = (slot * 2) + ((rel - 1) & 1);
                             tk.in_kind = MAFAT_BUF_SCRATCH;
@@ -506,8 +579,8 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             tk.in_x0 = ir.x0;
                             TmapReq req{};
                             req.task = (int)t.tasks.size();
-                            req.slot = slot;
-                            req.buf = b;
+                            req.elem_off = (int64_t)b * t.slot_buf_elems;
+                            req.frames = 1;
                             req.h = ir.h();
                             req.w = ir.w();
                             req.c8 = st.cin8;
@@ -533,6 +606,14 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             }
                             tk.out_y0 = 0;
                             tk.out_x0 = 0;
+                        } else if (cfg.halo_reuse) {
+                            tk.out_kind = MAFAT_BUF_MAP;
+                            tk.out_nhwc = 0;
+                            tk.out_off = map_off[s] + f * map_frame[s];
+                            tk.out_h = map_h[s];
+                            tk.out_w = map_w[s];
+                            tk.out_y0 = 0;
+                            tk.out_x0 = 0;
                         } else {
                             int b = (slot * 2) + (rel & 1);
                             tk.out_kind = MAFAT_BUF_SCRATCH;
@@ -547,8 +628,24 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         TaskDep d;
                         int qi = (int)(q - w0);
                         if (s == t.stage_first[g]) {
-                            if (tseq >= S) d.prev_task = last_task_of_seq[tseq - S];
+                            if (!cfg.halo_reuse && tseq >= S) d.prev_task = last_task_of_seq[tseq - S];
                             if (g == 1) d.frame_g1 = f;
+                        } else if (cfg.halo_reuse) {
+                            // every previous-stage task whose owned output meets this task's input
+                            // region (halo included): itself and the neighbours around it
+                            const int ps = s - 1;
+                            const int pol = stage_pool_layer[ps] >= 0 ? stage_pool_layer[ps] : t.stages[ps].layer;
+                            const Rect& need = ti.ins[st.layer];
+                            tk.dep_first = (int)t.deps.size();
+                            for (size_t q2 = w0; q2 < w1; ++q2) {
+                                const Rect& own = tl[q2].outs[pol];
+                                if (own.empty() || need.empty() || own.y1 <= need.y0 || need.y1 <= own.y0 ||
+                                    own.x1 <= need.x0 || need.x1 <= own.x0)
+                                    continue;
+                                const int pt = prev_stage_task[q2 - w0];
+                                t.deps.push_back(MafatDepDev{MAFAT_CTR_BASE + pt, t.tasks[pt].n_items});
+                            }
+                            tk.dep_count = (int)t.deps.size() - tk.dep_first;
                         } else {
                             d.prev_task = prev_of_tile[qi];
                         }
@@ -647,7 +744,8 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     const int64_t in_total = (int64_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in;
     const int64_t cut_total = (int64_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_total = (int64_t)t.cfg.batch * t.out_h * t.out_w * t.out_c;
-    const int64_t scratch_total = (int64_t)t.ring_slots * 2 * t.slot_buf_elems;
+    const int64_t scratch_total = t.scratch_elems;
+    if (!t.cfg.halo_reuse && scratch_total != (int64_t)t.ring_slots * 2 * t.slot_buf_elems) return "bad scratch size";
     auto buf_total = [&](int kind) {
         return kind == MAFAT_BUF_USER_IN ? in_total
                : kind == MAFAT_BUF_CUT   ? cut_total
@@ -697,6 +795,14 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (k.in_y0 + k.in_h > L.h_in || k.in_x0 + k.in_w > L.w_in || k.in_y0 < 0 || k.in_x0 < 0)
             return "input region outside the map";
         if (k.in_kind == MAFAT_BUF_SCRATCH && k.in_off % t.slot_buf_elems != 0) return "scratch input misaligned";
+        if ((k.in_kind == MAFAT_BUF_MAP) != (k.out_kind == MAFAT_BUF_MAP) && !t.cfg.halo_reuse) return "layer map without halo reuse";
+        if (k.dep_count < 0 || k.dep_first < 0 || k.dep_first + k.dep_count > (int)t.deps.size()) return "bad dependency list";
+        for (int d = k.dep_first; d < k.dep_first + k.dep_count; ++d) {
+            const int dt = t.deps[d].ctr - MAFAT_CTR_BASE;
+            if (dt < 0 || dt >= n_tasks) return "dependency list names no task";
+            if (t.deps[d].target != t.tasks[dt].n_items) return "dependency list target mismatch";
+            if (last_item[dt] >= first_item[ti]) return "dependency list names a later task";
+        }
         // output extent of the valid pixels
         int oy0 = k.cy0, oy1 = k.cy0 + k.ch, ox0 = k.cx0, ox1 = k.cx0 + k.cw;
         if (s.pool) {

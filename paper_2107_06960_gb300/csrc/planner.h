@@ -48,6 +48,10 @@ void back_interval(int a, int b, int k, int s, int p, int size_in, int* lo, int*
 // of the even n x m grid on layer last's output.
 void tile_regions(const Net& net, int first, int last, int n, int m, int i, int j,
                   std::vector<Rect>& out_rects, std::vector<Rect>& in_rects);
+// Halo reuse: the part of every layer's output a tile owns and the input region each
+// layer reads for it (vectors indexed by layer, as above).
+void owned_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
+                   std::vector<Rect>& in_rects);
 // The same traversal from any output rectangle of layer last.
 void rect_regions(const Net& net, int first, int last, const Rect& out_last, std::vector<Rect>& out_rects,
                   std::vector<Rect>& in_rects);
@@ -84,6 +88,8 @@ struct PlanConfig {
     int n_ctas = 0;           // persistent CTAs (shapes items; 0: 152)
     int fixed_nblk = 0;       // force the output-channel block of every stage (0: choose)
     int fixed_mb = 0;         // force blocks per item (0: choose)
+    bool halo_reuse = false;  // tiles compute only their own part of every layer and read the halo from
+                              // their neighbours' results in whole layer maps (no recompute)
     int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
     // explicit tile bounds per group (empty: even): rows[g] has grid_n[g] + 1 entries, cols[g] grid_m[g] + 1
     std::vector<int> row_bounds[2], col_bounds[2];
@@ -92,8 +98,8 @@ struct PlanConfig {
 // A tensor-map request for a task whose input is a scratch region buffer.
 struct TmapReq {
     int task;
-    int slot, buf;            // scratch ring slot and ping-pong buffer
-    int h, w, c8;             // buffer extent
+    int64_t elem_off;         // buffer start in the scratch allocation (elements)
+    int h, w, c8, frames;     // buffer extent (frames: 1 for a tile buffer, batch for a layer map)
     int rows_box, cols_box, chunk8;
 };
 
@@ -110,6 +116,8 @@ struct PlanTables {
     int64_t weight32_elems = 0;          // fp32 weight elements
     int64_t sb_elems = 0;                // scale / bias elements
     int64_t slot_buf_elems = 0;          // elements of one ping-pong buffer
+    int64_t scratch_elems = 0;           // the scratch allocation (ring, or layer maps with halo reuse)
+    std::vector<MafatDepDev> deps;       // task dependency lists (halo reuse)
     int ring_slots = 0, wave_tiles = 0;
     int n_counters = 0;                  // words after MAFAT_CTR_BASE
     int frame_ctr_base = 0;              // per-frame group-1 completion counters

@@ -33,6 +33,7 @@ struct mafat_plan_s {
     MafatStageDev* d_stages = nullptr;
     MafatTaskDev* d_tasks = nullptr;
     MafatItemDev* d_items = nullptr;
+    MafatDepDev* d_deps = nullptr;
     CUtensorMap* d_tmaps = nullptr;
     void* d_w = nullptr;
     float* d_scale = nullptr;
@@ -165,6 +166,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
     kp.stages = p->d_stages;
     kp.tasks = p->d_tasks;
     kp.items = p->d_items;
+    kp.deps = p->d_deps;
     kp.n_items = (int32_t)p->t.items.size();
     kp.tmaps = p->d_tmaps;
     kp.cut_tmap = p->t.cfg.n_groups == 2 ? (int)p->t.tmaps.size() : -1;
@@ -222,6 +224,7 @@ mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* 
     k.stages = p->d_stages;
     k.tasks = p->d_tasks;
     k.items = p->d_items;
+    k.deps = p->d_deps;
     k.n_items = (int32_t)p->t.items.size();
     k.tmaps = nullptr;
     k.cut_tmap = -1;
@@ -326,6 +329,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.fixed_nblk = o.force_nblk;
     cfg.fixed_mb = o.force_mb;
     cfg.lookahead_items = o.lookahead_items;
+    cfg.halo_reuse = o.halo_reuse != 0;
     if (o.tile_bounds) {
         // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
         const int32_t* b = o.tile_bounds;
@@ -366,7 +370,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     p->out_bytes = (size_t)t.cfg.batch * t.out_h * t.out_w * t.out_c * p->esz;
     p->cut_bytes = (size_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w * p->esz;
     p->ctr_bytes = (size_t)(MAFAT_CTR_BASE + t.n_counters) * sizeof(uint32_t);
-    p->scratch_bytes = (int64_t)t.ring_slots * 2 * t.slot_buf_elems * p->esz;
+    p->scratch_bytes = t.scratch_elems * p->esz;
     p->weight_bytes = (dt == MAFAT_BF16 ? t.weight_elems * 2 : t.weight32_elems * 4) + 2 * t.sb_elems * 4;
     if (p->dry_run) {
         *out = p;
@@ -391,6 +395,12 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     if ((e = dalloc(p, &p->d_stages, t.stages.size() * sizeof(MafatStageDev))) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_tasks, t.tasks.size() * sizeof(MafatTaskDev))) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_items, t.items.size() * sizeof(MafatItemDev))) != cudaSuccess) return bail(e, "cudaMalloc");
+    if (!t.deps.empty()) {
+        if ((e = dalloc(p, &p->d_deps, t.deps.size() * sizeof(MafatDepDev))) != cudaSuccess) return bail(e, "cudaMalloc");
+        if ((e = cudaMemcpy(p->d_deps, t.deps.data(), t.deps.size() * sizeof(MafatDepDev), cudaMemcpyHostToDevice)) !=
+            cudaSuccess)
+            return bail(e, "cudaMemcpy");
+    }
     if ((e = dalloc(p, &p->d_ctr, p->ctr_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_scale, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_bias, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
@@ -427,8 +437,8 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
         std::string merr;
         for (size_t i = 0; i < t.tmaps.size(); ++i) {
             const mafat::TmapReq& q = t.tmaps[i];
-            const char* base = (const char*)p->d_scratch + (size_t)q.buf * t.slot_buf_elems * 2;
-            if (!encode_planar_map(&maps[i], base, q.w, q.h, q.c8, 1, q.cols_box, q.rows_box, q.chunk8, &merr)) {
+            const char* base = (const char*)p->d_scratch + (size_t)q.elem_off * 2;
+            if (!encode_planar_map(&maps[i], base, q.w, q.h, q.c8, q.frames, q.cols_box, q.rows_box, q.chunk8, &merr)) {
                 free_plan_memory(p);
                 delete p;
                 return fail(MAFAT_ECUDA, merr);
@@ -604,7 +614,10 @@ mafat_status mafat_tile_region(const mafat_plan_t* plan, int32_t group, int32_t 
     r.y1 = t.rows[group][ti + 1];
     r.x0 = t.cols[group][tj];
     r.x1 = t.cols[group][tj + 1];
-    mafat::rect_regions(plan->shapes, t.groups[group][0], t.groups[group][1], r, outs, ins);
+    if (t.cfg.halo_reuse)
+        mafat::owned_regions(plan->shapes, t.groups[group][0], t.groups[group][1], r, outs, ins);
+    else
+        mafat::rect_regions(plan->shapes, t.groups[group][0], t.groups[group][1], r, outs, ins);
     const mafat::Rect& i = ins[layer];
     const mafat::Rect& o = outs[layer];
     in_rect[0] = i.y0; in_rect[1] = i.y1; in_rect[2] = i.x0; in_rect[3] = i.x1;

@@ -62,6 +62,35 @@ __device__ __forceinline__ void wait_counter(uint32_t* ctr, int idx, int target,
     }
 }
 
+__device__ __forceinline__ uint32_t ld_relaxed_u32(const uint32_t* p) {
+    uint32_t v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Wait for every entry of a task's dependency list (halo reuse: the tasks of the previous
+// layer around it).  The counters are read together, eight at a time (independent relaxed
+// loads, one round trip), and only those still short are polled; a fence then gives the
+// reads acquire order.
+__device__ __forceinline__ void wait_dep_list(uint32_t* ctr, const MafatDepDev* deps, int first, int count,
+                                              int64_t timeout_ns) {
+    for (int d0 = 0; d0 < count; d0 += 8) {
+        const int n = min(8, count - d0);
+        MafatDepDev e[8];
+        uint32_t v[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (i < n) e[i] = deps[first + d0 + i];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (i < n) v[i] = ld_relaxed_u32(ctr + e[i].ctr);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (i < n && v[i] < (uint32_t)e[i].target) wait_counter(ctr, e[i].ctr, e[i].target, timeout_ns);
+    }
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+
 // Wait for both dependencies of an item; afterwards the data they published is
 // visible to this thread's generic and async-proxy (TMA) reads.
 __device__ __forceinline__ void wait_item_deps(uint32_t* ctr, const MafatItemDev& it, int64_t timeout_ns) {

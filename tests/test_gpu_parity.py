@@ -252,6 +252,40 @@ def test_bf16_608_nonuniform_tiling(mf):
     assert np.array_equal(a, b)
 
 
+@pytest.mark.parametrize("cut,grids", [(8, [(5, 5), (2, 2)]), (None, [(3, 3)]), (2, [(4, 4), (3, 3)]),
+                                       (12, [(3, 2), (2, 3)])])
+def test_bf16_yolo16_96_halo_reuse_batch2(mf, cut, grids):
+    # inter-tile reuse (tiles read their neighbours' parts of the previous layer): the same
+    # outputs as the oracle, and bit-identical to halo recompute with fixed MMA shapes
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 41, "bf16")
+    x = synth.make_input(2, 96, 96, 3, 42, "bf16")
+    c, out = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=dict(halo_reuse=True))
+    refs = _oracle_groups(layers, params, x, cut, ("bf16_96", cut is None and 16 or cut))
+    _check_groups(c, out, refs, cut, TOL_BF16)
+    fixed = dict(force_nblk=32, force_mb=1)
+    _, a = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=dict(halo_reuse=True, **fixed))
+    _, b = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=fixed)
+    assert np.array_equal(a, b)
+
+
+def test_fp32_yolo16_96_halo_reuse(mf):
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 31, "fp32")
+    x = synth.make_input(2, 96, 96, 3, 32, "fp32")
+    c, out = run_plan(mf, layers, params, x, 8, [(3, 3), (2, 2)], mf.FP32, plan_kwargs=dict(halo_reuse=True))
+    _check_groups(c, out, _oracle_groups(layers, params, x, 8, ("fp32_96", 8)), 8, TOL_FP32)
+
+
+@pytest.mark.parametrize("name", ["yolo16_608_5x5_c8_2x2", "yolo25_608_5x5_c8_2x2"])
+def test_bf16_608_halo_reuse(mf, name):
+    wl = synth.workload(name)
+    c, out = run_plan(mf, wl["layers"], wl["params"], wl["input"], wl["cut"], wl["grids"], mf.BF16,
+                      plan_kwargs=dict(halo_reuse=True))
+    _check_groups(c, out, _oracle_groups(wl["layers"], wl["params"], wl["input"], wl["cut"], name), wl["cut"],
+                  TOL_BF16)
+
+
 def test_measured_search_picks_the_fastest_timed_plan(mf):
     # Algorithm 2 re-targeted at the GPU: candidates whose intermediates fit the L2 are timed,
     # the others refused; the fastest is reported, and it computes the network correctly

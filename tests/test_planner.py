@@ -241,3 +241,30 @@ def test_balanced_bounds_minimise_the_largest_part(mf, group, n):
     assert got == best
     even = oracle.grid_bounds(length, n)
     assert got <= max(work[r] for r in even)
+
+
+@pytest.mark.parametrize("cut,grids", [(None, [(5, 5)]), (2, [(4, 4), (3, 3)]), (8, [(5, 5), (2, 2)]),
+                                       (12, [(3, 2), (2, 3)])])
+def test_halo_reuse_plan_computes_each_pixel_once(mf, cut, grids):
+    # inter-tile reuse: every tile owns a part of every layer (the group-output tile scaled
+    # through the pools), the parts partition each map, and nothing is recomputed
+    layers = synth.YOLO16
+    net = _net(mf, layers, 608)
+    shapes = oracle.layer_shapes(layers, 608, 608, 3)
+    plan = mf.Plan(net, cut, grids, dry_run=True, halo_reuse=True)
+    st = plan.stats()
+    assert st["executed_flops"] == st["useful_flops"]
+    for gi, g in enumerate(oracle.groups_of(len(layers), cut)):
+        n, m = grids[gi]
+        for l in range(g[0], g[1] + 1):
+            cover = np.zeros((shapes[l]["h_out"], shapes[l]["w_out"]), dtype=np.int64)
+            for i in range(n):
+                for j in range(m):
+                    (oy0, oy1, ox0, ox1), (iy0, iy1, ix0, ix1) = plan.tile_region(gi, i, j, l)
+                    cover[oy0:oy1, ox0:ox1] += 1
+                    t, k, s, p, f = layers[l]
+                    # the input region is the owned part's receptive field, clipped to the map
+                    if oy1 > oy0 and ox1 > ox0:
+                        assert (iy0, iy1) == (max(oy0 * s - p, 0), min((oy1 - 1) * s - p + k, shapes[l]["h_in"]))
+                        assert (ix0, ix1) == (max(ox0 * s - p, 0), min((ox1 - 1) * s - p + k, shapes[l]["w_in"]))
+            assert np.all(cover == 1), (g, l)
