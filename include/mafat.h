@@ -55,6 +55,9 @@ typedef enum {
 
 typedef enum { MAFAT_CONV = 0, MAFAT_MAXPOOL = 1 } mafat_layer_type;
 
+/* Most layer groups a plan may have (the paper uses one or two). */
+#define MAFAT_MAX_GROUPS 4
+
 /* Arithmetic of a plan.  BF16: bf16 activations and weights, fp32 accumulation
  * on the tensor cores (tcgen05), every layer output rounded to bf16.  FP32: the
  * same fused tiling computed in fp32 on the CUDA cores (a check mode). */
@@ -147,8 +150,9 @@ mafat_status mafat_net_shape(const mafat_net_t* net, int32_t layer, int32_t shap
 mafat_status mafat_set_weights(mafat_net_t* net, int32_t layer, const float* w_host,
                                const float* scale, const float* bias);
 
-/* Plan fused-tile execution (Sec. 4): n_groups (1 or 2) layer groups split at
- * cuts[0] (ignored for one group), group g tiled grid_n[g] x grid_m[g], for
+/* Plan fused-tile execution (Sec. 4): n_groups (1..MAFAT_MAX_GROUPS; the paper
+ * uses 1 or 2) layer groups split at the increasing cuts[0..n_groups-2] (the
+ * first layer of each later group), group g tiled grid_n[g] x grid_m[g], for
  * `batch` images, in dtype dt.  The plan owns its device workspace (packed
  * weights, cut tensor, tile buffers, counters) on the current device; every
  * convolution must have weights set.  ENOFIT if a tile cannot be scheduled,

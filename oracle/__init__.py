@@ -16,8 +16,8 @@ Contents, each following the paper (MAFAT, arXiv 2107.06960):
 * ``predict_layer_group`` / ``predict_mem`` -- the memory predictor (Algorithm 1).
 * ``get_config``        -- the configuration search (Algorithm 2).
 * ``forward``           -- layer-by-layer fp64 forward (the plain definition).
-* ``forward_tiled``     -- the same network executed as fused tiles of up to two
-                           layer groups, merged and re-tiled at the cut (Sec. 4).
+* ``forward_tiled``     -- the same network executed as fused tiles of its layer
+                           groups, merged and re-tiled at every cut (Sec. 4).
 
 Readings of passages that are garbled or silent are stated where they are used.
 Parity of the predictor's absolute values beyond its units is unpinned (the
@@ -92,12 +92,16 @@ def layer_shapes(layers, h, w, c):
 def groups_of(n_layers, cut):
     """Layer groups for a cut (Sec. 4): group 1 is layers 0..cut-1, group 2 is
     cut..n-1.  The paper writes "to layer n"; with 0-based layers that is n-1.
-    A cut of None (or n, the paper's "16" / NoCut) means a single group."""
-    if cut is None or cut >= n_layers:
+    A cut of None (or n, the paper's "16" / NoCut) means a single group.  A list
+    of increasing cuts gives more groups the same way (the paper uses at most
+    two; more is the generalisation its Sec. 6 points to)."""
+    if cut is None or (not isinstance(cut, (list, tuple)) and cut >= n_layers):
         return [(0, n_layers - 1)]
-    if cut <= 0:
-        raise ValueError("cut must be in 1..n-1")
-    return [(0, cut - 1), (cut, n_layers - 1)]
+    cuts = list(cut) if isinstance(cut, (list, tuple)) else [cut]
+    if any(c <= 0 or c >= n_layers for c in cuts) or any(a >= b for a, b in zip(cuts, cuts[1:])):
+        raise ValueError("cuts must increase within 1..n-1")
+    bounds = [0] + cuts + [n_layers]
+    return [(a, b - 1) for a, b in zip(bounds, bounds[1:])]
 
 
 def grid_bounds(length, n):
@@ -284,7 +288,7 @@ def forward(layers, params, x):
 
 
 def group_outputs(layers, params, x, cut):
-    """Outputs of each layer group (the cut tensor, then the final output) of one image."""
+    """Outputs of each layer group (the cut tensors, then the final output) of one image."""
     outs = forward(layers, params, x)
     return [outs[last] for (first, last) in groups_of(len(layers), cut)]
 
@@ -317,11 +321,11 @@ def _region_layer(layer, prm, buf, in_rect, map_hw, out_rect):
 
 
 def forward_tiled(layers, params, x, cut, grids, bounds=None):
-    """Fused tile partitioning with up to two layer groups (Sec. 3, Sec. 4).
+    """Fused tile partitioning of the layer groups of ``cut`` (Sec. 3, Sec. 4).
 
     Each group's last-layer output is split into an N x M grid; every tile
     runs all layers of its group on its own regions (recomputing the overlap),
-    and writes its rectangle of the group output.  Group 2 re-tiles the merged
+    and writes its rectangle of the group output.  The next group re-tiles the merged
     cut tensor.  ``bounds`` (one (row bounds, column bounds) pair per group, or
     None) gives non-uniform grids.  Returns the group outputs; raises if the
     tiles do not cover the group output exactly once.

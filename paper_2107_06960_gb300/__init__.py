@@ -251,11 +251,14 @@ class Plan:
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
                  force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False):
         self.net = net
-        n_groups = 1 if cut is None else 2
+        # cut: None (one group), the first layer of group 2, or a list of increasing cuts
+        cut_list = [] if cut is None else (list(cut) if isinstance(cut, (list, tuple)) else [cut])
+        n_groups = 1 + len(cut_list)
         grids = list(grids)[:n_groups]
-        gn = (i32 * 2)(*[g[0] for g in grids] + [1] * (2 - len(grids)))
-        gm = (i32 * 2)(*[g[1] for g in grids] + [1] * (2 - len(grids)))
-        cuts = (i32 * 1)(cut if cut is not None else 0)
+        width = max(2, n_groups)
+        gn = (i32 * width)(*[g[0] for g in grids] + [1] * (width - len(grids)))
+        gm = (i32 * width)(*[g[1] for g in grids] + [1] * (width - len(grids)))
+        cuts = (i32 * max(1, len(cut_list)))(*(cut_list or [0]))
         opt = PlanOptions()
         opt.struct_size = ctypes.sizeof(PlanOptions)
         opt.ring_slots, opt.wave_tiles, opt.max_ctas = ring_slots, wave_tiles, max_ctas

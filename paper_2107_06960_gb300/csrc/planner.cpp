@@ -257,18 +257,19 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     const int n = (int)net.layers.size();
     t = PlanTables{};
     t.cfg = cfg;
-    if (cfg.n_groups != 1 && cfg.n_groups != 2) return "n_groups must be 1 or 2";
-    if (cfg.n_groups == 2 && (cfg.cut <= 0 || cfg.cut >= n)) return "cut must be in 1..n-1";
+    if (cfg.n_groups < 1 || cfg.n_groups > MAFAT_MAX_GROUPS) return "n_groups must be 1..4";
+    for (int c = 0; c + 1 < cfg.n_groups; ++c) {
+        if (cfg.cuts[c] <= 0 || cfg.cuts[c] >= n) return "cuts must be in 1..n-1";
+        if (c > 0 && cfg.cuts[c] <= cfg.cuts[c - 1]) return "cuts must increase";
+    }
     if (cfg.batch <= 0) return "batch must be positive";
     if (cfg.dtype != 0 && cfg.dtype != 1) return "unknown dtype";
     for (int g = 0; g < cfg.n_groups; ++g)
         if (cfg.grid_n[g] <= 0 || cfg.grid_m[g] <= 0) return "grid sizes must be positive";
     const int G = cfg.n_groups;
-    t.groups[0][0] = 0;
-    t.groups[0][1] = G == 2 ? cfg.cut - 1 : n - 1;
-    if (G == 2) {
-        t.groups[1][0] = cfg.cut;
-        t.groups[1][1] = n - 1;
+    for (int g = 0; g < G; ++g) {
+        t.groups[g][0] = g == 0 ? 0 : cfg.cuts[g - 1];
+        t.groups[g][1] = g == G - 1 ? n - 1 : cfg.cuts[g] - 1;
     }
 
     // ---- tiles of every group (non-empty only), on the even grid or the given bounds
@@ -435,7 +436,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     t.in_rows_box = s_in.rows_box;
     t.in_cols_box = s_in.cols_box;
     t.in_chunk8 = s_in.chunk8;
-    if (G == 2) {
+    if (G >= 2) {
         const Layer& Lc = net.layers[t.groups[0][1]];
         t.cut_h = Lc.h_out;
         t.cut_w = Lc.w_out;
@@ -510,11 +511,38 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             }
     }
 
+    // ---- outputs of groups 2 .. G-1 (group 1's is the cut tensor): whole maps of every
+    // frame after the ring or the layer maps, read by the next group's first stage through
+    // a tensor map of its own
+    std::vector<int64_t> bmap_off(G, -1), bmap_frame(G, 0);
+    for (int g = 1; g + 1 < G; ++g) {
+        const int s_last = t.stage_last[g];
+        const MafatStageDev& st = t.stages[s_last];
+        const Layer& Lo = net.layers[t.groups[g][1]];
+        bmap_frame[g] = (int64_t)ceil_div(st.cout, 8) * 8 * Lo.h_out * Lo.w_out;
+        bmap_off[g] = (t.scratch_elems + 127) / 128 * 128;
+        t.scratch_elems = bmap_off[g] + bmap_frame[g] * cfg.batch;
+        const int s_next = t.stage_first[g + 1];
+        const MafatStageDev& sn = t.stages[s_next];
+        TmapReq req{};
+        req.task = -1;
+        req.elem_off = bmap_off[g];
+        req.h = Lo.h_out;
+        req.w = Lo.w_out;
+        req.c8 = sn.cin8;
+        req.frames = cfg.batch;
+        req.rows_box = sn.rows_box;
+        req.cols_box = sn.cols_box;
+        req.chunk8 = sn.chunk8;
+        stage_tmap[s_next] = (int)t.tmaps.size();
+        t.tmaps.push_back(req);
+    }
+
     // ---- tasks in hand-out order, with their dependencies expressed as task indices
     struct TaskDep {
         int prev_task = -1;    // previous stage of the same tile, or the ring predecessor's last stage
-        int frame_g1 = -1;     // frame whose group 1 must be complete
-        bool last_g1 = false;  // last stage of group 1 (bumps the frame counter)
+        int group_ctr = -1;    // (frame, group) counter whose group must be complete (first stages)
+        int bump_ctr = -1;     // (frame, group) counter this last stage of a group bumps
     };
     std::vector<TaskDep> deps;
     std::vector<int> last_task_of_seq;
@@ -554,9 +582,9 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         tk.nbx = ceil_div(tk.cw, MAFAT_BLK_COLS);
                         int rel = s - t.stage_first[g];
                         if (s == t.stage_first[g]) {
-                            tk.in_kind = g == 0 ? MAFAT_BUF_USER_IN : MAFAT_BUF_CUT;
-                            tk.in_tmap = -1;
-                            tk.in_off = g == 0 ? f * in_frame : f * cut_frame;
+                            tk.in_kind = g == 0 ? MAFAT_BUF_USER_IN : g == 1 ? MAFAT_BUF_CUT : MAFAT_BUF_MAP;
+                            tk.in_tmap = g >= 2 ? stage_tmap[s] : -1;
+                            tk.in_off = g == 0 ? f * in_frame : g == 1 ? f * cut_frame : bmap_off[g - 1] + f * bmap_frame[g - 1];
                             tk.in_h = Lc.h_in;
                             tk.in_w = Lc.w_in;
                             tk.in_y0 = 0;
@@ -597,12 +625,18 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                                 tk.out_off = f * out_frame;
                                 tk.out_h = t.out_h;
                                 tk.out_w = t.out_w;
-                            } else {
+                            } else if (g == 0) {
                                 tk.out_kind = MAFAT_BUF_CUT;
                                 tk.out_nhwc = 0;
                                 tk.out_off = f * cut_frame;
                                 tk.out_h = t.cut_h;
                                 tk.out_w = t.cut_w;
+                            } else {
+                                tk.out_kind = MAFAT_BUF_MAP;
+                                tk.out_nhwc = 0;
+                                tk.out_off = bmap_off[g] + f * bmap_frame[g];
+                                tk.out_h = net.layers[t.groups[g][1]].h_out;
+                                tk.out_w = net.layers[t.groups[g][1]].w_out;
                             }
                             tk.out_y0 = 0;
                             tk.out_x0 = 0;
@@ -629,7 +663,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         int qi = (int)(q - w0);
                         if (s == t.stage_first[g]) {
                             if (!cfg.halo_reuse && tseq >= S) d.prev_task = last_task_of_seq[tseq - S];
-                            if (g == 1) d.frame_g1 = f;
+                            if (g >= 1) d.group_ctr = f * (G - 1) + (g - 1);
                         } else if (cfg.halo_reuse) {
                             // every previous-stage task whose owned output meets this task's input
                             // region (halo included): itself and the neighbours around it
@@ -649,7 +683,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         } else {
                             d.prev_task = prev_of_tile[qi];
                         }
-                        d.last_g1 = (G == 2 && g == 0 && s == t.stage_last[g]);
+                        if (g + 1 < G && s == t.stage_last[g]) d.bump_ctr = f * (G - 1) + g;
                         prev_of_tile[qi] = (int)t.tasks.size();
                         t.tasks.push_back(tk);
                         deps.push_back(d);
@@ -670,11 +704,11 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     // ---- counters: one per task, then one per frame (group-1 completion)
     const int n_tasks = (int)t.tasks.size();
     t.frame_ctr_base = MAFAT_CTR_BASE + n_tasks;
-    t.n_counters = n_tasks + cfg.batch;
-    std::vector<int> g1_items(cfg.batch, 0);
+    t.n_counters = n_tasks + cfg.batch * (G - 1);
+    std::vector<int> group_items((size_t)cfg.batch * std::max(G - 1, 1), 0);
     for (int ti = 0; ti < n_tasks; ++ti) {
         t.tasks[ti].done_ctr = MAFAT_CTR_BASE + ti;
-        if (deps[ti].last_g1) g1_items[t.tasks[ti].frame] += t.tasks[ti].n_items;
+        if (deps[ti].bump_ctr >= 0) group_items[deps[ti].bump_ctr] += t.tasks[ti].n_items;
     }
     // ---- items
     for (int ti = 0; ti < n_tasks; ++ti) {
@@ -704,11 +738,11 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         it.dep0 = MAFAT_CTR_BASE + d.prev_task;
                         it.dep0_target = t.tasks[d.prev_task].n_items;
                     }
-                    if (d.frame_g1 >= 0) {
-                        it.dep1 = t.frame_ctr_base + d.frame_g1;
-                        it.dep1_target = g1_items[d.frame_g1];
+                    if (d.group_ctr >= 0) {
+                        it.dep1 = t.frame_ctr_base + d.group_ctr;
+                        it.dep1_target = group_items[d.group_ctr];
                     }
-                    if (d.last_g1) it.extra_ctr = t.frame_ctr_base + tk.frame;
+                    if (d.bump_ctr >= 0) it.extra_ctr = t.frame_ctr_base + d.bump_ctr;
                     t.items.push_back(it);
                 }
     }
@@ -731,10 +765,18 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         if (L.type == L_CONV)
             t.useful_flops += 2.0 * L.h_out * L.w_out * (double)L.c_out * L.c_in * L.k * L.k * cfg.batch;
     }
-    int64_t io = in_frame + out_frame + (G == 2 ? 2 * cut_frame : 0);
+    int64_t io = in_frame + out_frame + (G >= 2 ? 2 * cut_frame : 0);
+    for (int g = 1; g + 1 < G; ++g) io += 2 * bmap_frame[g];
     t.group_io_elems = io * cfg.batch;
-    t.predicted_mib = predict_mem(net, G == 2 ? cfg.cut : 0, cfg.grid_n[0], cfg.grid_m[0],
-                                  G == 2 ? cfg.grid_n[1] : 1, G == 2 ? cfg.grid_m[1] : 1, 31.0);
+    if (G <= 2) {
+        t.predicted_mib = predict_mem(net, G == 2 ? cfg.cuts[0] : 0, cfg.grid_n[0], cfg.grid_m[0],
+                                      G == 2 ? cfg.grid_n[1] : 1, G == 2 ? cfg.grid_m[1] : 1, 31.0);
+    } else {  // predictMem's maximum over the groups, for any number of them
+        t.predicted_mib = 0.0;
+        for (int g = 0; g < G; ++g)
+            t.predicted_mib = std::max(t.predicted_mib, predict_layer_group(net, t.groups[g][0], t.groups[g][1],
+                                                                            cfg.grid_n[g], cfg.grid_m[g], 31.0, 2));
+    }
     return validate_plan(net, t);
 }
 
@@ -745,7 +787,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     const int64_t cut_total = (int64_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_total = (int64_t)t.cfg.batch * t.out_h * t.out_w * t.out_c;
     const int64_t scratch_total = t.scratch_elems;
-    if (!t.cfg.halo_reuse && scratch_total != (int64_t)t.ring_slots * 2 * t.slot_buf_elems) return "bad scratch size";
+    if (!t.cfg.halo_reuse && scratch_total < (int64_t)t.ring_slots * 2 * t.slot_buf_elems) return "scratch below the ring";
     auto buf_total = [&](int kind) {
         return kind == MAFAT_BUF_USER_IN ? in_total
                : kind == MAFAT_BUF_CUT   ? cut_total
@@ -795,7 +837,6 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (k.in_y0 + k.in_h > L.h_in || k.in_x0 + k.in_w > L.w_in || k.in_y0 < 0 || k.in_x0 < 0)
             return "input region outside the map";
         if (k.in_kind == MAFAT_BUF_SCRATCH && k.in_off % t.slot_buf_elems != 0) return "scratch input misaligned";
-        if ((k.in_kind == MAFAT_BUF_MAP) != (k.out_kind == MAFAT_BUF_MAP) && !t.cfg.halo_reuse) return "layer map without halo reuse";
         if (k.dep_count < 0 || k.dep_first < 0 || k.dep_first + k.dep_count > (int)t.deps.size()) return "bad dependency list";
         for (int d = k.dep_first; d < k.dep_first + k.dep_count; ++d) {
             const int dt = t.deps[d].ctr - MAFAT_CTR_BASE;
@@ -818,7 +859,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (k.done_ctr < MAFAT_CTR_BASE || k.done_ctr >= MAFAT_CTR_BASE + t.n_counters) return "bad done counter";
     }
     // dependencies: every counter an item waits on is fed only by items handed out before it
-    std::vector<int> frame_last(t.cfg.batch, -1);
+    std::vector<int> frame_last((size_t)t.cfg.batch * std::max(t.cfg.n_groups - 1, 1), -1);
     for (size_t i = 0; i < t.items.size(); ++i) {
         const MafatItemDev& it = t.items[i];
         const MafatTaskDev& k = t.tasks[it.task];

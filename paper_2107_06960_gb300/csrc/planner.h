@@ -8,6 +8,7 @@
 #include <string>
 #include <vector>
 
+#include "../../include/mafat.h"
 #include "device_types.h"
 
 namespace mafat {
@@ -78,8 +79,8 @@ void search(const Net& net, double limit_mib, double bias_mib, int* top, int* cu
 
 struct PlanConfig {
     int n_groups = 1;
-    int cut = 0;
-    int grid_n[2] = {1, 1}, grid_m[2] = {1, 1};
+    int cuts[MAFAT_MAX_GROUPS - 1] = {0, 0, 0};  // first layer of groups 2.. (increasing)
+    int grid_n[MAFAT_MAX_GROUPS] = {1, 1, 1, 1}, grid_m[MAFAT_MAX_GROUPS] = {1, 1, 1, 1};
     int batch = 1;
     int dtype = 0;            // 0 bf16, 1 fp32
     int ring_slots = 0;
@@ -92,7 +93,7 @@ struct PlanConfig {
                               // their neighbours' results in whole layer maps (no recompute)
     int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
     // explicit tile bounds per group (empty: even): rows[g] has grid_n[g] + 1 entries, cols[g] grid_m[g] + 1
-    std::vector<int> row_bounds[2], col_bounds[2];
+    std::vector<int> row_bounds[MAFAT_MAX_GROUPS], col_bounds[MAFAT_MAX_GROUPS];
 };
 
 // A tensor-map request for a task whose input is a scratch region buffer.
@@ -105,9 +106,9 @@ struct TmapReq {
 
 struct PlanTables {
     PlanConfig cfg;
-    int groups[2][2];         // [g] = {first, last} layer
-    std::vector<int> rows[2], cols[2];   // tile bounds of each group on its last layer's output
-    int stage_first[2], stage_last[2];   // stage index range per group
+    int groups[MAFAT_MAX_GROUPS][2];     // [g] = {first, last} layer
+    std::vector<int> rows[MAFAT_MAX_GROUPS], cols[MAFAT_MAX_GROUPS];  // tile bounds on each group's output
+    int stage_first[MAFAT_MAX_GROUPS], stage_last[MAFAT_MAX_GROUPS];  // stage index range per group
     std::vector<MafatStageDev> stages;
     std::vector<MafatTaskDev> tasks;
     std::vector<MafatItemDev> items;
@@ -120,9 +121,11 @@ struct PlanTables {
     std::vector<MafatDepDev> deps;       // task dependency lists (halo reuse)
     int ring_slots = 0, wave_tiles = 0;
     int n_counters = 0;                  // words after MAFAT_CTR_BASE
-    int frame_ctr_base = 0;              // per-frame group-1 completion counters
+    int frame_ctr_base = 0;              // completion counters of every group but the last, per frame:
+                                         // frame_ctr_base + frame * (n_groups - 1) + group
     int n_tiles = 0;
-    // input / cut / output geometry
+    // input / cut / output geometry (the cut tensor is group 1's output; the outputs of
+    // groups 2 .. n_groups - 1 are layer maps in the scratch allocation)
     int in_c8 = 0;
     int cut_h = 0, cut_w = 0, cut_c8 = 0;
     int out_h = 0, out_w = 0, out_c = 0;

@@ -169,7 +169,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
     kp.deps = p->d_deps;
     kp.n_items = (int32_t)p->t.items.size();
     kp.tmaps = p->d_tmaps;
-    kp.cut_tmap = p->t.cfg.n_groups == 2 ? (int)p->t.tmaps.size() : -1;
+    kp.cut_tmap = p->t.cfg.n_groups >= 2 ? (int)p->t.tmaps.size() : -1;
     kp.w_bf16 = (const uint16_t*)p->d_w;
     kp.w_f32 = (const float*)p->d_w;
     kp.scale = p->d_scale;
@@ -235,7 +235,7 @@ mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* 
     k.timeout_ns = p->timeout_ns;
     *kp = k;
     *ctr_bytes = p->ctr_bytes;
-    *cut_bytes = p->t.cfg.n_groups == 2 ? p->cut_bytes : 0;
+    *cut_bytes = p->t.cfg.n_groups >= 2 ? p->cut_bytes : 0;
     *scratch_bytes = (size_t)p->scratch_bytes;
     *grid = p->grid;
     *device = p->device;
@@ -303,8 +303,8 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
                            mafat_plan_t** out) {
     if (!net || !grid_n || !grid_m || !out) return fail(MAFAT_EINVAL, "null argument");
     *out = nullptr;
-    if (n_groups == 2 && !cuts) return fail(MAFAT_EINVAL, "two groups need a cut");
-    if (n_groups != 1 && n_groups != 2) return fail(MAFAT_EINVAL, "n_groups must be 1 or 2");
+    if (n_groups >= 2 && !cuts) return fail(MAFAT_EINVAL, "several groups need cuts");
+    if (n_groups < 1 || n_groups > MAFAT_MAX_GROUPS) return fail(MAFAT_EINVAL, "n_groups must be 1..4");
     if (dt != MAFAT_BF16 && dt != MAFAT_FP32) return fail(MAFAT_EINVAL, "unknown dtype");
     mafat_plan_options o{};
     if (opt) {
@@ -316,7 +316,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     }
     mafat::PlanConfig cfg;
     cfg.n_groups = n_groups;
-    cfg.cut = n_groups == 2 ? cuts[0] : 0;
+    for (int c = 0; c + 1 < n_groups; ++c) cfg.cuts[c] = cuts[c];
     for (int g = 0; g < n_groups; ++g) {
         cfg.grid_n[g] = grid_n[g];
         cfg.grid_m[g] = grid_m[g];
@@ -405,7 +405,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     if ((e = dalloc(p, &p->d_scale, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_bias, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_scratch, (size_t)p->scratch_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
-    if (t.cfg.n_groups == 2 && (e = dalloc(p, &p->d_cut, p->cut_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if (t.cfg.n_groups >= 2 && (e = dalloc(p, &p->d_cut, p->cut_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
 
     std::vector<float> w32, sc, bi;
     mafat::pack_weights_fp32(net->net, t, w32, sc, bi);
@@ -433,7 +433,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
 
     if (dt == MAFAT_BF16) {
         // one map per scratch-input task, then the cut tensor map
-        std::vector<CUtensorMap> maps(t.tmaps.size() + (t.cfg.n_groups == 2 ? 1 : 0));
+        std::vector<CUtensorMap> maps(t.tmaps.size() + (t.cfg.n_groups >= 2 ? 1 : 0));
         std::string merr;
         for (size_t i = 0; i < t.tmaps.size(); ++i) {
             const mafat::TmapReq& q = t.tmaps[i];
@@ -444,7 +444,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
                 return fail(MAFAT_ECUDA, merr);
             }
         }
-        if (t.cfg.n_groups == 2) {
+        if (t.cfg.n_groups >= 2) {
             if (!encode_planar_map(&maps.back(), p->d_cut, t.cut_w, t.cut_h, t.cut_c8, t.cfg.batch, t.cut_cols_box,
                                    t.cut_rows_box, t.cut_chunk8, &merr)) {
                 free_plan_memory(p);
@@ -482,7 +482,7 @@ mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* 
     std::lock_guard<std::mutex> lk(p->mu);
     mafat_status s = launch(p, input, output, (cudaStream_t)stream);
     if (s != MAFAT_OK) return s;
-    if (p->t.cfg.n_groups == 2 && cut_out) {
+    if (p->t.cfg.n_groups >= 2 && cut_out) {
         cudaError_t e = cudaMemcpyAsync(cut_out, p->d_cut, p->cut_bytes, cudaMemcpyDeviceToDevice, (cudaStream_t)stream);
         if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync");
     }

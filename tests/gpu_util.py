@@ -26,8 +26,8 @@ def run_plan(mf, layers, params, x, cut, grids, dtype, plan_kwargs=None, repeat=
     out = torch.full((B, sh[3], sh[4], sh[5]), float("nan"), dtype=tdt, device="cuda")
     cut_out = None
     cut_c = None
-    if cut is not None:
-        sc = net.shape(cut - 1)
+    if cut is not None:  # the cut tensor is group 1's output
+        sc = net.shape((cut[0] if isinstance(cut, (list, tuple)) else cut) - 1)
         cut_c = sc[5]
         cut_out = torch.full((B, (sc[5] + 7) // 8, sc[3], sc[4], 8), float("nan"), dtype=tdt, device="cuda")
     for _ in range(repeat):

@@ -286,6 +286,44 @@ def test_bf16_608_halo_reuse(mf, name):
                   TOL_BF16)
 
 
+@pytest.mark.parametrize("cuts,grids", [([4, 8], [(3, 3), (2, 2), (2, 1)]), ([2, 6, 12], [(2, 2), (3, 2), (2, 2), (1, 2)])])
+def test_bf16_yolo16_96_more_groups(mf, cuts, grids):
+    # three and four layer groups (the outputs of groups 2.. are layer maps on the device):
+    # the cut tensor and the output against the oracle, and bit-identical to a two-group
+    # plan with fixed MMA shapes
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 41, "bf16")
+    x = synth.make_input(2, 96, 96, 3, 42, "bf16")
+    c, out = run_plan(mf, layers, params, x, cuts, grids, mf.BF16)
+    refs = [oracle.group_outputs(layers, params, x[b], cuts) for b in range(2)]
+    for b in range(2):
+        assert rel_err(c[b], refs[b][0]) <= TOL_BF16 and rel_err(out[b], refs[b][-1]) <= TOL_BF16
+    fixed = dict(force_nblk=32, force_mb=1)
+    _, a = run_plan(mf, layers, params, x, cuts, grids, mf.BF16, plan_kwargs=fixed)
+    _, e = run_plan(mf, layers, params, x, 8, [(2, 2), (1, 1)], mf.BF16, plan_kwargs=fixed)
+    assert np.array_equal(a, e)
+
+
+def test_fp32_yolo16_96_four_groups(mf):
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 31, "fp32")
+    x = synth.make_input(2, 96, 96, 3, 32, "fp32")
+    cuts = [2, 6, 12]
+    c, out = run_plan(mf, layers, params, x, cuts, [(2, 2), (3, 2), (2, 2), (1, 2)], mf.FP32)
+    for b in range(2):
+        refs = oracle.group_outputs(layers, params, x[b], cuts)
+        assert rel_err(c[b], refs[0]) <= TOL_FP32 and rel_err(out[b], refs[-1]) <= TOL_FP32
+
+
+def test_bf16_608_three_groups(mf):
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    layers, params, x = wl["layers"], wl["params"], wl["input"]
+    cuts = [4, 8]
+    c, out = run_plan(mf, layers, params, x, cuts, [(5, 5), (3, 3), (2, 2)], mf.BF16)
+    outs = oracle.forward(layers, params, x[0])
+    assert rel_err(c[0], outs[3]) <= TOL_BF16 and rel_err(out[0], outs[-1]) <= TOL_BF16
+
+
 def test_measured_search_picks_the_fastest_timed_plan(mf):
     # Algorithm 2 re-targeted at the GPU: candidates whose intermediates fit the L2 are timed,
     # the others refused; the fastest is reported, and it computes the network correctly

@@ -203,6 +203,20 @@ def test_yolo16_uneven_tiling_is_bit_identical_to_unfused(cut, bounds):
         assert np.array_equal(a, b)
 
 
+@pytest.mark.parametrize("cuts,grids", [([4, 8], [(3, 3), (2, 2), (2, 1)]), ([2, 6, 12], [(2, 2), (3, 2), (2, 2), (1, 2)]),
+                                        ([8, 12], [(1, 1), (2, 2), (2, 2)])])
+def test_yolo16_more_groups_are_bit_identical_to_unfused(cuts, grids):
+    # more than two layer groups, each merged and re-tiled at its cut
+    layers = synth.YOLO16
+    x = synth.make_input(1, 64, 64, 3, 25, "fp32")[0]
+    params = _params(layers, 3, 26)
+    ref = oracle.group_outputs(layers, params, x, cuts)
+    got = oracle.forward_tiled(layers, params, x, cuts, grids)
+    assert len(got) == len(cuts) + 1
+    for a, b in zip(got, ref):
+        assert np.array_equal(a, b)
+
+
 def test_region_that_misses_halo_is_rejected():
     # A region one row short of the receptive field must be refused, not silently padded.
     layers = [_conv_layer(3, 2)]

@@ -268,3 +268,30 @@ def test_halo_reuse_plan_computes_each_pixel_once(mf, cut, grids):
                         assert (iy0, iy1) == (max(oy0 * s - p, 0), min((oy1 - 1) * s - p + k, shapes[l]["h_in"]))
                         assert (ix0, ix1) == (max(ox0 * s - p, 0), min((ox1 - 1) * s - p + k, shapes[l]["w_in"]))
             assert np.all(cover == 1), (g, l)
+
+
+@pytest.mark.parametrize("cuts,grids", [([4, 8], [(5, 5), (3, 3), (2, 2)]), ([2, 6, 12], [(4, 4), (3, 3), (2, 2), (1, 1)])])
+def test_plan_with_more_groups(mf, cuts, grids):
+    # three and four layer groups: regions, executed work and group I/O as the oracle's
+    layers = synth.YOLO16
+    net = _net(mf, layers, 608)
+    plan = mf.Plan(net, cuts, grids, dry_run=True)
+    st = plan.stats()
+    assert st["n_groups"] == len(cuts) + 1
+    assert st["executed_flops"] == _region_flops(layers, 608, cuts, grids, 1)
+    shapes = oracle.layer_shapes(layers, 608, 608, 3)
+    for gi, g in enumerate(oracle.groups_of(len(layers), cuts)):
+        n, m = grids[gi]
+        for i in range(n):
+            for j in range(m):
+                ref = oracle.tile_regions(layers, shapes, g, n, m, i, j)
+                for l in (g[0], g[1]):
+                    assert plan.tile_region(gi, i, j, l) == ref[l]
+    planar = lambda l: (shapes[l]["c_out"] + 7) // 8 * 8 * shapes[l]["h_out"] * shapes[l]["w_out"]
+    io = 8 * 608 * 608 + 19 * 19 * 0 + shapes[15]["h_out"] * shapes[15]["w_out"] * shapes[15]["c_out"]
+    io += sum(2 * planar(c - 1) for c in cuts)
+    assert st["group_io_bytes"] == io * 2
+    with pytest.raises(mf.MafatError):
+        mf.Plan(net, [8, 4], [(2, 2)] * 3, dry_run=True)      # cuts must increase
+    with pytest.raises(mf.MafatError):
+        mf.Plan(net, [2, 4, 8, 12], [(2, 2)] * 5, dry_run=True)  # at most four groups
