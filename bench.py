@@ -279,6 +279,9 @@ def main():
     ap.add_argument("--impl", default="mafat", choices=["mafat", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--frames-in-flight", type=int, default=16,
+                    help="frames of the steady-state leg (one launch of a plan of this many frames, "
+                         "frame f's second group overlapped with frame f+1's first); 0: skip it")
     ap.add_argument("--sweep", action="store_true",
                     help="time every plan of the 608x608 net over cuts {none, 2, 4, 8, 12} x grids 1..5 per "
                          "group (one JSON line per plan, then the fastest), instead of the benchmark line")
@@ -347,6 +350,40 @@ def main():
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     dev_s = sum(step_ms) / 1e3
 
+    # Steady state with frames in flight: one launch of a K-frame plan, whose hand-out order
+    # overlaps frame f's second group (a chain of small-map stages that leaves SMs idle)
+    # with frame f + 1's first.  Each frame is still a 608x608 batch-1 image; the L2 is
+    # flushed before every launch as in the device leg.
+    ss = None
+    K = args.frames_in_flight
+    if K > 1 and B == 1 and wl["cut"] is not None:
+        plan_k = mf.Plan(net, wl["cut"], wl["grids"], batch=K, dtype=dt)
+        st_k = plan_k.stats()
+        xk = torch.from_numpy(mf.to_planar(synth.make_input(K, H, W, 3, synth.SEED_BASE + 77, wl["dtype"])))
+        xk = xk.to(tdt).to(dev)
+        outk = torch.empty((K, sh[3], sh[4], sh[5]), dtype=tdt, device=dev)
+        for _ in range(args.warmup):
+            plan_k.run(xk, outk, stream=stream)
+        plan_k.sync_status(stream=stream)
+        ss_steps = max(3, min(args.steps // 20, 100))
+        s_ev = [torch.cuda.Event(enable_timing=True) for _ in range(ss_steps)]
+        e_ev = [torch.cuda.Event(enable_timing=True) for _ in range(ss_steps)]
+        if pg:
+            pg.barrier()
+        torch.cuda.synchronize()
+        for i in range(ss_steps):
+            flush.fill_(i)
+            s_ev[i].record(stream)
+            plan_k.run(xk, outk, stream=stream)
+            e_ev[i].record(stream)
+        torch.cuda.synchronize()
+        plan_k.sync_status(stream=stream)
+        ss_ms = [a.elapsed_time(b) for a, b in zip(s_ev, e_ev)]
+        ss = {"frames_in_flight": K, "launches": ss_steps, "seconds": sum(ss_ms) / 1e3,
+              "overlapped": bool(st_k["frames_overlapped"]), "items": st_k["n_items"]}
+        plan_k.close()
+        del xk, outk
+
     # End to end through the C ABI on pinned host buffers, every step's upload of its
     # input and read-back of its output inside the timed region.  Streamed the way a
     # serving loop would (mafat_run_host_async: the upload of one frame overlaps the run
@@ -371,7 +408,8 @@ def main():
         plan.run_host(xh, oh, stream=stream)
     sync_s = time.perf_counter() - t0
 
-    dev_s_max, e2e_s_max, sync_s_max = reduce_max(pg, [dev_s, e2e_s, sync_s], dev)
+    dev_s_max, e2e_s_max, sync_s_max, ss_s_max = reduce_max(
+        pg, [dev_s, e2e_s, sync_s, ss["seconds"] if ss else 0.0], dev)
     if rank != 0:
         if pg:
             pg.destroy_process_group()
@@ -429,6 +467,17 @@ def main():
         "gpu_launches": args.steps * plan.launches_per_run(),
         "clocks": clk,
     }
+    if ss is not None:
+        ss_value = aggregate([ss["frames_in_flight"] * ss["launches"]] * ws, [ss_s_max])
+        ss_tf = st["useful_flops"] / B * ss_value / ws / 1e12
+        line["steady_state"] = {
+            "value": ss_value, "unit": "frames/s", "frames_in_flight": ss["frames_in_flight"],
+            "ms_per_frame": 1e3 * ss_s_max / (ss["frames_in_flight"] * ss["launches"]),
+            "launches": ss["launches"], "gpu_launches": ss["launches"] * plan.launches_per_run(),
+            "work_items_per_launch": ss["items"], "frames_overlapped": ss["overlapped"],
+            "roofline_frac": ss_tf / peak_burst, "achieved_tflops": ss_tf,
+            "mode": "one launch of a %d-frame plan per step (frame f's second group overlapped with frame "
+                    "f+1's first), L2 flushed before every launch" % ss["frames_in_flight"]}
     if cpu is not None:
         line["cpu_baseline"] = cpu
     print(json.dumps(line), flush=True)

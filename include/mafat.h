@@ -105,7 +105,9 @@ typedef struct {
                                    and reads the halo its next layer needs from its neighbours' parts
                                    (each layer waits for those neighbours); 0: the fused tiles of
                                    Sec. 3-4, every tile recomputing its halo */
-    int32_t reserved;
+    int32_t frame_major;        /* batch > 1 with two groups: 1 hands the frames out strictly one after
+                                   another; 0 (default) overlaps frame f's second group with frame
+                                   f + 1's first (the second group's small maps leave SMs idle) */
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */
@@ -128,6 +130,9 @@ typedef struct {
     int32_t wave_tiles;
     int32_t max_ctas;
     int32_t dtype;
+    int32_t frames_overlapped;  /* 1: the hand-out order overlaps frame f's second group with frame
+                                   f + 1's first (batch > 1, two groups, ring of a whole frame) */
+    int32_t reserved;
 } mafat_plan_stats;
 
 /* Build a network description: validates the layers and infers every layer's

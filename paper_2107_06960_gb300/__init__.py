@@ -35,7 +35,7 @@ class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
                 ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32),
-                ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("reserved", i32)]
+                ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("frame_major", i32)]
 
 
 class PlanStats(ctypes.Structure):
@@ -43,7 +43,8 @@ class PlanStats(ctypes.Structure):
                 ("n_items", i64), ("useful_flops", dbl), ("executed_flops", dbl), ("issued_flops", dbl),
                 ("predicted_mib", dbl), ("group_io_bytes", i64), ("weight_bytes", i64),
                 ("scratch_bytes", i64), ("workspace_bytes", i64), ("smem_bytes_per_cta", i64),
-                ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32), ("dtype", i32)]
+                ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32), ("dtype", i32),
+                ("frames_overlapped", i32), ("reserved", i32)]
 
 
 class SearchOptions(ctypes.Structure):
@@ -249,7 +250,8 @@ class Plan:
 
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
-                 force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False):
+                 force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False,
+                 frame_major=False):
         self.net = net
         # cut: None (one group), the first layer of group 2, or a list of increasing cuts
         cut_list = [] if cut is None else (list(cut) if isinstance(cut, (list, tuple)) else [cut])
@@ -269,6 +271,7 @@ class Plan:
         opt.force_nblk, opt.force_mb = force_nblk, force_mb
         opt.lookahead_items = lookahead_items
         opt.halo_reuse = int(halo_reuse)
+        opt.frame_major = int(frame_major)
         if tile_bounds is not None:
             # per group (rows, cols): the non-uniform tiling; kept alive with the plan
             flat = [v for rows, cols in list(tile_bounds)[:n_groups] for v in list(rows) + list(cols)]
@@ -323,7 +326,7 @@ class Plan:
         s = PlanStats()
         s.struct_size = ctypes.sizeof(PlanStats)
         _check(lib.mafat_plan_stats_get(self.handle, ctypes.byref(s)))
-        return {k: getattr(s, k) for k, _ in PlanStats._fields_ if k != "struct_size"}
+        return {k: getattr(s, k) for k, _ in PlanStats._fields_ if k not in ("struct_size", "reserved")}
 
     def trace(self, stream=None):
         """Per-item records of the last run (plan made with trace=True): numpy uint64

@@ -329,13 +329,14 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 *unsupported = true;
                 return "layer " + std::to_string(l) + ": input channels above 8 must be a multiple of 16";
             }
-            // M blocks of this stage over all tiles and frames
+            // M blocks of this stage over the tiles of one frame: frames go through a stage one
+            // after another (or overlapped with another group), never all side by side, so
+            // a stage's parallelism is one frame's
             int64_t blocks = 0;
             for (const TileInfo& ti : tiles[g]) {
                 const Rect& cr = ti.outs[l];
                 blocks += (int64_t)ceil_div(cr.h(), MAFAT_BLK_ROWS) * ceil_div(cr.w(), MAFAT_BLK_COLS);
             }
-            blocks *= cfg.batch;
             // Output-channel block (MMA N, a multiple of 16 dividing the padded cout; zero
             // weights pad it, only cout channels are stored): the narrowest block of at least
             // 64 channels whose items fit one wave of CTAs, else the widest.  A stage with few
@@ -454,7 +455,13 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     const int64_t cut_frame = (int64_t)t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_frame = (int64_t)t.out_h * t.out_w * t.out_c;
 
-    int S = cfg.ring_slots > 0 ? cfg.ring_slots : std::min(max_tiles, 64);
+    // The ring holds one frame's tiles of every group when several frames go through it, so
+    // that a tile's slot predecessor is the same tile of the previous frame (the frames'
+    // groups may then overlap in the hand-out order below)
+    int tiles_per_frame = 0;
+    for (int g = 0; g < G; ++g) tiles_per_frame += (int)tiles[g].size();
+    int S = cfg.ring_slots > 0 ? cfg.ring_slots
+                               : std::min(cfg.batch > 1 ? std::max(max_tiles, tiles_per_frame) : max_tiles, 64);
     int W = cfg.wave_tiles > 0 ? std::min(cfg.wave_tiles, S) : S;
     if (cfg.halo_reuse) {
         // a layer's tasks read their neighbours' previous layer, so every tile of a group
@@ -701,6 +708,78 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     }
     t.n_tiles = seq;
 
+    // ---- frames in flight (batch > 1, two groups): the second group of a frame is a chain of
+    // stages over a few small tiles that leaves most SMs idle, so the next frame's first-group
+    // tasks are handed out between its stages, split in proportion to their items.  Every
+    // dependency still points to an earlier task: a first-group task depends on its own frame's
+    // earlier tasks and on the same tile of the previous frame (its ring slot); a second-group
+    // task on its own frame's first group, all of which was handed out before.
+    if (cfg.batch > 1 && G == 2 && !cfg.halo_reuse && !cfg.frame_major && S >= tiles_per_frame && W >= max_tiles) {
+        const int n_t = (int)t.tasks.size();
+        std::vector<std::vector<int>> fill(cfg.batch), chain(cfg.batch);
+        for (int i = 0; i < n_t; ++i)
+            (t.tasks[i].stage <= t.stage_last[0] ? fill : chain)[t.tasks[i].frame].push_back(i);
+        std::vector<int> order;
+        order.reserve(n_t);
+        order.insert(order.end(), fill[0].begin(), fill[0].end());
+        for (int f = 0; f < cfg.batch; ++f) {
+            const std::vector<int>& cf = chain[f];
+            std::vector<size_t> cuts_at;  // starts of the runs of one stage
+            for (size_t i = 0; i < cf.size(); ++i)
+                if (i == 0 || t.tasks[cf[i]].stage != t.tasks[cf[i - 1]].stage) cuts_at.push_back(i);
+            cuts_at.push_back(cf.size());
+            static const std::vector<int> none;
+            const std::vector<int>& nx = f + 1 < cfg.batch ? fill[f + 1] : none;
+            int64_t nx_items = 0;
+            for (int i : nx) nx_items += t.tasks[i].n_items;
+            // Share of the next frame's first group handed out behind each second-group stage:
+            // in proportion to the stage's estimated duration, in units of one 128x128x16 MMA
+            // (a fixed part for the halo load, epilogue and completion round trip, plus the
+            // MMAs of one item), and a share ahead of the first stage, whose CTAs would
+            // otherwise wait for the whole first group of their own frame (measured on the
+            // 608x608 network, 16 frames: 83 us per frame against 88 with an even split).
+            const size_t n_runs = cuts_at.size() - 1;
+            const double kFixedMma = 72.0, kAheadMma = 288.0;
+            std::vector<double> share(n_runs + 1, 0.0);
+            share[0] = kAheadMma;
+            double total = kAheadMma;
+            for (size_t r = 0; r < n_runs; ++r) {
+                const MafatStageDev& st = t.stages[t.tasks[cf[cuts_at[r]]].stage];
+                share[r + 1] = kFixedMma + (double)st.n_blk / 128.0 * st.n_chunks * st.n_bsteps * st.kst * st.mb;
+                total += share[r + 1];
+            }
+            size_t pos = 0;
+            int64_t taken = 0;
+            double acc = 0.0;
+            for (size_t r = 0; r <= n_runs; ++r) {
+                if (r > 0)
+                    for (size_t i = cuts_at[r - 1]; i < cuts_at[r]; ++i) order.push_back(cf[i]);
+                acc += share[r];
+                const int64_t target = (int64_t)((double)nx_items * acc / total + 0.5);
+                while (pos < nx.size() && taken < target) {
+                    taken += t.tasks[nx[pos]].n_items;
+                    order.push_back(nx[pos++]);
+                }
+            }
+            while (pos < nx.size()) order.push_back(nx[pos++]);
+        }
+        if ((int)order.size() != n_t) return "internal: frame interleave lost a task";
+        std::vector<int> new_of(n_t);
+        for (int k = 0; k < n_t; ++k) new_of[order[k]] = k;
+        std::vector<MafatTaskDev> tasks2(n_t);
+        std::vector<TaskDep> deps2(n_t);
+        for (int k = 0; k < n_t; ++k) {
+            tasks2[k] = t.tasks[order[k]];
+            deps2[k] = deps[order[k]];
+            if (deps2[k].prev_task >= 0) deps2[k].prev_task = new_of[deps2[k].prev_task];
+        }
+        t.tasks.swap(tasks2);
+        deps.swap(deps2);
+        for (TmapReq& r : t.tmaps)
+            if (r.task >= 0) r.task = new_of[r.task];
+        t.frames_overlapped = 1;
+    }
+
     // ---- counters: one per task, then one per frame (group-1 completion)
     const int n_tasks = (int)t.tasks.size();
     t.frame_ctr_base = MAFAT_CTR_BASE + n_tasks;
@@ -747,14 +826,15 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 }
     }
     if (t.items.size() > (size_t)0x7fffffff) return "too many work items";
-    // Stages with many items (all tiles and frames) keep every CTA busy whatever it holds,
+    // Stages with many items (all tiles of one frame) keep every CTA busy whatever it holds,
     // so their CTAs take the next ticket early; stages with about a wave of items or fewer
     // take it only when the CTA can start it, so that no idle CTA waits for a busy one.
     {
         const int n_ctas = cfg.n_ctas > 0 ? cfg.n_ctas : 152;
         const int64_t thr = cfg.lookahead_items > 0 ? cfg.lookahead_items : (int64_t)n_ctas * 5 / 4;
         std::vector<int64_t> stage_items(t.stages.size(), 0);
-        for (const MafatTaskDev& tk : t.tasks) stage_items[tk.stage] += tk.n_items;
+        for (const MafatTaskDev& tk : t.tasks)
+            if (tk.frame == 0) stage_items[tk.stage] += tk.n_items;
         for (size_t s = 0; s < t.stages.size(); ++s)
             t.stages[s].lookahead = (cfg.lookahead_items >= 0 && stage_items[s] >= thr) ? 1 : 0;
     }

@@ -92,6 +92,7 @@ struct PlanConfig {
     bool halo_reuse = false;  // tiles compute only their own part of every layer and read the halo from
                               // their neighbours' results in whole layer maps (no recompute)
     int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
+    bool frame_major = false; // batch > 1: hand frames out one after another, never overlapped
     // explicit tile bounds per group (empty: even): rows[g] has grid_n[g] + 1 entries, cols[g] grid_m[g] + 1
     std::vector<int> row_bounds[MAFAT_MAX_GROUPS], col_bounds[MAFAT_MAX_GROUPS];
 };
@@ -106,6 +107,7 @@ struct TmapReq {
 
 struct PlanTables {
     PlanConfig cfg;
+    int frames_overlapped = 0;           // 1: frame f's second group overlaps frame f + 1's first in the order
     int groups[MAFAT_MAX_GROUPS][2];     // [g] = {first, last} layer
     std::vector<int> rows[MAFAT_MAX_GROUPS], cols[MAFAT_MAX_GROUPS];  // tile bounds on each group's output
     int stage_first[MAFAT_MAX_GROUPS], stage_last[MAFAT_MAX_GROUPS];  // stage index range per group

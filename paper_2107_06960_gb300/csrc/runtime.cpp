@@ -330,6 +330,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.fixed_mb = o.force_mb;
     cfg.lookahead_items = o.lookahead_items;
     cfg.halo_reuse = o.halo_reuse != 0;
+    cfg.frame_major = o.frame_major != 0;
     if (o.tile_bounds) {
         // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
         const int32_t* b = o.tile_bounds;
@@ -706,6 +707,7 @@ mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* ou
     s.wave_tiles = t.wave_tiles;
     s.max_ctas = plan->grid;
     s.dtype = plan->dtype;
+    s.frames_overlapped = t.frames_overlapped;
     *out = s;
     return MAFAT_OK;
 }

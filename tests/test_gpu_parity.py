@@ -188,6 +188,24 @@ def test_fp32_yolov2_trunk_96(mf):
     _check_groups(c, out, _oracle_groups(layers, params, x, 8), 8, TOL_FP32)
 
 
+def test_bf16_608_frames_in_flight(mf):
+    # three 608x608 frames in one launch, frame f's second group overlapped with frame
+    # f + 1's first in the hand-out order: every frame is bit-identical to the same frame
+    # run alone and to the frame-major order (same items, only their order differs), and
+    # the first frame matches the oracle
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    layers, params, cut, grids = wl["layers"], wl["params"], wl["cut"], wl["grids"]
+    x = np.concatenate([wl["input"], synth.make_input(2, 608, 608, 3, synth.SEED_BASE + 90, "bf16")], 0)
+    c3, o3 = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
+    cm, om = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs={"frame_major": True})
+    assert np.array_equal(o3, om) and np.array_equal(c3, cm)
+    for f in range(3):
+        c1, o1 = run_plan(mf, layers, params, x[f:f + 1], cut, grids, mf.BF16)
+        assert np.array_equal(o3[f], o1[0]) and np.array_equal(c3[f], c1[0]), "frame %d" % f
+    refs = _oracle_groups(layers, params, wl["input"], cut, "yolo16_608_5x5_c8_2x2")
+    _check_groups(c3[:1], o3[:1], refs, cut, TOL_BF16)
+
+
 def test_bf16_1216_batch8_stress(mf):
     wl = synth.workload("yolo16_1216_b8_8x8_c8_4x4")
     c, out = run_plan(mf, wl["layers"], wl["params"], wl["input"], wl["cut"], wl["grids"], mf.BF16)

@@ -295,3 +295,29 @@ def test_plan_with_more_groups(mf, cuts, grids):
         mf.Plan(net, [8, 4], [(2, 2)] * 3, dry_run=True)      # cuts must increase
     with pytest.raises(mf.MafatError):
         mf.Plan(net, [2, 4, 8, 12], [(2, 2)] * 5, dry_run=True)  # at most four groups
+
+
+def test_frames_in_flight_plan(mf):
+    # batch > 1 with two groups: the ring spans one frame's 25 + 4 tiles and the hand-out
+    # order overlaps frame f's second group with frame f + 1's first (the planner's own
+    # check then guarantees every dependency points to an earlier item); the work per
+    # frame is the same as at batch 1, and the overlap is only taken where it is safe
+    wl = synth.WORKLOADS["yolo16_608_5x5_c8_2x2"]
+    net = _net(mf, wl["layers"], 608)
+    one = mf.Plan(net, 8, wl["grids"], dry_run=True).stats()
+    assert one["frames_overlapped"] == 0
+    for k in (2, 3, 5):
+        st = mf.Plan(net, 8, wl["grids"], batch=k, dry_run=True).stats()
+        assert st["frames_overlapped"] == 1 and st["ring_slots"] == 29
+        assert st["n_items"] == k * one["n_items"] and st["n_tasks"] == k * one["n_tasks"]
+        assert abs(st["executed_flops"] - k * one["executed_flops"]) < 1e-3 * st["executed_flops"]
+        fm = mf.Plan(net, 8, wl["grids"], batch=k, dry_run=True, frame_major=True).stats()
+        assert fm["frames_overlapped"] == 0 and fm["n_items"] == st["n_items"]
+    # not taken: one group, halo reuse, or a ring too small for a whole frame
+    assert mf.Plan(net, None, [(3, 3)], batch=2, dry_run=True).stats()["frames_overlapped"] == 0
+    assert mf.Plan(net, 8, wl["grids"], batch=2, dry_run=True, halo_reuse=True).stats()["frames_overlapped"] == 0
+    assert mf.Plan(net, 8, wl["grids"], batch=2, dry_run=True, ring_slots=25).stats()["frames_overlapped"] == 0
+    big = synth.WORKLOADS["yolo16_1216_b8_8x8_c8_4x4"]
+    net2 = _net(mf, big["layers"], 1216)
+    st = mf.Plan(net2, 8, big["grids"], batch=2, dry_run=True).stats()
+    assert st["frames_overlapped"] == 0 and st["ring_slots"] == 64  # 80 tiles per frame
