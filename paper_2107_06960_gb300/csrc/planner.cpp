@@ -461,7 +461,8 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     int tiles_per_frame = 0;
     for (int g = 0; g < G; ++g) tiles_per_frame += (int)tiles[g].size();
     int S = cfg.ring_slots > 0 ? cfg.ring_slots
-                               : std::min(cfg.batch > 1 ? std::max(max_tiles, tiles_per_frame) : max_tiles, 64);
+            : cfg.batch > 1    ? std::min(std::max(max_tiles, tiles_per_frame), 256)
+                               : std::min(max_tiles, 64);
     int W = cfg.wave_tiles > 0 ? std::min(cfg.wave_tiles, S) : S;
     if (cfg.halo_reuse) {
         // a layer's tasks read their neighbours' previous layer, so every tile of a group

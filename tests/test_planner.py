@@ -320,4 +320,5 @@ def test_frames_in_flight_plan(mf):
     big = synth.WORKLOADS["yolo16_1216_b8_8x8_c8_4x4"]
     net2 = _net(mf, big["layers"], 1216)
     st = mf.Plan(net2, 8, big["grids"], batch=2, dry_run=True).stats()
-    assert st["frames_overlapped"] == 0 and st["ring_slots"] == 64  # 80 tiles per frame
+    assert st["frames_overlapped"] == 1 and st["ring_slots"] == 80  # 64 + 16 tiles per frame
+    assert mf.Plan(net2, 8, big["grids"], dry_run=True).stats()["ring_slots"] == 64  # one frame: 64 tiles
