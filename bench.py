@@ -422,12 +422,18 @@ def main():
     avg_launch_s = dev_s / args.steps
     achieved_tf = st["useful_flops"] / avg_launch_s / 1e12
     traffic = None
+    ss_traffic = None
     try:
         with open(TRAFFIC_FILE) as fh:
             tr = json.load(fh)
+        h = kernel_source_hash()
         ent = tr.get(args.workload)
-        if ent and ent.get("kernel_source_hash") == kernel_source_hash():
+        if ent and ent.get("kernel_source_hash") == h:
             traffic = ent["dram_bytes_per_launch"]
+        if ss is not None:
+            ent = tr.get("%s@%d" % (args.workload, ss["frames_in_flight"]))
+            if ent and ent.get("kernel_source_hash") == h:
+                ss_traffic = ent["dram_bytes_per_launch"] / ss["frames_in_flight"]
     except Exception:
         pass
 
@@ -475,7 +481,7 @@ def main():
             "ms_per_frame": 1e3 * ss_s_max / (ss["frames_in_flight"] * ss["launches"]),
             "launches": ss["launches"], "gpu_launches": ss["launches"] * plan.launches_per_run(),
             "work_items_per_launch": ss["items"], "frames_overlapped": ss["overlapped"],
-            "roofline_frac": ss_tf / peak_burst, "achieved_tflops": ss_tf,
+            "roofline_frac": ss_tf / peak_burst, "achieved_tflops": ss_tf, "dram_bytes_per_frame": ss_traffic,
             "mode": "one launch of a %d-frame plan per step (frame f's second group overlapped with frame "
                     "f+1's first), L2 flushed before every launch" % ss["frames_in_flight"]}
     if cpu is not None:
