@@ -345,11 +345,16 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // dominates.  Stages with more blocks than CTAs keep the widest block, which
             // reuses every A operand for the most output channels.
             const int cout_pad = (L.c_out + 15) / 16 * 16;
+            // With several frames in flight the SMs are kept busy by the next frame anyway, and a
+            // 1x1 layer's item reads a whole K = c_in halo for few MMAs: there the narrowest block
+            // considered is 128 (608x608, 16 frames: 81.3 against 83.0 us per frame; at one frame
+            // the extra parallelism of N = 64 wins, 117.4 against 121.5 us).
+            const int min_nb = (cfg.batch > 1 && L.k == 1) ? 128 : 64;
             if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
                 s.n_blk = cfg.fixed_nblk;
             } else {
                 s.n_blk = largest_nblk(cout_pad);
-                for (int nb = std::min(64, cout_pad); nb <= std::min(cout_pad, MAFAT_MAX_NBLK); nb += 16) {
+                for (int nb = std::min(min_nb, cout_pad); nb <= std::min(cout_pad, MAFAT_MAX_NBLK); nb += 16) {
                     if (cout_pad % nb != 0) continue;
                     if (blocks * (cout_pad / nb) <= n_ctas) {
                         s.n_blk = nb;

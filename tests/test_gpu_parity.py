@@ -190,9 +190,10 @@ def test_fp32_yolov2_trunk_96(mf):
 
 def test_bf16_608_frames_in_flight(mf):
     # three 608x608 frames in one launch, frame f's second group overlapped with frame
-    # f + 1's first in the hand-out order: every frame is bit-identical to the same frame
-    # run alone and to the frame-major order (same items, only their order differs), and
-    # the first frame matches the oracle
+    # f + 1's first in the hand-out order: bit-identical to the frame-major order (same
+    # items, only their order differs), every frame within the bf16 tolerance of the same
+    # frame run alone (1x1 layers use other channel blocks there), the first frame
+    # against the oracle
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     layers, params, cut, grids = wl["layers"], wl["params"], wl["cut"], wl["grids"]
     x = np.concatenate([wl["input"], synth.make_input(2, 608, 608, 3, synth.SEED_BASE + 90, "bf16")], 0)
@@ -201,7 +202,8 @@ def test_bf16_608_frames_in_flight(mf):
     assert np.array_equal(o3, om) and np.array_equal(c3, cm)
     for f in range(3):
         c1, o1 = run_plan(mf, layers, params, x[f:f + 1], cut, grids, mf.BF16)
-        assert np.array_equal(o3[f], o1[0]) and np.array_equal(c3[f], c1[0]), "frame %d" % f
+        assert rel_err(o3[f], o1[0]) <= TOL_BF16 and rel_err(c3[f], c1[0]) <= TOL_BF16, "frame %d" % f
+        assert np.array_equal(c3[f], c1[0]), "frame %d: the first group has the same items" % f
     refs = _oracle_groups(layers, params, wl["input"], cut, "yolo16_608_5x5_c8_2x2")
     _check_groups(c3[:1], o3[:1], refs, cut, TOL_BF16)
 

@@ -300,8 +300,9 @@ def test_plan_with_more_groups(mf, cuts, grids):
 def test_frames_in_flight_plan(mf):
     # batch > 1 with two groups: the ring spans one frame's 25 + 4 tiles and the hand-out
     # order overlaps frame f's second group with frame f + 1's first (the planner's own
-    # check then guarantees every dependency points to an earlier item); the work per
-    # frame is the same as at batch 1, and the overlap is only taken where it is safe
+    # check then guarantees every dependency points to an earlier item); the tasks and
+    # the work per frame are those of batch 1 (1x1 layers take wider output-channel
+    # blocks, hence fewer items), and the overlap is only taken where it is safe
     wl = synth.WORKLOADS["yolo16_608_5x5_c8_2x2"]
     net = _net(mf, wl["layers"], 608)
     one = mf.Plan(net, 8, wl["grids"], dry_run=True).stats()
@@ -309,7 +310,7 @@ def test_frames_in_flight_plan(mf):
     for k in (2, 3, 5):
         st = mf.Plan(net, 8, wl["grids"], batch=k, dry_run=True).stats()
         assert st["frames_overlapped"] == 1 and st["ring_slots"] == 29
-        assert st["n_items"] == k * one["n_items"] and st["n_tasks"] == k * one["n_tasks"]
+        assert st["n_tasks"] == k * one["n_tasks"] and st["n_items"] < k * one["n_items"]
         assert abs(st["executed_flops"] - k * one["executed_flops"]) < 1e-3 * st["executed_flops"]
         fm = mf.Plan(net, 8, wl["grids"], batch=k, dry_run=True, frame_major=True).stats()
         assert fm["frames_overlapped"] == 0 and fm["n_items"] == st["n_items"]
