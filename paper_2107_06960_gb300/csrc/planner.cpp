@@ -835,9 +835,13 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     // Stages with many items (all tiles of one frame) keep every CTA busy whatever it holds,
     // so their CTAs take the next ticket early; stages with about a wave of items or fewer
     // take it only when the CTA can start it, so that no idle CTA waits for a busy one.
+    // With frames overlapped the next frame keeps every CTA busy in any stage (608x608, 16
+    // frames: 80.4 against 80.9 us per frame).
     {
         const int n_ctas = cfg.n_ctas > 0 ? cfg.n_ctas : 152;
-        const int64_t thr = cfg.lookahead_items > 0 ? cfg.lookahead_items : (int64_t)n_ctas * 5 / 4;
+        const int64_t thr = cfg.lookahead_items > 0 ? cfg.lookahead_items
+                            : t.frames_overlapped  ? 1
+                                                   : (int64_t)n_ctas * 5 / 4;
         std::vector<int64_t> stage_items(t.stages.size(), 0);
         for (const MafatTaskDev& tk : t.tasks)
             if (tk.frame == 0) stage_items[tk.stage] += tk.n_items;
