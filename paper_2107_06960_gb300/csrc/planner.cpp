@@ -716,7 +716,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
 
     // ---- frames in flight (batch > 1, two groups): the second group of a frame is a chain of
     // stages over a few small tiles that leaves most SMs idle, so the next frame's first-group
-    // tasks are handed out between its stages, split in proportion to their items.  Every
+    // tasks are handed out between its stages (shares below).  Every
     // dependency still points to an earlier task: a first-group task depends on its own frame's
     // earlier tasks and on the same tile of the previous frame (its ring slot); a second-group
     // task on its own frame's first group, all of which was handed out before.
