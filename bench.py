@@ -379,10 +379,19 @@ def main():
         torch.cuda.synchronize()
         plan_k.sync_status(stream=stream)
         ss_ms = [a.elapsed_time(b) for a, b in zip(s_ev, e_ev)]
+        # self-check outside the timed region: the first and last frames of the K-frame
+        # launch against the same frames run one at a time through the 1-frame plan
+        one = torch.empty_like(out)
+        ss_err = 0.0
+        for f in (0, K - 1):
+            plan.run(xk[f:f + 1], one, stream=stream)
+            plan.sync_status(stream=stream)
+            ref = one.float()
+            ss_err = max(ss_err, float((outk[f:f + 1].float() - ref).abs().max()) / max(float(ref.abs().max()), 1e-30))
         ss = {"frames_in_flight": K, "launches": ss_steps, "seconds": sum(ss_ms) / 1e3,
-              "overlapped": bool(st_k["frames_overlapped"]), "items": st_k["n_items"]}
+              "overlapped": bool(st_k["frames_overlapped"]), "items": st_k["n_items"], "check": ss_err}
         plan_k.close()
-        del xk, outk
+        del xk, outk, one
 
     # End to end through the C ABI on pinned host buffers, every step's upload of its
     # input and read-back of its output inside the timed region.  Streamed the way a
@@ -481,6 +490,8 @@ def main():
             "ms_per_frame": 1e3 * ss_s_max / (ss["frames_in_flight"] * ss["launches"]),
             "launches": ss["launches"], "gpu_launches": ss["launches"] * plan.launches_per_run(),
             "work_items_per_launch": ss["items"], "frames_overlapped": ss["overlapped"],
+            "check_vs_one_frame": {"max_rel_err": ss["check"], "frames": [0, ss["frames_in_flight"] - 1],
+                                   "tolerance": 2e-2},
             "roofline_frac": ss_tf / peak_burst, "achieved_tflops": ss_tf, "dram_bytes_per_frame": ss_traffic,
             "mode": "one launch of a %d-frame plan per step (frame f's second group overlapped with frame "
                     "f+1's first), L2 flushed before every launch" % ss["frames_in_flight"]}
