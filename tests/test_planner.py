@@ -323,3 +323,16 @@ def test_frames_in_flight_plan(mf):
     st = mf.Plan(net2, 8, big["grids"], batch=2, dry_run=True).stats()
     assert st["frames_overlapped"] == 1 and st["ring_slots"] == 80  # 64 + 16 tiles per frame
     assert mf.Plan(net2, 8, big["grids"], dry_run=True).stats()["ring_slots"] == 64  # one frame: 64 tiles
+
+
+@pytest.mark.parametrize("cut", [2, 4, 8, 12])
+@pytest.mark.parametrize("grids", [[(1, 1), (1, 1)], [(5, 5), (2, 2)], [(2, 2), (5, 5)], [(3, 4), (4, 3)]])
+def test_frames_in_flight_every_cut_and_grid(mf, cut, grids):
+    # the overlapped hand-out order is built (and passes the planner's dependency check)
+    # for every cut and tiling, with the tasks of batch 1 once per frame
+    net = _net(mf, synth.YOLO16, 96)
+    one = mf.Plan(net, cut, grids, dry_run=True).stats()
+    st = mf.Plan(net, cut, grids, batch=3, dry_run=True).stats()
+    assert st["frames_overlapped"] == 1
+    assert st["n_tasks"] == 3 * one["n_tasks"]
+    assert abs(st["executed_flops"] - 3 * one["executed_flops"]) < 1e-6 * st["executed_flops"]
