@@ -137,8 +137,11 @@ def test_bf16_tiny3_64_grid2x2(mf):
 
 @pytest.mark.parametrize("cut,grids", [(None, [(1, 1)]), (None, [(3, 3)]), (2, [(5, 5), (2, 2)]),
                                        (4, [(4, 4), (3, 3)]), (8, [(5, 5), (2, 2)]), (8, [(1, 1), (1, 1)]),
-                                       (12, [(5, 5), (5, 5)]), (12, [(7, 2), (1, 3)])])
+                                       (12, [(5, 5), (5, 5)]), (12, [(7, 2), (1, 3)]),
+                                       (8, [(2, 2), (5, 5)]), (4, [(3, 4), (4, 3)])])
 def test_bf16_yolo16_96_batch2(mf, cut, grids):
+    # two frames in one launch: with two groups the second frame's first group is handed
+    # out between the first frame's second-group stages
     layers = synth.YOLO16
     params = synth.make_params(layers, 3, 41, "bf16")
     x = synth.make_input(2, 96, 96, 3, 42, "bf16")
