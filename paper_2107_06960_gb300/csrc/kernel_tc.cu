@@ -590,20 +590,32 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
         const uint32_t a_hi = (uint32_t)(a_desc0 >> 32);
         uint32_t a_lo = (uint32_t)a_desc0;  // tap (ky, kx) of the plain form: + ky * cols_box + kx
         int kx = 0;
+        // paired form: offset (16-byte units) and column of tap 2t, advanced by two taps per blob
+        const uint32_t a_base16 = (a_base & 0x3FFFFu) >> 4;
+        uint32_t oa16 = 0;
+        int xa = 0;
         for (int t = 0; t < j.n_bsteps; ++t) {
             uint32_t a_lo_t, a_hi_t;
             if (PAIRED) {
-                // taps (2t, 2t+1) as the two K halves: LBO = their distance; for an odd tap
-                // count the last blob pairs zero weights with the last tap
-                int ta = 2 * t, tb = 2 * t + 1;
-                if (tb >= taps) {
-                    ta = taps - 2;
-                    tb = taps - 1;
+                // taps (2t, 2t+1) as the two K halves: LBO = their distance (in the low word's
+                // bits 16-29; the high word, SBO = one halo row, is the plain form's); for an odd
+                // tap count the last blob pairs zero weights with the last tap
+                uint32_t pa, pb;
+                if (2 * t + 1 < taps) {
+                    pa = oa16;
+                    pb = xa + 1 == j.k ? oa16 + (uint32_t)(j.cols_box - j.k + 1) : oa16 + 1u;
+                } else {
+                    pa = tap_off(taps - 2, j.k, j.cols_box) >> 4;
+                    pb = tap_off(taps - 1, j.k, j.cols_box) >> 4;
                 }
-                const uint32_t oa = tap_off(ta, j.k, j.cols_box);
-                const uint64_t ad = smem_desc(a_base + oa, tap_off(tb, j.k, j.cols_box) - oa, j.a_row);
-                a_lo_t = (uint32_t)ad;  // block offsets only touch the address field (no carry: addresses < 2^18)
-                a_hi_t = (uint32_t)(ad >> 32);
+                a_lo_t = (a_base16 + pa) | ((pb - pa) << 16);
+                a_hi_t = a_hi;
+                oa16 += 2u;
+                xa += 2;
+                if (xa >= j.k) {  // paired stages are 3x3 (a 1x1 layer needs more than 8 channels)
+                    xa -= j.k;
+                    oa16 += (uint32_t)(j.cols_box - j.k);
+                }
             } else {
                 a_lo_t = a_lo;
                 a_hi_t = a_hi;
