@@ -1028,10 +1028,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool pool = (rc.flags & 1) != 0, nhwc = (rc.flags & 2) != 0;
             // Work split between the warpgroups in units of one block x 32 output columns
             // (16 when N is an odd multiple of 16), dealt round-robin.
-            const int uw = (rc.n_blk % 32 == 0) ? 32 : 16;
-            const int upb = rc.n_blk / uw;  // units per block
-            for (int u = h; u < rc.nbk * upb; u += kEpiGroups) {
-                const int b = u / upb, q = (u - b * upb) * uw;
+            const int uw = (rc.n_blk & 31) == 0 ? 32 : 16;
+            const int upb = uw == 32 ? rc.n_blk >> 5 : rc.n_blk >> 4;  // units per block
+            // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
+            for (int b = 0, qi = h;; qi += kEpiGroups) {
+                while (qi >= upb) {
+                    qi -= upb;
+                    ++b;
+                }
+                if (b >= rc.nbk) break;
+                const int q = qi * uw;
                 const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
                 const bool valid = (Y < rc.ylim) && (X < rc.xlim);
                 // a pooled stage's conv region starts on even rows and columns and has even
