@@ -169,7 +169,9 @@ __device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, uint32_
 // the MMA issue loop (even one whose exit is a warp vote) more than halves the MMA
 // issue rate of the whole loop, while the same loop inside one asm statement costs
 // nothing.  So the poll, with its deadline on %globaltimer, lives in the asm, and a
-// timeout is recorded by every lane alike (no branch on the lane).
+// timeout is recorded by every lane alike (no branch on the lane).  The lanes poll in
+// step, so the result needs no vote: a vote and a warp barrier after every wait cost the
+// first layer ~7 % of its MMA phase.
 __device__ __forceinline__ void mbar_wait_mma(uint32_t bar, uint32_t parity, uint32_t* ctr, int64_t limit_ns,
                                               volatile int* broken) {
     const uint64_t lim = (uint64_t)(*broken ? 1000000LL : limit_ns);
@@ -192,11 +194,10 @@ __device__ __forceinline__ void mbar_wait_mma(uint32_t bar, uint32_t parity, uin
         : "=r"(ok)
         : "r"(bar), "r"(parity), "l"(lim)
         : "memory");
-    if (__any_sync(0xffffffffu, ok == 0u)) {
+    if (ok == 0u) {  // every lane polled the same barrier in step: ok is warp-uniform
         mafat_dev::record_status(ctr, MAFAT_DEV_PIPE);
         *broken = 1;
     }
-    __syncwarp();
 }
 
 __device__ __forceinline__ void mbar_arrive_elect(uint32_t bar) {
