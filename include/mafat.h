@@ -133,7 +133,7 @@ typedef struct {
     int32_t frames_overlapped;  /* 1: the hand-out order overlaps frame f's second group with frame
                                    f + 1's first (batch > 1, two groups, ring of a whole frame) */
     int32_t reserved;
-} mafat_plan_stats;
+} mafat_plan_stats_t;
 
 /* Build a network description: validates the layers and infers every layer's
  * shape, out = floor((in + 2*pad - k) / stride) + 1 (Sec. 4.1, Algorithm 2's
@@ -307,8 +307,12 @@ mafat_status mafat_search_measured(const mafat_net_t* net, const mafat_search_op
                                    mafat_search_candidate* out, int32_t max_out, int32_t* n_out,
                                    int32_t* best);
 
-/* Plan statistics (struct_size must be set by the caller). */
-mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out);
+/* Statistics of a plan: the useful, executed (halo recompute included) and issued
+ * FLOPs of a run, Algorithm 1's prediction for its configuration (Sec. 4.1), its
+ * tiles, tasks and work items, and the device memory it owns.  out is caller-owned
+ * host memory; out->struct_size must be set to sizeof(mafat_plan_stats_t) (EINVAL if
+ * smaller).  Host only; works on dry-run plans. */
+mafat_status mafat_plan_stats(const mafat_plan_t* plan, mafat_plan_stats_t* out);
 
 /* Per-item trace of the last run of a plan created with options.trace = 1
  * (synchronises `stream`).  out receives n_items records of MAFAT_TRACE_WORDS
@@ -344,20 +348,28 @@ const char* mafat_version(void);
  * device area inside this library, which every GPU that loads the library
  * keeps until exit; it calls no allocation routine.  Plans needing more
  * scratch than 32 MiB are refused with MAFAT_EINVAL; BF16 plans with
- * MAFAT_EUNSUPPORTED.  Layouts as mafat_run; asynchronous on `stream`.  All
- * calls share the area: calls that overlap on the GPU race.  The first call
- * on each device looks up the area's device address, so make it before any
- * stream capture starts.  Device-side wait errors of these calls are not
- * reported by mafat_sync_status (which reads the plan's own status word). */
+ * MAFAT_EUNSUPPORTED; input and output that overlap with MAFAT_EINVAL.  Layouts
+ * as mafat_run; asynchronous on `stream`.  All calls share the area: calls that
+ * overlap on the GPU race.  The first call on each device looks up the area's
+ * device address and clears its status word (a synchronous step), so make it
+ * before any stream capture starts.  Device-side wait errors of these calls go
+ * to the area's own status word: read them with mafat_noalloc_sync_status, not
+ * mafat_sync_status (which reads the plan's). */
 mafat_status mafat_run_fp32_noalloc(const mafat_plan_t* plan, const void* input, void* output, void* stream);
 
+/* Device status of mafat_run_fp32_noalloc calls on the current device; no
+ * counterpart in the paper.  Synchronises `stream`, then reads and clears the
+ * status word of the static area: MAFAT_OK, MAFAT_ETIMEOUT (a tile waited on
+ * another that never finished) or MAFAT_EDEVICE.  The first error since the last
+ * read is kept; later calls do not overwrite it.  Allocates nothing. */
+mafat_status mafat_noalloc_sync_status(void* stream);
+
 /* Diagnostic with no counterpart in the paper: one 128 x n x 16 bf16 tensor-core
- * product D = A * B^T on one CTA, to check the operand and accumulator layouts
- * the kernels use.  a_dev [128][16], b_dev [n][16] (bf16, row-major, device),
- * d_dev [128][n] fp32 (device); n in {16, 32, ..., 256}.  lbo_is_k selects which
- * descriptor offset field carries the K-direction stride.  Synchronous. */
-mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n,
-                             int32_t lbo_is_k, void* stream);
+ * product D = A * B^T on one CTA, with the shared-memory descriptor encoding and
+ * the accumulator layout the fused kernel uses, to check them.  a_dev [128][16],
+ * b_dev [n][16] (bf16, row-major, device), d_dev [128][n] fp32 (device); n in
+ * {16, 32, ..., 256}.  Synchronous. */
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, void* stream);
 
 #ifdef __cplusplus
 }

@@ -82,7 +82,7 @@ _SIGNATURES = [
     ("mafat_predict_mem", i32, [vp, i32, i32, i32, i32, i32, dbl, ctypes.POINTER(dbl)]),
     ("mafat_search", i32, [vp, dbl, dbl, ctypes.POINTER(i32), ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_balanced_bounds", i32, [vp, i32, i32, i32, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)]),
-    ("mafat_plan_stats_get", i32, [vp, ctypes.POINTER(PlanStats)]),
+    ("mafat_plan_stats", i32, [vp, ctypes.POINTER(PlanStats)]),
     ("mafat_search_measured", i32, [vp, ctypes.POINTER(SearchOptions), vp, ctypes.POINTER(SearchCandidate), i32,
                                     ctypes.POINTER(i32), ctypes.POINTER(i32)]),
     ("mafat_launches_per_run", i32, [vp]),
@@ -91,8 +91,9 @@ _SIGNATURES = [
     ("mafat_net_destroy", None, [vp]),
     ("mafat_last_error", ctypes.c_char_p, []),
     ("mafat_version", ctypes.c_char_p, []),
-    ("mafat_diag_umma", i32, [vp, vp, vp, i32, i32, vp]),
+    ("mafat_diag_umma", i32, [vp, vp, vp, i32, vp]),
     ("mafat_run_fp32_noalloc", i32, [vp, vp, vp, vp]),
+    ("mafat_noalloc_sync_status", i32, [vp]),
 ]
 EXPORTED = [s[0] for s in _SIGNATURES]
 
@@ -296,6 +297,12 @@ class Plan:
         area and must not overlap on the GPU."""
         _check(lib.mafat_run_fp32_noalloc(self.handle, _ptr(inp), _ptr(out), _stream(stream, inp)))
 
+    @staticmethod
+    def noalloc_sync_status(stream=None, like=None):
+        """Raises MafatError (ETIMEOUT / EDEVICE) if a device-side wait of an earlier
+        run_noalloc call on the current device ran out (mafat_noalloc_sync_status)."""
+        _check(lib.mafat_noalloc_sync_status(_stream(stream, like)))
+
     def run_host(self, inp_host, out_host, stream=None):
         """End to end on host tensors: inp_host NHWC [B][H][W][C] (the image batch as it
         comes, pinned for asynchronous copies), out_host NHWC; synchronises the stream."""
@@ -325,7 +332,7 @@ class Plan:
     def stats(self):
         s = PlanStats()
         s.struct_size = ctypes.sizeof(PlanStats)
-        _check(lib.mafat_plan_stats_get(self.handle, ctypes.byref(s)))
+        _check(lib.mafat_plan_stats(self.handle, ctypes.byref(s)))
         return {k: getattr(s, k) for k, _ in PlanStats._fields_ if k not in ("struct_size", "reserved")}
 
     def trace(self, stream=None):
@@ -354,8 +361,10 @@ class Plan:
             pass
 
 
-def diag_umma(a_dev, b_dev, d_dev, n, lbo_is_k=1, stream=None):
-    _check(lib.mafat_diag_umma(_ptr(a_dev), _ptr(b_dev), _ptr(d_dev), n, lbo_is_k, _stream(stream, a_dev)))
+def diag_umma(a_dev, b_dev, d_dev, n, stream=None):
+    """One 128 x n x 16 bf16 tensor-core product d = a * b^T with the fused kernel's
+    descriptor encoding and accumulator layout (mafat_diag_umma)."""
+    _check(lib.mafat_diag_umma(_ptr(a_dev), _ptr(b_dev), _ptr(d_dev), n, _stream(stream, a_dev)))
 
 
 def version():

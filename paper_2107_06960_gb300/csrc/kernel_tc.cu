@@ -49,10 +49,6 @@
 
 #include "sched.cuh"
 
-#ifndef MAFAT_NOSWZ_LBO_IS_K
-#define MAFAT_NOSWZ_LBO_IS_K 1
-#endif
-
 namespace {
 
 constexpr int kEpiGroups = 2;           // epilogue warpgroups, each over all 128 TMEM lanes
@@ -243,13 +239,12 @@ __device__ __forceinline__ void tc_commit_warp(uint32_t bar) {
 }
 
 // Shared-memory matrix descriptor, no swizzle: start >> 4 in bits 0-13, LBO >> 4
-// in 16-29, SBO >> 4 in 32-45, descriptor version 1 in bits 46-47, layout 0.
+// in 16-29, SBO >> 4 in 32-45, descriptor version 1 in bits 46-47, layout 0.  For
+// the K-major no-swizzle layout LBO is the stride between the two core matrices
+// along K and SBO the stride between 8-row groups along M / N (checked by
+// mafat_diag_umma against a float64 product).
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t k_stride, uint32_t mn_stride) {
-#if MAFAT_NOSWZ_LBO_IS_K
     const uint32_t lbo = k_stride, sbo = mn_stride;
-#else
-    const uint32_t lbo = mn_stride, sbo = k_stride;
-#endif
     uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
     d |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;
     d |= (uint64_t)((sbo & 0x3FFFFu) >> 4) << 32;
@@ -1090,13 +1085,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------------------
-// Diagnostic: one 128 x n x 16 MMA.  Operands are written to shared memory in
-// an interleaved core-matrix order [8-row group][K half][8 rows][8 k] (K stride
-// 128 B, M/N stride 256 B), chosen so that both assignments of the two
-// descriptor offset fields stay inside the operand buffers.
+// Diagnostic: one 128 x n x 16 MMA with the operand and accumulator layouts of
+// the fused kernel.  Operands are written to shared memory as K-major no-swizzle
+// core matrices, [8-row group][K half][8 rows][8 k] (K-direction core-matrix
+// stride 128 B, M / N stride 256 B), read through smem_desc as the kernel does.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(128, 1)
-    mafat_diag_umma_kernel(const __nv_bfloat16* a, const __nv_bfloat16* b, float* d, int n, int lbo_is_k) {
+    mafat_diag_umma_kernel(const __nv_bfloat16* a, const __nv_bfloat16* b, float* d, int n) {
     __shared__ __align__(1024) __nv_bfloat16 sa[128 * 16];
     __shared__ __align__(1024) __nv_bfloat16 sb[256 * 16];
     __shared__ __align__(8) uint64_t done_bar;
@@ -1127,22 +1122,8 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
     if (tid == 0) {
-        uint64_t adesc, bdesc;
-        const uint32_t kst = 128, mst = 256;
-        auto mk = [&](uint32_t addr, uint32_t lbo, uint32_t sbo) {
-            uint64_t dd = (uint64_t)((addr & 0x3FFFFu) >> 4);
-            dd |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;
-            dd |= (uint64_t)((sbo & 0x3FFFFu) >> 4) << 32;
-            dd |= (uint64_t)1 << 46;
-            return dd;
-        };
-        if (lbo_is_k) {
-            adesc = mk(smem_u32(sa), kst, mst);
-            bdesc = mk(smem_u32(sb), kst, mst);
-        } else {
-            adesc = mk(smem_u32(sa), mst, kst);
-            bdesc = mk(smem_u32(sb), mst, kst);
-        }
+        const uint64_t adesc = smem_desc(smem_u32(sa), 128u, 256u);
+        const uint64_t bdesc = smem_desc(smem_u32(sb), 128u, 256u);
         mma_bf16(tmem, adesc, bdesc, instr_desc_bf16(n, 128), 0u);
         tc_commit(smem_u32(&done_bar));
     }
@@ -1187,7 +1168,7 @@ cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, in
     return cudaGetLastError();
 }
 
-cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int lbo_is_k, cudaStream_t s) {
-    mafat_diag_umma_kernel<<<1, 128, 0, s>>>((const __nv_bfloat16*)a, (const __nv_bfloat16*)b, d, n, lbo_is_k);
+cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, cudaStream_t s) {
+    mafat_diag_umma_kernel<<<1, 128, 0, s>>>((const __nv_bfloat16*)a, (const __nv_bfloat16*)b, d, n);
     return cudaGetLastError();
 }

@@ -216,7 +216,8 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
 // parameters of an fp32 plan with its own scratch, cut tensor and counters left
 // out (the caller supplies them), plus the sizes those three need.
 mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* kp, size_t* ctr_bytes,
-                                        size_t* cut_bytes, size_t* scratch_bytes, int* grid, int* device) {
+                                        size_t* cut_bytes, size_t* scratch_bytes, size_t* in_bytes,
+                                        size_t* out_bytes, int* grid, int* device) {
     const mafat_plan_s* p = plan;
     if (p->dry_run) return fail(MAFAT_EINVAL, "plan was created with dry_run");
     if (p->dtype != MAFAT_FP32) return fail(MAFAT_EUNSUPPORTED, "this entry point runs fp32 plans only");
@@ -237,6 +238,8 @@ mafat_status mafat_internal_fp32_params(const mafat_plan_t* plan, MafatKParams* 
     *ctr_bytes = p->ctr_bytes;
     *cut_bytes = p->t.cfg.n_groups >= 2 ? p->cut_bytes : 0;
     *scratch_bytes = (size_t)p->scratch_bytes;
+    *in_bytes = p->in_bytes;
+    *out_bytes = p->out_bytes;
     *grid = p->grid;
     *device = p->device;
     return MAFAT_OK;
@@ -501,19 +504,40 @@ mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_ho
     const mafat::Layer& L0 = p->shapes.layers[0];
     const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
     if (!p->s_h2d) {
-        if ((e = cudaStreamCreateWithFlags(&p->s_h2d, cudaStreamNonBlocking)) != cudaSuccess ||
-            (e = cudaStreamCreateWithFlags(&p->s_d2h, cudaStreamNonBlocking)) != cudaSuccess)
-            return cuda_fail(e, "cudaStreamCreate");
-        for (auto& h : p->hs) {
+        // set up into locals and publish only when everything exists, so that a failure
+        // part-way leaves nothing half-made behind (the next call starts over)
+        mafat_plan_s::HostSlot hs[2];
+        cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
+        auto undo = [&](cudaError_t err, const char* what) {
+            for (auto& h : hs) {
+                if (h.d_nhwc) cudaFree(h.d_nhwc);
+                if (h.d_planar) cudaFree(h.d_planar);
+                if (h.d_out) cudaFree(h.d_out);
+                if (h.h2d_done) cudaEventDestroy(h.h2d_done);
+                if (h.compute_done) cudaEventDestroy(h.compute_done);
+                if (h.d2h_done) cudaEventDestroy(h.d2h_done);
+            }
+            if (s_h2d) cudaStreamDestroy(s_h2d);
+            if (s_d2h) cudaStreamDestroy(s_d2h);
+            return cuda_fail(err, what);
+        };
+        if ((e = cudaStreamCreateWithFlags(&s_h2d, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaStreamCreateWithFlags(&s_d2h, cudaStreamNonBlocking)) != cudaSuccess)
+            return undo(e, "cudaStreamCreate");
+        for (auto& h : hs) {
             if ((e = cudaMalloc(&h.d_nhwc, nhwc_bytes)) != cudaSuccess ||
                 (e = cudaMalloc(&h.d_planar, p->in_bytes)) != cudaSuccess ||
                 (e = cudaMalloc(&h.d_out, p->out_bytes)) != cudaSuccess)
-                return cuda_fail(e, "cudaMalloc");
+                return undo(e, "cudaMalloc");
             if ((e = cudaEventCreateWithFlags(&h.h2d_done, cudaEventDisableTiming)) != cudaSuccess ||
                 (e = cudaEventCreateWithFlags(&h.compute_done, cudaEventDisableTiming)) != cudaSuccess ||
                 (e = cudaEventCreateWithFlags(&h.d2h_done, cudaEventDisableTiming)) != cudaSuccess)
-                return cuda_fail(e, "cudaEventCreate");
+                return undo(e, "cudaEventCreate");
         }
+        p->hs[0] = hs[0];
+        p->hs[1] = hs[1];
+        p->s_d2h = s_d2h;
+        p->s_h2d = s_h2d;  // last: its presence marks the set-up as done
     }
     const int k = p->hs_next;
     mafat_plan_s::HostSlot& h = p->hs[k];
@@ -584,9 +608,18 @@ mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, vo
         const mafat::Layer& L0 = p->shapes.layers[0];
         const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
         if (!p->d_in_stage) {
-            if ((e = cudaMalloc(&p->d_in_stage, p->in_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
-            if ((e = cudaMalloc(&p->d_out_stage, p->out_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
-            if ((e = cudaMalloc(&p->d_in_nhwc, nhwc_bytes)) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+            // all three buffers or none (a failure part-way frees what it made)
+            void *in_stage = nullptr, *out_stage = nullptr, *in_nhwc = nullptr;
+            if ((e = cudaMalloc(&in_stage, p->in_bytes)) != cudaSuccess ||
+                (e = cudaMalloc(&out_stage, p->out_bytes)) != cudaSuccess ||
+                (e = cudaMalloc(&in_nhwc, nhwc_bytes)) != cudaSuccess) {
+                if (in_stage) cudaFree(in_stage);
+                if (out_stage) cudaFree(out_stage);
+                return cuda_fail(e, "cudaMalloc");
+            }
+            p->d_out_stage = out_stage;
+            p->d_in_nhwc = in_nhwc;
+            p->d_in_stage = in_stage;  // last: its presence marks the set-up as done
         }
         if ((e = cudaMemcpyAsync(p->d_in_nhwc, input_host, nhwc_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
             return cuda_fail(e, "cudaMemcpyAsync");
@@ -684,12 +717,12 @@ mafat_status mafat_search(const mafat_net_t* net, double limit_mib, double bias_
     return MAFAT_OK;
 }
 
-mafat_status mafat_plan_stats_get(const mafat_plan_t* plan, mafat_plan_stats* out) {
+mafat_status mafat_plan_stats(const mafat_plan_t* plan, mafat_plan_stats_t* out) {
     if (!plan || !out) return fail(MAFAT_EINVAL, "null argument");
-    if (out->struct_size < (int32_t)sizeof(mafat_plan_stats)) return fail(MAFAT_EINVAL, "struct_size too small");
+    if (out->struct_size < (int32_t)sizeof(mafat_plan_stats_t)) return fail(MAFAT_EINVAL, "struct_size too small");
     const mafat::PlanTables& t = plan->t;
-    mafat_plan_stats s{};
-    s.struct_size = (int32_t)sizeof(mafat_plan_stats);
+    mafat_plan_stats_t s{};
+    s.struct_size = (int32_t)sizeof(mafat_plan_stats_t);
     s.n_groups = t.cfg.n_groups;
     s.n_tiles = t.n_tiles;
     s.n_tasks = (int32_t)t.tasks.size();
@@ -739,11 +772,10 @@ void mafat_plan_destroy(mafat_plan_t* plan) {
 
 void mafat_net_destroy(mafat_net_t* net) { delete net; }
 
-mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, int32_t lbo_is_k,
-                             void* stream) {
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, void* stream) {
     if (!a_dev || !b_dev || !d_dev) return fail(MAFAT_EINVAL, "null argument");
     if (n < 16 || n > 256 || n % 16 != 0) return fail(MAFAT_EINVAL, "n must be a multiple of 16 in 16..256");
-    cudaError_t e = mafat_launch_diag_umma(a_dev, b_dev, d_dev, n, lbo_is_k ? 1 : 0, (cudaStream_t)stream);
+    cudaError_t e = mafat_launch_diag_umma(a_dev, b_dev, d_dev, n, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "diag launch");
     e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "diag sync");

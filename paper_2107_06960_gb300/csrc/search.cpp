@@ -118,9 +118,9 @@ mafat_status mafat_search_measured(const mafat_net_t* net, const mafat_search_op
         mafat_plan_t* plan = nullptr;
         st = mafat_plan_ex(net, c.n_groups, &cut, c.gn, c.gm, batch, opt->dtype, &po, &plan);
         if (st == MAFAT_OK) {
-            mafat_plan_stats ps{};
+            mafat_plan_stats_t ps{};
             ps.struct_size = (int32_t)sizeof(ps);
-            mafat_plan_stats_get(plan, &ps);
+            mafat_plan_stats(plan, &ps);
             mafat_plan_destroy(plan);
             plan = nullptr;
             int64_t cut_bytes = 0;

@@ -23,10 +23,14 @@ def mf():
     return mf
 
 
-def test_header_declares_the_three_paper_calls():
+def test_header_declares_the_boundary_calls():
+    """The three calls of the problem statement and the rest of the boundary: weights,
+    status, debug run, region / predictor / search / statistics queries, cleanup."""
     names = _declared()
-    for n in ("mafat_describe_net", "mafat_plan", "mafat_run"):
-        assert n in names
+    for n in ("mafat_describe_net", "mafat_plan", "mafat_run", "mafat_set_weights", "mafat_sync_status",
+              "mafat_run_debug", "mafat_tile_region", "mafat_predict_mem", "mafat_search", "mafat_plan_stats",
+              "mafat_plan_destroy", "mafat_net_destroy", "mafat_last_error"):
+        assert n in names, n
 
 
 def test_library_exports_every_declared_symbol(mf):

@@ -32,7 +32,7 @@ def mf():
     a = torch.from_numpy(rng.standard_normal((128, 16)).astype(np.float32)).to(torch.bfloat16).cuda()
     b = torch.from_numpy(rng.standard_normal((256, 16)).astype(np.float32)).to(torch.bfloat16).cuda()
     d = torch.zeros((128, 256), dtype=torch.float32, device="cuda")
-    mf.diag_umma(a, b, d, 256, 1)
+    mf.diag_umma(a, b, d, 256)
     ref = a.double().cpu().numpy() @ b.double().cpu().numpy().T
     if not np.allclose(d.cpu().numpy(), ref, rtol=1e-5, atol=1e-5):
         pytest.fail("tensor-core descriptor layout check failed; not launching the fused kernels")
