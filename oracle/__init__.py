@@ -158,9 +158,10 @@ def tile_regions(layers, shapes, group, n, m, i, j, bounds=None):
 # ---------------------------------------------------------------------------
 
 def layer_group_terms(layers, shapes, group, n, m, i, j, l):
-    """The four terms Algorithm 1 accumulates for tile (i, j) at layer l, in
+    """The three sizes Algorithm 1 computes for tile (i, j) at layer l, in
     elements: scratch = w_out*h_out*c_in*F^2/S, input = w_in*h_in*c_in,
-    output = w_out*h_out*c_out (tile sizes from the Grid traversal)."""
+    output = w_out*h_out*c_out, with the tile's w/h in/out from the Grid
+    traversal (tile_regions) and c_in, c_out the layer's channel counts."""
     t, k, s, p, f = layers[l]
     (oy0, oy1, ox0, ox1), (iy0, iy1, ix0, ix1) = tile_regions(layers, shapes, group, n, m, i, j)[l]
     w_out, h_out = ox1 - ox0, oy1 - oy0
@@ -175,25 +176,17 @@ def layer_group_terms(layers, shapes, group, n, m, i, j, l):
 def predict_layer_group(layers, shapes, group, n, m, bias_mib=BIAS_MIB,
                         input_factor=2, bytes_per_elem=BYTES_PER_ELEM):
     """Algorithm 1, literal reading: the maximum over tiles (i, j) of the grid
-    and over the layers of the group of scratch + output + 2*input, converted
-    from elements to MiB, plus the bias.  The printed loop ``l <- bottom;
-    while l <= top; l <- l - 1`` is read as visiting every layer of the group
-    once (the order does not matter to a maximum); ``for i in 0..N`` is read
-    as i = 0..N-1."""
+    and over the layers of the group of scratch + output + 2*input (the terms
+    of layer_group_terms), converted from elements to MiB, plus the bias.  The
+    printed loop ``l <- bottom; while l <= top; l <- l - 1`` is read as visiting
+    every layer of the group once (the order does not matter to a maximum);
+    ``for i in 0..N`` is read as i = 0..N-1."""
     first, last = group
     best = 0.0
     for i in range(n):
         for j in range(m):
-            regs = tile_regions(layers, shapes, group, n, m, i, j)
             for l in range(first, last + 1):
-                t, k, s, p, f = layers[l]
-                (oy0, oy1, ox0, ox1), (iy0, iy1, ix0, ix1) = regs[l]
-                w_out, h_out = ox1 - ox0, oy1 - oy0
-                w_in, h_in = ix1 - ix0, iy1 - iy0
-                c_in, c_out = shapes[l]["c_in"], shapes[l]["c_out"]
-                scratch = w_out * h_out * c_in * (k * k) / s
-                inp = w_in * h_in * c_in
-                outp = w_out * h_out * c_out
+                scratch, inp, outp = layer_group_terms(layers, shapes, group, n, m, i, j, l)
                 mem = scratch + outp + inp * input_factor
                 if mem > best:
                     best = mem

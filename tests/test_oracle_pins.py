@@ -254,6 +254,46 @@ def test_predictor_units_reproduce_layer2_figures():
     assert oracle.BIAS_MIB == g["bias_mb"]
 
 
+ALG1_NET = [("conv", 3, 1, 1, 8), ("max", 2, 2, 0, 0), ("conv", 3, 1, 1, 16)]
+
+
+def _alg1_golden():
+    rows, mx = [], {}
+    for r in _read_golden("alg1_tiled_2x2.txt"):
+        if r[0].startswith("max_mem_elements"):
+            mx[r[0]] = int(r[1])
+        else:
+            rows.append(tuple(int(v) for v in r))
+    return rows, mx
+
+
+def test_predictor_tiled_terms_and_maximum_match_hand_computed_case():
+    # Algorithm 1 on a 2x2 tiling of a conv / pool / conv group over an 18x14x4 input,
+    # every tile's w/h in/out and the four terms worked out by hand from the
+    # algorithm's statement (tests/golden/alg1_tiled_2x2.txt).  The unique maximum
+    # sits at tile (1, 1), the last tile of both loops, whose rows and columns both
+    # carry halo from their neighbours; rows (9) and columns (7) differ, so a
+    # transposed axis, a skipped tile or a dropped term changes the value.
+    rows, mxs = _alg1_golden()
+    mx = mxs["max_mem_elements"]
+    shapes = oracle.layer_shapes(ALG1_NET, 18, 14, 4)
+    group = (0, 2)
+    for i, j, l, wo, ho, wi, hi, scratch, inp, outp, mem in rows:
+        (oy0, oy1, ox0, ox1), (iy0, iy1, ix0, ix1) = oracle.tile_regions(ALG1_NET, shapes, group, 2, 2, i, j)[l]
+        assert (ox1 - ox0, oy1 - oy0, ix1 - ix0, iy1 - iy0) == (wo, ho, wi, hi), (i, j, l)
+        s, a, o = oracle.layer_group_terms(ALG1_NET, shapes, group, 2, 2, i, j, l)
+        assert (s, a, o) == (scratch, inp, outp), (i, j, l)
+        assert s + o + 2 * a == mem
+    assert mx == max(r[-1] for r in rows)
+    assert oracle.predict_layer_group(ALG1_NET, shapes, group, 2, 2, bias_mib=0.0) == mx * 4 / 2 ** 20
+    assert oracle.predict_layer_group(ALG1_NET, shapes, group, 2, 2) == mx * 4 / 2 ** 20 + 31.0
+    # one group: predictMem is the group's prediction
+    assert oracle.predict_mem(ALG1_NET, shapes, None, [(2, 2)]) == mx * 4 / 2 ** 20 + 31.0
+    # non-square grids: rows and columns are not interchangeable
+    for (n, m), key in (((2, 1), "max_mem_elements_2x1"), ((1, 2), "max_mem_elements_1x2")):
+        assert oracle.predict_layer_group(ALG1_NET, shapes, group, n, m, bias_mib=0.0) == mxs[key] * 4 / 2 ** 20
+
+
 def test_predictor_untiled_is_whole_layer_maximum_plus_bias():
     layers = synth.YOLO16
     shapes = oracle.layer_shapes(layers, 608, 608, 3)

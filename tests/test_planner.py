@@ -1,3 +1,4 @@
+import os
 """Host planner of the C ABI (shapes, Grid regions, Algorithms 1-2, work tables) against the oracle.
 
 All on the CPU: network queries need no device, and plans are built with
@@ -66,6 +67,24 @@ def test_predictor_matches_oracle_exactly(mf, size):
         for f in (1, 2):
             ref = oracle.predict_layer_group(layers, shapes, (first, last), 3, 2, 31.0, input_factor=f)
             assert net.predict_layer_group(first, last, 3, 2, 31.0, f) == ref
+
+
+def test_predictor_matches_hand_computed_tiled_case(mf):
+    # the library's Algorithm 1 on the hand-worked 2x2 case of tests/golden/alg1_tiled_2x2.txt
+    layers = [("conv", 3, 1, 1, 8), ("max", 2, 2, 0, 0), ("conv", 3, 1, 1, 16)]
+    net = mf.Net(layers, 18, 14, 4)
+    mx = {}
+    with open(os.path.join(os.path.dirname(__file__), "golden", "alg1_tiled_2x2.txt")) as fh:
+        for line in fh:
+            if line.startswith("max_mem_elements"):
+                mx[line.split()[0]] = int(line.split()[1])
+    assert net.predict_layer_group(0, 2, 2, 2, 0.0, 2) == mx["max_mem_elements"] * 4 / 2 ** 20
+    assert net.predict_layer_group(0, 2, 2, 1, 0.0, 2) == mx["max_mem_elements_2x1"] * 4 / 2 ** 20
+    assert net.predict_layer_group(0, 2, 1, 2, 0.0, 2) == mx["max_mem_elements_1x2"] * 4 / 2 ** 20
+    for (i, j) in ((0, 0), (1, 1)):
+        out_r, in_r = net.tile_region(0, 2, 2, 2, i, j, 0)
+        ref = oracle.tile_regions(layers, oracle.layer_shapes(layers, 18, 14, 4), (0, 2), 2, 2, i, j)[0]
+        assert out_r == ref[0] and in_r == ref[1]
 
 
 def test_search_matches_oracle_for_table1_limits(mf):
