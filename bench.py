@@ -216,7 +216,7 @@ def run_sweep(args):
     H, W = wl["h"], wl["w"]
     net = mf.Net(wl["layers"], H, W, 3)
     net.set_params(wl["params"])
-    xin = torch.from_numpy(mf.to_planar(wl["input"])).to(torch.bfloat16).cuda()
+    xin = torch.from_numpy(wl["input"]).to(torch.bfloat16).cuda()
     sh = net.shape(len(wl["layers"]) - 1)
     out = torch.empty((1, sh[3], sh[4], sh[5]), dtype=torch.bfloat16, device="cuda")
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device="cuda")
@@ -321,7 +321,7 @@ def main():
     plan = mf.Plan(net, wl["cut"], wl["grids"], batch=B, dtype=dt)
     st = plan.stats()
     sh = net.shape(len(wl["layers"]) - 1)
-    xin = torch.from_numpy(mf.to_planar(wl["input"])).to(tdt).to(dev)
+    xin = torch.from_numpy(wl["input"]).to(tdt).to(dev)  # NHWC [B][H][W][3], as the image comes
     out = torch.empty((B, sh[3], sh[4], sh[5]), dtype=tdt, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()
@@ -359,7 +359,7 @@ def main():
     if K > 1 and B == 1 and wl["cut"] is not None:
         plan_k = mf.Plan(net, wl["cut"], wl["grids"], batch=K, dtype=dt)
         st_k = plan_k.stats()
-        xk = torch.from_numpy(mf.to_planar(synth.make_input(K, H, W, 3, synth.SEED_BASE + 77, wl["dtype"])))
+        xk = torch.from_numpy(synth.make_input(K, H, W, 3, synth.SEED_BASE + 77, wl["dtype"]))
         xk = xk.to(tdt).to(dev)
         outk = torch.empty((K, sh[3], sh[4], sh[5]), dtype=tdt, device=dev)
         for _ in range(args.warmup):

@@ -172,14 +172,19 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
                            const int32_t* grid_n, const int32_t* grid_m, int32_t batch,
                            int32_t dt, const mafat_plan_options* opt, mafat_plan_t** out);
 
-/* Run the plan on `stream` (asynchronous): one persistent fused kernel.
- *   input : device, [batch][ceil(C/8)][H][W][8] elements of the plan's dtype
- *           (channel octets outermost; for C <= 8 this is NHWC with the
- *           channel dimension padded to 8), padded channels zero.
+/* Run the plan on `stream` (asynchronous): one persistent fused kernel running
+ * every group and tile of the plan (Sec. 3-4).
+ *   input : device, NHWC [batch][H][W][C] elements of the plan's dtype, the
+ *           image batch as it comes (C = the net's input channels, e.g. 3).
  *   output: device, NHWC [batch][H_out][W_out][C_out] of the plan's dtype.
- * Both caller-owned.  Returns launch errors only; device-side wait errors are
- * reported by mafat_sync_status.  Calls on one plan must not overlap in time
- * (they share the plan's workspace).  Capturable into a CUDA graph. */
+ * Both caller-owned, 16-byte aligned, not overlapping (EINVAL otherwise).  The
+ * first layer reads the NHWC input in place: BF16 plans with C < 8 load raw
+ * image rows and widen them to 8 channels inside the kernel, which needs rows of
+ * W * C * 2 bytes to be a multiple of 16 (and C = 8 is read as it is); for other
+ * widths, and for C > 8, one small layout kernel first writes an octet-planar
+ * copy into plan-owned memory (two launches, see mafat_launches_per_run).  Returns launch errors only; device-side wait
+ * errors are reported by mafat_sync_status.  Calls on one plan must not overlap
+ * in time (they share the plan's workspace).  Capturable into a CUDA graph. */
 mafat_status mafat_run(const mafat_plan_t* plan, const void* input, void* output, void* stream);
 
 /* mafat_run, then copy the group-1 output (the cut tensor, layout
@@ -191,8 +196,7 @@ mafat_status mafat_run_debug(const mafat_plan_t* plan, const void* input, void* 
 /* End-to-end call on HOST buffers.  input_host is the image batch as it comes,
  * NHWC [batch][H][W][C] in the plan's dtype (C = the net's input channels, no
  * padding); output_host is NHWC [batch][H_out][W_out][C_out] as for mafat_run.
- * Copies the input to plan-owned device memory, converts it there to the
- * octet-planar layout mafat_run reads (one small kernel), runs, copies the
+ * Copies the input to plan-owned device memory, runs mafat_run on it, copies the
  * output back and synchronises `stream`; returns the device status as
  * mafat_sync_status does.  Pinned host memory gives asynchronous copies.
  * Allocates the plan's staging buffers on its first call. */
@@ -201,7 +205,7 @@ mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, vo
 
 /* Frames in flight on HOST buffers: the asynchronous form of mafat_run_host
  * (same layouts).  Enqueues the input upload on a plan-owned copy stream, the
- * layout conversion and the run on `stream`, and the read-back of the output on a
+ * run on `stream`, and the read-back of the output on a
  * second plan-owned copy stream, then returns; two staging slots alternate, so
  * the upload of one frame overlaps the run of the one before.  input_host must
  * stay unchanged, and output_host unread, until mafat_run_host_wait returns (or
@@ -326,7 +330,9 @@ mafat_status mafat_plan_stats(const mafat_plan_t* plan, mafat_plan_stats_t* out)
 #define MAFAT_TRACE_WORDS 10
 mafat_status mafat_plan_trace(const mafat_plan_t* plan, uint64_t* out, int64_t max_words, void* stream);
 
-/* Number of kernel launches one mafat_run makes. */
+/* Number of kernel launches one mafat_run makes: 1, or 2 for a BF16 plan whose
+ * input needs the layout kernel (C > 8, or C < 8 with rows of W * C * 2 bytes
+ * that are not a multiple of 16). */
 int32_t mafat_launches_per_run(const mafat_plan_t* plan);
 
 void mafat_plan_destroy(mafat_plan_t* plan);

@@ -285,6 +285,8 @@ class Plan:
         self.cut, self.grids, self.batch, self.dtype = cut, grids, batch, dtype
 
     def run(self, inp, out, stream=None):
+        """mafat_run: inp NHWC [B][H][W][C] and out NHWC [B][H_out][W_out][C_out], both
+        device tensors of the plan's dtype."""
         _check(lib.mafat_run(self.handle, _ptr(inp), _ptr(out), _stream(stream, inp)))
 
     def run_debug(self, inp, cut_out, out, stream=None):
@@ -371,19 +373,9 @@ def version():
     return lib.mafat_version().decode()
 
 
-def to_planar(x):
-    """Host layout helper: [B][H][W][C] array -> the input layout [B][ceil(C/8)][H][W][8],
-    padded channels zero (numpy)."""
-    import numpy as np
-    B, H, W, C = x.shape
-    c8 = (C + 7) // 8
-    xp = np.zeros((B, H, W, c8 * 8), dtype=np.float32)
-    xp[..., :C] = x
-    return np.ascontiguousarray(xp.reshape(B, H, W, c8, 8).transpose(0, 3, 1, 2, 4))
-
-
 def from_planar(xp, C):
-    """Host layout helper: [B][C8][H][W][8] -> [B][H][W][C] (numpy)."""
+    """Host layout helper for the cut tensor of run_debug: octet-planar
+    [B][C8][H][W][8] -> NHWC [B][H][W][C] (numpy)."""
     import numpy as np
     B, c8, H, W, _ = xp.shape
     return np.ascontiguousarray(xp.transpose(0, 2, 3, 1, 4).reshape(B, H, W, c8 * 8)[..., :C])

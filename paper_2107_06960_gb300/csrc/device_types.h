@@ -21,6 +21,12 @@
 #pragma once
 #include <stdint.h>
 
+#if defined(__CUDACC__)
+#define MAFAT_HD __host__ __device__
+#else
+#define MAFAT_HD
+#endif
+
 #define MAFAT_BLK_ROWS 16   // conv output rows of one M block
 #define MAFAT_BLK_COLS 8    // conv output columns of one M block (M = 128)
 #define MAFAT_MAX_MB 4      // M blocks per work item
@@ -64,7 +70,24 @@ struct MafatStageDev {
     int32_t sb_off;       // offset into the scale / bias arrays
     int32_t lookahead;    // 1: a CTA takes its next item as soon as this stage's item is loaded
     int64_t w32_off;      // element offset of the fp32 weights [cout][cin][k][k]
+    // How a task of this stage that reads the caller's input (NHWC [frames][H][W][cin]) gets its
+    // A halo into shared memory (tensor-core kernel; other tasks read octet-planar buffers):
+    //   MAFAT_IN_PLANAR: one 4-D box per chunk (cin == 8, whose NHWC is one octet plane, or a
+    //                    copy converted to octet-planar before the launch);
+    //   MAFAT_IN_GATHER: cin < 8: the box's rows of raw NHWC elements (raw_e per row, from a
+    //                    16-byte aligned element) land in the stage's tail, and the gather warp
+    //                    expands them into the one-octet halo, channels cin..7 zero.
+    int32_t in_mode;
+    int32_t raw_e;        // MAFAT_IN_GATHER: elements of one raw row in shared memory (multiple of 8)
 };
+
+enum { MAFAT_IN_PLANAR = 0, MAFAT_IN_GATHER = 1 };
+
+// Byte offset of the raw rows inside an A stage (MAFAT_IN_GATHER): after the expanded
+// one-octet halo of rows_box x cols_box pixels, on a 128-byte boundary.
+inline MAFAT_HD int mafat_raw_offset(int rows_box, int cols_box) {
+    return (rows_box * cols_box * 16 + 127) & ~127;
+}
 
 struct MafatTaskDev {
     int32_t stage;        // index into the stage table

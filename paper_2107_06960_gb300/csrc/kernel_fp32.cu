@@ -61,15 +61,18 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
             float acc[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+            // the caller's input is NHWC; every other buffer is octet-planar
+            const bool nhwc_in = tk.in_kind == MAFAT_BUF_USER_IN;
+            const int pix_stride = nhwc_in ? st.cin : 8;
             for (int ci = 0; ci < st.cin; ++ci) {
-                const float* in_c = in + (size_t)(ci >> 3) * tk.in_h * tk.in_w * 8 + (ci & 7);
+                const float* in_c = nhwc_in ? in + ci : in + (size_t)(ci >> 3) * tk.in_h * tk.in_w * 8 + (ci & 7);
                 for (int ky = 0; ky < k; ++ky) {
                     const int ly = Y + ky - st.pad - tk.in_y0;
                     for (int kx = 0; kx < k; ++kx) {
                         const int lx = X + kx - st.pad - tk.in_x0;
                         float v = 0.f;
                         if (ly >= 0 && ly < tk.in_h && lx >= 0 && lx < tk.in_w)
-                            v = in_c[((size_t)ly * tk.in_w + lx) * 8];
+                            v = in_c[((size_t)ly * tk.in_w + lx) * pix_stride];
                         const float* wp = w + ((size_t)o0 * st.cin + ci) * kk + ky * k + kx;
 #pragma unroll
                         for (int q = 0; q < 8; ++q) acc[q] = fmaf(__ldg(wp + (size_t)q * st.cin * kk), v, acc[q]);

@@ -28,12 +28,13 @@
 //    it, larger sets stream piece by piece (every copy costs a few hundred cycles
 //    of TMA time however small it is, so copies are large and few).
 //
-// Warp roles (352 threads): warps 0-7 epilogue (warp w reads TMEM lanes
+// Warp roles (384 threads): warps 0-7 epilogue (warp w reads TMEM lanes
 // 32(w%4)..+31 = conv rows 4(w%4)..+3 of a block; the two warpgroups take units
 // of one block x 32 columns in turn), warp 8 scheduler + TMA producer, warp 9 TMEM
 // allocator + MMA issuer, warp 10 publisher (bumps an item's completion counter
 // once all epilogue threads have stored it, so that the epilogue warps never wait
-// for their stores to reach L2).  Shared memory: 2 A halo stages, 2 weight
+// for their stores to reach L2), warp 11 gather (expands raw rows of a narrow NHWC
+// input image, e.g. 3-channel RGB, into the 8-channel halo layout of the first layer).  Shared memory: 2 A halo stages, 2 weight
 // buffers, a 4-deep queue of items with the record the epilogue needs (written by
 // the producer, so the epilogue reads no work table from global memory), and one
 // scale / bias slot per accumulator (copied in by the MMA warp and landing on the
@@ -57,7 +58,8 @@ constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr int kProducerWarp = kEpiWarps;
 constexpr int kMmaWarp = kEpiWarps + 1;
 constexpr int kPubWarp = kEpiWarps + 2;
-constexpr int kThreads = (kEpiWarps + 3) * 32;
+constexpr int kGatherWarp = kEpiWarps + 3;
+constexpr int kThreads = (kEpiWarps + 4) * 32;
 constexpr int kAStages = 2;
 constexpr int kQDepth = 4;
 constexpr int kAStageBytes = MAFAT_A_STAGE_BYTES;   // one A halo box, multiple of 1024
@@ -77,7 +79,8 @@ constexpr int kBarQEmpty = kBarQFull + kQDepth;
 constexpr int kBarDone = kBarQEmpty + kQDepth;
 constexpr int kBarEpiDone = kBarDone + 1;          // every epilogue thread has stored item e (slot e % 2)
 constexpr int kBarPubDone = kBarEpiDone + 2;       // the publisher has published item e (slot e % 2)
-constexpr int kNumBars = kBarPubDone + 2;
+constexpr int kBarRawFull = kBarPubDone + 2;       // raw NHWC rows have landed in A stage s (gather items)
+constexpr int kNumBars = kBarRawFull + kAStages;
 constexpr int kOffRec = 256;                        // kQDepth epilogue records
 constexpr int kRecStride = 128;
 constexpr int kOffQItems = kOffRec + kQDepth * kRecStride;
@@ -209,6 +212,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map
         "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
         " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
         : "memory");
 }
 
@@ -347,6 +359,14 @@ struct MmaRec {
 // What the MMA issuer, the epilogue and the publisher need of an item, written into its
 // queue slot by the producer (which has the work tables in registers anyway), so that
 // none of them reads a work table from global memory on its critical path.
+// What the gather warp needs of an item that reads raw NHWC rows (MAFAT_IN_GATHER).
+struct GatherRec {
+    int16_t on;              // 1: this item's A halo is built from raw rows by the gather warp
+    int16_t c;               // channels of the input (1..7)
+    int16_t raw_e;           // elements of one raw row in shared memory
+    int16_t s0;              // element of the first halo pixel's channel 0 within a raw row
+};
+
 struct EpiRec {
     __nv_bfloat16* out;      // output buffer of the task (frame and tile offset applied)
     int32_t x0, xlim;        // conv column of the item's block column; end of the task's columns
@@ -358,6 +378,7 @@ struct EpiRec {
     int32_t flags;           // bit 0: fused max-pool, bit 1: NHWC output, bit 2: never published (test hook)
     int32_t done_ctr, extra_ctr;
     MmaRec mma;
+    GatherRec gather;
 };
 static_assert(sizeof(EpiRec) <= kRecStride, "item record");
 
@@ -650,6 +671,42 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     }
 }
 
+// Gather of a 3x3 halo row from raw NHWC elements: the one-octet pixel x of a halo row
+// holds elements S0 + C x .. S0 + C x + C - 1 of the raw row (the rest zero).  One lane
+// builds whole rows: the row's RAW_E elements come in as 16-byte loads, and with C, S0 and
+// the row length fixed at compile time every pixel is a few byte permutes and one 16-byte
+// store.  The rows of a halo are dealt to the lanes in turn.
+template <int C, int S0, int RAW_E>
+__device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, int rows, int lane) {
+    constexpr int kCols = MAFAT_BLK_COLS + 2;  // a gathered stage is a 3x3 convolution
+    constexpr int kWords = RAW_E / 2;
+    static_assert(RAW_E % 8 == 0 && S0 + C * kCols <= RAW_E, "raw row");
+    for (int r = lane; r < rows; r += 32) {
+        uint32_t w[kWords];
+        const uint4* src = reinterpret_cast<const uint4*>(raw + (size_t)r * RAW_E * 2);
+#pragma unroll
+        for (int q = 0; q < kWords / 4; ++q) {
+            const uint4 v = src[q];
+            w[4 * q] = v.x;
+            w[4 * q + 1] = v.y;
+            w[4 * q + 2] = v.z;
+            w[4 * q + 3] = v.w;
+        }
+        uint4* out = reinterpret_cast<uint4*>(dst + (size_t)r * kCols * 16);
+#pragma unroll
+        for (int x = 0; x < kCols; ++x) {
+            uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+            for (int ch = 0; ch < C; ++ch) {
+                const int i = S0 + C * x + ch;
+                const uint32_t e = (w[i >> 1] >> (16 * (i & 1))) & 0xFFFFu;
+                o[ch >> 1] |= e << (16 * (ch & 1));
+            }
+            out[x] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     mafat_tc_kernel(const __grid_constant__ MafatKParams p, const __grid_constant__ CUtensorMap in_map) {
     extern __shared__ uint8_t smem_raw[];
@@ -683,8 +740,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < kQDepth; ++i) {
             mbar_init(bar(kBarQFull + i), 1);
-            mbar_init(bar(kBarQEmpty + i), kEpiWarps + 2);  // epilogue warps, MMA warp, publisher
+            mbar_init(bar(kBarQEmpty + i), kEpiWarps + 3);  // epilogue warps, MMA warp, publisher, gather warp
         }
+        for (int i = 0; i < kAStages; ++i) mbar_init(bar(kBarRawFull + i), 1);
         mbar_init(bar(kBarDone), 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(kBarEpiDone + i), kEpiThreads);
@@ -784,6 +842,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.mma.key = tk.stage * 256 + it.nb;
                     rc.mma.blob_elems = st.blob_elems;
                     rc.mma.sb = st.sb_off + it.nb * st.n_blk;
+                    rc.gather.on = 0;
+                    if (tk.in_kind == MAFAT_BUF_USER_IN && st.in_mode == MAFAT_IN_GATHER) {
+                        const int e_start = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * st.cin;
+                        rc.gather.on = 1;
+                        rc.gather.c = (int16_t)st.cin;
+                        rc.gather.raw_e = (int16_t)st.raw_e;
+                        rc.gather.s0 = (int16_t)(e_start - (e_start & ~7));
+                    }
                 }
                 mbar_arrive(bar(kBarQFull + qs));  // release: the record is visible to the consumers
                 ++q_cnt;
@@ -813,7 +879,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                                          : tk.in_kind == MAFAT_BUF_CUT   ? p.tmaps + p.cut_tmap
                                                                          : p.tmaps + tk.in_tmap;
                 const int c3 = tk.in_kind == MAFAT_BUF_SCRATCH ? 0 : tk.frame;
-                const int x0 = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * 8;
+                const int in_mode = tk.in_kind == MAFAT_BUF_USER_IN ? st.in_mode : MAFAT_IN_PLANAR;
+                const int px0 = tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0;  // first halo column
+                const int x0 = px0 * 8;
                 const int y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS - st.pad - tk.in_y0;
                 const uint32_t a_bytes = (uint32_t)(st.chunk8 * st.rows_box * st.cols_box * 16);
                 bool waited = false;
@@ -838,10 +906,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
+                    const uint32_t a_dst = sbase + kOffA + as * kAStageBytes;
                     mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
-                    mbar_arrive_expect_tx(bar(kBarAFull + as), a_bytes);
-                    tma_load_4d(sbase + kOffA + as * kAStageBytes, map, x0, y0, c * st.chunk8, c3,
-                                bar(kBarAFull + as));
+                    if (in_mode == MAFAT_IN_GATHER) {
+                        // raw NHWC rows from the 16-byte aligned element at or before the halo's
+                        // first one into the stage's tail; the gather warp builds the halo from
+                        // them and completes the stage's full barrier itself
+                        const int e_start = px0 * st.cin;
+                        mbar_arrive_expect_tx(bar(kBarRawFull + as), (uint32_t)(st.rows_box * st.raw_e * 2));
+                        tma_load_3d(a_dst + (uint32_t)mafat_raw_offset(st.rows_box, st.cols_box), map,
+                                    e_start & ~7, y0, c3, bar(kBarRawFull + as));
+                    } else {
+                        mbar_arrive_expect_tx(bar(kBarAFull + as), a_bytes);
+                        tma_load_4d(a_dst, map, x0, y0, c * st.chunk8, c3, bar(kBarAFull + as));
+                    }
                     ++a_cnt;
                     if (P > 1)
                         for (int g = c * st.n_bsteps; g < (c + 1) * st.n_bsteps; ++g)
@@ -991,6 +1069,77 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(bar(kBarPubDone + es));
                 ++e_cnt;
             }
+        }
+        __syncwarp();
+    } else if (warp == kGatherWarp) {
+        // ------------------------------------------------------------ gather warp (warp 11)
+        // For items whose input is a narrow NHWC image (fewer than 8 channels, e.g. RGB), the
+        // producer lands raw rows of the image in the A stage's tail; this warp expands them
+        // into the one-octet halo the MMAs read ([rows][cols][8 channels], channels c..7
+        // zero), makes the stores visible to the tensor core (async proxy) and completes the
+        // stage's full barrier.  It walks the item queue like the other consumers, counting A
+        // stages as the producer and the MMA warp do.
+        uint32_t q_cnt = 0, a_cnt = 0, raw_uses0 = 0, raw_uses1 = 0;
+        while (true) {
+            const int qs = (int)(q_cnt % kQDepth);
+            mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
+            const int ticket = q_items[qs];
+            GatherRec g{};
+            int n_chunks = 0, rows = 0, cols = 0;
+            if (ticket >= 0) {
+                g = recs[qs].gather;
+                n_chunks = recs[qs].mma.n_chunks;
+                rows = recs[qs].mma.rows_box;
+                cols = recs[qs].mma.cols_box;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
+            ++q_cnt;
+            if (ticket < 0) break;
+            if (g.on) {
+                const int as = (int)(a_cnt % kAStages);
+                const uint32_t uses = as ? raw_uses1++ : raw_uses0++;
+                mbar_wait(bar(kBarRawFull + as), uses & 1u, p.ctr, pipe_limit, broken, 32);
+                uint8_t* stage = smem + kOffA + as * kAStageBytes;
+                const uint8_t* raw_b = stage + mafat_raw_offset(rows, cols);
+                if (g.c == 3 && g.raw_e == 40 && cols == MAFAT_BLK_COLS + 2) {
+                    // RGB: the common case, one instance per alignment of the first element
+                    switch (g.s0) {
+#define MAFAT_GATHER_CASE(S) \
+    case S: gather_rows<3, S, 40>(raw_b, stage, rows, lane); break;
+                        MAFAT_GATHER_CASE(0) MAFAT_GATHER_CASE(1) MAFAT_GATHER_CASE(2) MAFAT_GATHER_CASE(3)
+                        MAFAT_GATHER_CASE(4) MAFAT_GATHER_CASE(5) MAFAT_GATHER_CASE(6) MAFAT_GATHER_CASE(7)
+#undef MAFAT_GATHER_CASE
+                        default: break;
+                    }
+                } else {
+                    // other channel counts: pixel by pixel (idx = r * cols + x dealt to the lanes)
+                    const uint16_t* raw = reinterpret_cast<const uint16_t*>(raw_b);
+                    uint4* dst = reinterpret_cast<uint4*>(stage);
+                    int r = 0, x = lane;
+                    while (x >= cols) {
+                        x -= cols;
+                        ++r;
+                    }
+                    for (int idx = lane; idx < rows * cols; idx += 32) {
+                        const uint16_t* src = raw + r * g.raw_e + g.s0 + x * g.c;
+                        uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                        for (int ch = 0; ch < 7; ++ch)
+                            if (ch < g.c) w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
+                        dst[idx] = make_uint4(w[0], w[1], w[2], w[3]);
+                        x += 32;
+                        while (x >= cols) {
+                            x -= cols;
+                            ++r;
+                        }
+                    }
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarAFull + as));
+            }
+            a_cnt += (uint32_t)n_chunks;
         }
         __syncwarp();
     } else {

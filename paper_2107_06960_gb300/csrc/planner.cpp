@@ -377,10 +377,34 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // fixed cost per item dominates)
             s.mb = std::min(s.mb, s.cin8 == 1 ? MAFAT_MAX_MB_PAIRED : MAFAT_MAX_MB);
             s.cols_box = MAFAT_BLK_COLS + L.k - 1;
+            // How the caller's NHWC input reaches the first stage's A halo (tensor-core plans; the
+            // fp32 kernel reads NHWC directly).  An image of fewer than 8 channels is read in place
+            // as raw rows, which a TMA box needs to be a multiple of 16 bytes; 8 channels are one
+            // octet plane already.  Other inputs (rows of another size, or more than 8 channels,
+            // i.e. not an image) are converted to octet-planar by a small kernel before the launch.
+            s.in_mode = MAFAT_IN_PLANAR;
+            s.raw_e = 0;
+            if (l == 0 && cfg.dtype == 0) {
+                if (L.c_in < 8 && ((int64_t)L.w_in * L.c_in) % 8 == 0) {
+                    s.in_mode = MAFAT_IN_GATHER;
+                    s.raw_e = (L.c_in * s.cols_box + 7 + 7) / 8 * 8;  // up to 7 leading elements of alignment
+                } else if (L.c_in != 8) {
+                    t.in_convert = 1;
+                }
+            }
             // input octets per A chunk: the largest that fits the A stage with mb blocks
             for (;;) {
                 s.rows_box = MAFAT_BLK_ROWS * s.mb + L.k - 1;
                 const int row_bytes = s.cols_box * 16 * s.rows_box;
+                if (s.in_mode == MAFAT_IN_GATHER) {
+                    // the expanded halo plus the raw rows it is built from share the stage
+                    s.chunk8 = 1;
+                    if (mafat_raw_offset(s.rows_box, s.cols_box) + s.rows_box * s.raw_e * 2 <= MAFAT_A_STAGE_BYTES ||
+                        s.mb == 1)
+                        break;
+                    s.mb /= 2;
+                    continue;
+                }
                 if (s.cin8 == 1) {
                     s.chunk8 = 1;
                 } else {
@@ -456,7 +480,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
     t.out_h = Ln.h_out;
     t.out_w = Ln.w_out;
     t.out_c = Ln.c_out;
-    const int64_t in_frame = (int64_t)t.in_c8 * 8 * L0.h_in * L0.w_in;
+    const int64_t in_frame = (int64_t)L0.c_in * L0.h_in * L0.w_in;  // the caller's NHWC input
     const int64_t cut_frame = (int64_t)t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_frame = (int64_t)t.out_h * t.out_w * t.out_c;
 
@@ -873,7 +897,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
 std::string validate_plan(const Net& net, const PlanTables& t) {
     const int n_tasks = (int)t.tasks.size();
     const Layer& L0 = net.layers[0];
-    const int64_t in_total = (int64_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in;
+    const int64_t in_total = (int64_t)t.cfg.batch * L0.c_in * L0.h_in * L0.w_in;
     const int64_t cut_total = (int64_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w;
     const int64_t out_total = (int64_t)t.cfg.batch * t.out_h * t.out_w * t.out_c;
     const int64_t scratch_total = t.scratch_elems;
@@ -903,6 +927,15 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
             return "K steps per blob must be 1, 2 or 4 (1 when taps are paired)";
         if (s.b_swz && (s.kst != 4 || s.paired || (s.blob_elems * 2) % 1024 != 0))
             return "swizzled blobs need 64 channels and whole 1024-byte atoms";
+        if (s.in_mode == MAFAT_IN_GATHER) {
+            const Layer& L = net.layers[s.layer];
+            if (s.layer != 0 || !s.paired || L.c_in >= 8 || (int64_t)L.w_in * L.c_in % 8 != 0)
+                return "raw-row gather on a stage that does not read a narrow NHWC input";
+            if (s.raw_e % 8 != 0 || s.raw_e > 256 || s.raw_e < 7 + L.c_in * s.cols_box)
+                return "raw row does not hold the halo's elements";
+            if (mafat_raw_offset(s.rows_box, s.cols_box) + (int64_t)s.rows_box * s.raw_e * 2 > MAFAT_A_STAGE_BYTES)
+                return "raw rows exceed their A stage";
+        }
     }
     std::vector<int> first_item(n_tasks, -1), last_item(n_tasks, -1);
     for (size_t i = 0; i < t.items.size(); ++i) {
@@ -918,8 +951,9 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         const Layer& L = net.layers[s.layer];
         if (last_item[ti] - first_item[ti] + 1 != k.n_items) return "task items not contiguous";
         // input buffer extent and coverage of every in-map tap of the conv rectangle
-        if (k.in_off < 0 || k.in_off + (int64_t)s.cin8 * 8 * k.in_h * k.in_w > buf_total(k.in_kind))
-            return "input buffer outside its allocation";
+        const int64_t in_elems = k.in_kind == MAFAT_BUF_USER_IN ? (int64_t)s.cin * k.in_h * k.in_w
+                                                                 : (int64_t)s.cin8 * 8 * k.in_h * k.in_w;
+        if (k.in_off < 0 || k.in_off + in_elems > buf_total(k.in_kind)) return "input buffer outside its allocation";
         int ny0 = std::max(k.cy0 - s.pad, 0), ny1 = std::min(k.cy0 + k.ch - 1 - s.pad + s.k, L.h_in);
         int nx0 = std::max(k.cx0 - s.pad, 0), nx1 = std::min(k.cx0 + k.cw - 1 - s.pad + s.k, L.w_in);
         if (k.in_y0 > ny0 || k.in_y0 + k.in_h < ny1 || k.in_x0 > nx0 || k.in_x0 + k.in_w < nx1)

@@ -129,6 +129,8 @@ struct PlanTables {
     // input / cut / output geometry (the cut tensor is group 1's output; the outputs of
     // groups 2 .. n_groups - 1 are layer maps in the scratch allocation)
     int in_c8 = 0;
+    int in_convert = 0;                  // 1: the NHWC input is converted to octet-planar before the launch
+                                         // (tensor-core plans whose raw input rows are not 16-byte multiples)
     int cut_h = 0, cut_w = 0, cut_c8 = 0;
     int out_h = 0, out_w = 0, out_c = 0;
     // box of the group-1 first stage (user input map) and group-2 first stage (cut map)

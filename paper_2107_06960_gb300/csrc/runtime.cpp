@@ -48,14 +48,16 @@ struct mafat_plan_s {
     // user-input tensor map, re-encoded when the input pointer changes
     CUtensorMap in_map;
     const void* in_map_ptr = nullptr;
-    // staging for mafat_run_host
+    // octet-planar copy of the input for tensor-core plans whose raw NHWC rows are not a
+    // multiple of 16 bytes (t.in_convert), made by a small kernel before each launch
+    void* d_in_planar = nullptr;
+    size_t in_planar_bytes = 0;
+    // staging for mafat_run_host: the NHWC input batch as copied from the host, the output
     void* d_in_stage = nullptr;
     void* d_out_stage = nullptr;
-    void* d_in_nhwc = nullptr;   // the NHWC image batch as copied from the host
     // two staging slots of mafat_run_host_async (frames in flight), its copy streams
     struct HostSlot {
-        void* d_nhwc = nullptr;
-        void* d_planar = nullptr;
+        void* d_in = nullptr;
         void* d_out = nullptr;
         cudaEvent_t h2d_done = nullptr, compute_done = nullptr, d2h_done = nullptr;
         bool used = false;
@@ -118,6 +120,31 @@ bool encode_planar_map(CUtensorMap* m, const void* base, int w, int h, int c8, i
     return true;
 }
 
+// 3-D tiled map over a narrow NHWC bf16 input (c < 8 channels) seen as rows of raw
+// elements [frames][h][w*c]: dim0 = w*c elements, dim1 = h, dim2 = frames.  Box = raw_e
+// elements (from a 16-byte aligned element) x rows_box rows x 1 frame; elements outside
+// the image read as zero (the convolution's zero padding, left and right included).
+bool encode_raw_rows_map(CUtensorMap* m, const void* base, int w, int h, int c, int frames, int raw_e,
+                         int rows_box, std::string* err) {
+    auto fn = encode_fn();
+    if (!fn) {
+        *err = "cuTensorMapEncodeTiled unavailable";
+        return false;
+    }
+    cuuint64_t dims[3] = {(cuuint64_t)w * c, (cuuint64_t)h, (cuuint64_t)frames};
+    cuuint64_t strides[2] = {(cuuint64_t)w * c * 2, (cuuint64_t)h * w * c * 2};
+    cuuint32_t box[3] = {(cuuint32_t)raw_e, (cuuint32_t)rows_box, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        *err = "cuTensorMapEncodeTiled (raw rows) failed (" + std::to_string((int)r) + ")";
+        return false;
+    }
+    return true;
+}
+
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 void free_plan_memory(mafat_plan_s* p) {
@@ -125,11 +152,9 @@ void free_plan_memory(mafat_plan_s* p) {
     p->allocs.clear();
     if (p->d_in_stage) cudaFree(p->d_in_stage);
     if (p->d_out_stage) cudaFree(p->d_out_stage);
-    if (p->d_in_nhwc) cudaFree(p->d_in_nhwc);
-    p->d_in_stage = p->d_out_stage = p->d_in_nhwc = nullptr;
+    p->d_in_stage = p->d_out_stage = nullptr;
     for (auto& h : p->hs) {
-        if (h.d_nhwc) cudaFree(h.d_nhwc);
-        if (h.d_planar) cudaFree(h.d_planar);
+        if (h.d_in) cudaFree(h.d_in);
         if (h.d_out) cudaFree(h.d_out);
         if (h.h2d_done) cudaEventDestroy(h.h2d_done);
         if (h.compute_done) cudaEventDestroy(h.compute_done);
@@ -183,8 +208,21 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
     kp.timeout_ns = p->timeout_ns;
     kp.trace = p->d_trace;
     if (p->dtype == MAFAT_BF16) {
-        const void* pf[] = {input, p->d_w, p->d_items, p->d_tasks, p->d_stages, p->d_scale, p->d_bias};
-        const int64_t pb[] = {(int64_t)p->in_bytes, (int64_t)p->t.weight_elems * 2,
+        const mafat::Layer& L0 = p->shapes.layers[0];
+        const MafatStageDev& s0 = p->t.stages[p->t.stage_first[0]];
+        const void* in_dev = input;
+        int64_t in_dev_bytes = (int64_t)p->in_bytes;
+        if (p->t.in_convert) {
+            // raw rows of this input are no multiple of 16 bytes (TMA strides must be): one small
+            // kernel writes the octet-planar copy the first stage reads
+            e = mafat_launch_to_planar(input, p->d_in_planar, p->t.cfg.batch, L0.h_in, L0.w_in, L0.c_in, p->t.in_c8,
+                                       2, s);
+            if (e != cudaSuccess) return cuda_fail(e, "layout conversion launch");
+            in_dev = p->d_in_planar;
+            in_dev_bytes = (int64_t)p->in_planar_bytes;
+        }
+        const void* pf[] = {in_dev, p->d_w, p->d_items, p->d_tasks, p->d_stages, p->d_scale, p->d_bias};
+        const int64_t pb[] = {in_dev_bytes, (int64_t)p->t.weight_elems * 2,
                               (int64_t)(p->t.items.size() * sizeof(MafatItemDev)),
                               (int64_t)(p->t.tasks.size() * sizeof(MafatTaskDev)),
                               (int64_t)(p->t.stages.size() * sizeof(MafatStageDev)), (int64_t)p->t.sb_elems * 4,
@@ -194,13 +232,17 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
             kp.pf_bytes[i] = pb[i];
             kp.pf_per[i] = ((pb[i] + p->grid - 1) / p->grid + 15) & ~(int64_t)15;
         }
-        if (p->in_map_ptr != input) {
+        if (p->in_map_ptr != in_dev) {
             std::string err;
-            const mafat::Layer& L0 = p->shapes.layers[0];
-            if (!encode_planar_map(&p->in_map, input, L0.w_in, L0.h_in, p->t.in_c8, p->t.cfg.batch,
-                                   p->t.in_cols_box, p->t.in_rows_box, p->t.in_chunk8, &err))
-                return fail(MAFAT_ECUDA, err);
-            p->in_map_ptr = input;
+            bool ok;
+            if (s0.in_mode == MAFAT_IN_GATHER)
+                ok = encode_raw_rows_map(&p->in_map, in_dev, L0.w_in, L0.h_in, L0.c_in, p->t.cfg.batch, s0.raw_e,
+                                         s0.rows_box, &err);
+            else  // octet-planar: an 8-channel NHWC input is one octet plane, or the converted copy
+                ok = encode_planar_map(&p->in_map, in_dev, L0.w_in, L0.h_in, p->t.in_c8, p->t.cfg.batch,
+                                       p->t.in_cols_box, p->t.in_rows_box, p->t.in_chunk8, &err);
+            if (!ok) return fail(MAFAT_ECUDA, err);
+            p->in_map_ptr = in_dev;
         }
         e = mafat_launch_tc(kp, p->in_map, p->grid, s);
     } else {
@@ -370,7 +412,8 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     p->dry_run = o.dry_run != 0;
     const mafat::PlanTables& t = p->t;
     const mafat::Layer& L0 = net->net.layers[0];
-    p->in_bytes = (size_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in * p->esz;
+    p->in_bytes = (size_t)t.cfg.batch * L0.c_in * L0.h_in * L0.w_in * p->esz;  // NHWC, as the caller holds it
+    p->in_planar_bytes = t.in_convert ? (size_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in * p->esz : 0;
     p->out_bytes = (size_t)t.cfg.batch * t.out_h * t.out_w * t.out_c * p->esz;
     p->cut_bytes = (size_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w * p->esz;
     p->ctr_bytes = (size_t)(MAFAT_CTR_BASE + t.n_counters) * sizeof(uint32_t);
@@ -410,6 +453,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     if ((e = dalloc(p, &p->d_bias, t.sb_elems * 4)) != cudaSuccess) return bail(e, "cudaMalloc");
     if ((e = dalloc(p, &p->d_scratch, (size_t)p->scratch_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
     if (t.cfg.n_groups >= 2 && (e = dalloc(p, &p->d_cut, p->cut_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
+    if (t.in_convert && (e = dalloc(p, &p->d_in_planar, p->in_planar_bytes)) != cudaSuccess) return bail(e, "cudaMalloc");
 
     std::vector<float> w32, sc, bi;
     mafat::pack_weights_fp32(net->net, t, w32, sc, bi);
@@ -501,8 +545,6 @@ mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_ho
     cudaStream_t s = (cudaStream_t)stream;
     std::lock_guard<std::mutex> lk(p->mu);
     cudaError_t e;
-    const mafat::Layer& L0 = p->shapes.layers[0];
-    const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
     if (!p->s_h2d) {
         // set up into locals and publish only when everything exists, so that a failure
         // part-way leaves nothing half-made behind (the next call starts over)
@@ -510,8 +552,7 @@ mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_ho
         cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
         auto undo = [&](cudaError_t err, const char* what) {
             for (auto& h : hs) {
-                if (h.d_nhwc) cudaFree(h.d_nhwc);
-                if (h.d_planar) cudaFree(h.d_planar);
+                if (h.d_in) cudaFree(h.d_in);
                 if (h.d_out) cudaFree(h.d_out);
                 if (h.h2d_done) cudaEventDestroy(h.h2d_done);
                 if (h.compute_done) cudaEventDestroy(h.compute_done);
@@ -525,8 +566,7 @@ mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_ho
             (e = cudaStreamCreateWithFlags(&s_d2h, cudaStreamNonBlocking)) != cudaSuccess)
             return undo(e, "cudaStreamCreate");
         for (auto& h : hs) {
-            if ((e = cudaMalloc(&h.d_nhwc, nhwc_bytes)) != cudaSuccess ||
-                (e = cudaMalloc(&h.d_planar, p->in_bytes)) != cudaSuccess ||
+            if ((e = cudaMalloc(&h.d_in, p->in_bytes)) != cudaSuccess ||
                 (e = cudaMalloc(&h.d_out, p->out_bytes)) != cudaSuccess)
                 return undo(e, "cudaMalloc");
             if ((e = cudaEventCreateWithFlags(&h.h2d_done, cudaEventDisableTiming)) != cudaSuccess ||
@@ -544,17 +584,14 @@ mafat_status mafat_run_host_async(const mafat_plan_t* plan, const void* input_ho
     // upload into slot k once the run that last read it is done
     if (h.used && (e = cudaStreamWaitEvent(p->s_h2d, h.compute_done, 0)) != cudaSuccess)
         return cuda_fail(e, "cudaStreamWaitEvent");
-    if ((e = cudaMemcpyAsync(h.d_nhwc, input_host, nhwc_bytes, cudaMemcpyHostToDevice, p->s_h2d)) != cudaSuccess ||
+    if ((e = cudaMemcpyAsync(h.d_in, input_host, p->in_bytes, cudaMemcpyHostToDevice, p->s_h2d)) != cudaSuccess ||
         (e = cudaEventRecord(h.h2d_done, p->s_h2d)) != cudaSuccess)
         return cuda_fail(e, "upload");
     // run on the caller's stream once the upload landed and slot k's last result was read back
     if ((e = cudaStreamWaitEvent(s, h.h2d_done, 0)) != cudaSuccess ||
         (h.used && (e = cudaStreamWaitEvent(s, h.d2h_done, 0)) != cudaSuccess))
         return cuda_fail(e, "cudaStreamWaitEvent");
-    if ((e = mafat_launch_to_planar(h.d_nhwc, h.d_planar, p->t.cfg.batch, L0.h_in, L0.w_in, L0.c_in, p->t.in_c8,
-                                    (int)p->esz, s)) != cudaSuccess)
-        return cuda_fail(e, "layout conversion launch");
-    mafat_status st = launch(p, h.d_planar, h.d_out, s);
+    mafat_status st = launch(p, h.d_in, h.d_out, s);
     if (st != MAFAT_OK) return st;
     if ((e = cudaEventRecord(h.compute_done, s)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
     // read the result back on its own stream
@@ -605,27 +642,19 @@ mafat_status mafat_run_host(const mafat_plan_t* plan, const void* input_host, vo
     {
         std::lock_guard<std::mutex> lk(p->mu);
         cudaError_t e;
-        const mafat::Layer& L0 = p->shapes.layers[0];
-        const size_t nhwc_bytes = (size_t)p->t.cfg.batch * L0.h_in * L0.w_in * L0.c_in * p->esz;
         if (!p->d_in_stage) {
-            // all three buffers or none (a failure part-way frees what it made)
-            void *in_stage = nullptr, *out_stage = nullptr, *in_nhwc = nullptr;
+            // both buffers or none (a failure part-way frees what it made)
+            void *in_stage = nullptr, *out_stage = nullptr;
             if ((e = cudaMalloc(&in_stage, p->in_bytes)) != cudaSuccess ||
-                (e = cudaMalloc(&out_stage, p->out_bytes)) != cudaSuccess ||
-                (e = cudaMalloc(&in_nhwc, nhwc_bytes)) != cudaSuccess) {
+                (e = cudaMalloc(&out_stage, p->out_bytes)) != cudaSuccess) {
                 if (in_stage) cudaFree(in_stage);
-                if (out_stage) cudaFree(out_stage);
                 return cuda_fail(e, "cudaMalloc");
             }
             p->d_out_stage = out_stage;
-            p->d_in_nhwc = in_nhwc;
             p->d_in_stage = in_stage;  // last: its presence marks the set-up as done
         }
-        if ((e = cudaMemcpyAsync(p->d_in_nhwc, input_host, nhwc_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        if ((e = cudaMemcpyAsync(p->d_in_stage, input_host, p->in_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
             return cuda_fail(e, "cudaMemcpyAsync");
-        if ((e = mafat_launch_to_planar(p->d_in_nhwc, p->d_in_stage, p->t.cfg.batch, L0.h_in, L0.w_in, L0.c_in,
-                                        p->t.in_c8, (int)p->esz, s)) != cudaSuccess)
-            return cuda_fail(e, "layout conversion launch");
         mafat_status st = launch(p, p->d_in_stage, p->d_out_stage, s);
         if (st != MAFAT_OK) return st;
         if ((e = cudaMemcpyAsync(output_host, p->d_out_stage, p->out_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
@@ -745,7 +774,10 @@ mafat_status mafat_plan_stats(const mafat_plan_t* plan, mafat_plan_stats_t* out)
     return MAFAT_OK;
 }
 
-int32_t mafat_launches_per_run(const mafat_plan_t* plan) { return plan ? 1 : 0; }
+int32_t mafat_launches_per_run(const mafat_plan_t* plan) {
+    if (!plan) return 0;
+    return plan->dtype == MAFAT_BF16 && plan->t.in_convert ? 2 : 1;
+}
 
 mafat_status mafat_plan_trace(const mafat_plan_t* plan, uint64_t* out, int64_t max_words, void* stream) {
     if (!plan || !out) return fail(MAFAT_EINVAL, "null argument");

@@ -2,11 +2,6 @@
 import numpy as np
 
 
-def to_planar(x):
-    from paper_2107_06960_gb300 import to_planar as tp
-    return tp(x)
-
-
 def from_planar(xp, C):
     from paper_2107_06960_gb300 import from_planar as fp
     return fp(xp, C)
@@ -20,7 +15,7 @@ def run_plan(mf, layers, params, x, cut, grids, dtype, plan_kwargs=None, repeat=
     net.set_params(params)
     plan = mf.Plan(net, cut, grids, batch=B, dtype=dtype, **(plan_kwargs or {}))
     tdt = torch.bfloat16 if dtype == mf.BF16 else torch.float32
-    xin = torch.from_numpy(to_planar(x)).to(tdt).cuda()
+    xin = torch.from_numpy(np.ascontiguousarray(x)).to(tdt).cuda()  # NHWC, as the image comes
     n = len(layers)
     sh = net.shape(n - 1)
     out = torch.full((B, sh[3], sh[4], sh[5]), float("nan"), dtype=tdt, device="cuda")

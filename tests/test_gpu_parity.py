@@ -107,6 +107,12 @@ def test_fp32_full_size(mf, name):
     (256, 512, 3, False, 20, 18, (1, 2)), # two output-channel blocks, four chunks
     (512, 256, 1, False, 19, 19, (2, 2)),
     (16, 16, 3, True, 18, 34, (4, 4)),    # smallest K chunk (2 octets)
+    (3, 32, 3, True, 36, 40, (2, 3)),     # RGB rows of 240 bytes: raw rows widened to 8 channels in the kernel
+    (3, 16, 3, False, 18, 56, (1, 8)),    # RGB, tiles starting at every column mod 8: all raw-row alignments
+    (4, 16, 3, False, 21, 34, (3, 2)),    # 4 channels, rows of 272 bytes, ragged blocks
+    (1, 16, 3, True, 20, 24, (2, 2)),     # 1 channel
+    (7, 16, 3, False, 17, 16, (1, 1)),    # 7 channels
+    (8, 32, 3, True, 20, 22, (2, 2)),     # 8 channels: the NHWC input is one octet plane
 ])
 def test_bf16_single_layer(mf, cin, cout, k, pool, h, w, grid):
     layers = [("conv", k, 1, (k - 1) // 2, cout)] + ([("max", 2, 2, 0, 0)] if pool else [])
@@ -377,16 +383,15 @@ def test_measured_search_picks_the_fastest_timed_plan(mf):
 
 def test_run_host_matches_device_run(mf):
     import torch
-    from tests.gpu_util import to_planar
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     net = mf.Net(wl["layers"], 608, 608, 3)
     net.set_params(wl["params"])
     plan = mf.Plan(net, 8, wl["grids"], batch=1, dtype=mf.BF16)
-    xin = torch.from_numpy(to_planar(wl["input"])).to(torch.bfloat16)
+    xin = torch.from_numpy(wl["input"]).to(torch.bfloat16)
     out_dev = torch.empty((1, 38, 38, 256), dtype=torch.bfloat16, device="cuda")
     plan.run(xin.cuda(), out_dev)
     plan.sync_status(like=out_dev)
-    # the host call takes the image as it comes (NHWC, 3 channels) and converts on the device
+    # the host call takes the same NHWC image from (pinned) host memory
     xh = torch.from_numpy(wl["input"]).to(torch.bfloat16).pin_memory()
     oh = torch.empty((1, 38, 38, 256), dtype=torch.bfloat16).pin_memory()
     plan.run_host(xh, oh)
@@ -397,7 +402,6 @@ def test_run_host_matches_device_run(mf):
 
 def test_run_host_async_frames_in_flight_match_device_runs(mf):
     import torch
-    from tests.gpu_util import to_planar
     wl = synth.workload("yolo16_416_1x3x3")
     net = mf.Net(wl["layers"], 416, 416, 3)
     net.set_params(wl["params"])
@@ -406,7 +410,7 @@ def test_run_host_async_frames_in_flight_match_device_runs(mf):
     ref = []
     for x in frames:
         out = torch.empty((1, 26, 26, 256), dtype=torch.bfloat16, device="cuda")
-        plan.run(torch.from_numpy(to_planar(x)).to(torch.bfloat16).cuda(), out)
+        plan.run(torch.from_numpy(x).to(torch.bfloat16).cuda(), out)
         plan.sync_status(like=out)
         ref.append(out.cpu())
     xh = [torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in frames]
@@ -421,13 +425,12 @@ def test_run_host_async_frames_in_flight_match_device_runs(mf):
 
 def test_run_host_fp32_matches_device_run(mf):
     import torch
-    from tests.gpu_util import to_planar
     wl = synth.workload("tiny3_64_fp32")
     net = mf.Net(wl["layers"], wl["h"], wl["w"], 3)
     net.set_params(wl["params"])
     plan = mf.Plan(net, wl["cut"], wl["grids"], batch=wl["batch"], dtype=mf.FP32)
     sh = net.shape(len(wl["layers"]) - 1)
-    xin = torch.from_numpy(to_planar(wl["input"])).float()
+    xin = torch.from_numpy(wl["input"]).float()
     out_dev = torch.empty((wl["batch"], sh[3], sh[4], sh[5]), dtype=torch.float32, device="cuda")
     plan.run(xin.cuda(), out_dev)
     plan.sync_status(like=out_dev)
@@ -439,12 +442,11 @@ def test_run_host_fp32_matches_device_run(mf):
 
 def test_cuda_graph_replay_matches(mf):
     import torch
-    from tests.gpu_util import to_planar
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     net = mf.Net(wl["layers"], 608, 608, 3)
     net.set_params(wl["params"])
     plan = mf.Plan(net, 8, wl["grids"], batch=1, dtype=mf.BF16)
-    xin = torch.from_numpy(to_planar(wl["input"])).to(torch.bfloat16).cuda()
+    xin = torch.from_numpy(wl["input"]).to(torch.bfloat16).cuda()
     out = torch.empty((1, 38, 38, 256), dtype=torch.bfloat16, device="cuda")
     plan.run(xin, out)
     plan.sync_status(like=xin)

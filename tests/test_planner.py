@@ -307,7 +307,7 @@ def test_plan_with_more_groups(mf, cuts, grids):
                 for l in (g[0], g[1]):
                     assert plan.tile_region(gi, i, j, l) == ref[l]
     planar = lambda l: (shapes[l]["c_out"] + 7) // 8 * 8 * shapes[l]["h_out"] * shapes[l]["w_out"]
-    io = 8 * 608 * 608 + 19 * 19 * 0 + shapes[15]["h_out"] * shapes[15]["w_out"] * shapes[15]["c_out"]
+    io = 3 * 608 * 608 + shapes[15]["h_out"] * shapes[15]["w_out"] * shapes[15]["c_out"]  # NHWC image, output
     io += sum(2 * planar(c - 1) for c in cuts)
     assert st["group_io_bytes"] == io * 2
     with pytest.raises(mf.MafatError):
@@ -355,3 +355,19 @@ def test_frames_in_flight_every_cut_and_grid(mf, cut, grids):
     assert st["frames_overlapped"] == 1
     assert st["n_tasks"] == 3 * one["n_tasks"]
     assert abs(st["executed_flops"] - 3 * one["executed_flops"]) < 1e-6 * st["executed_flops"]
+
+
+@pytest.mark.parametrize("c,w,launches", [(3, 608, 1), (3, 40, 1), (3, 28, 2), (4, 34, 1), (1, 20, 2), (8, 22, 1),
+                                          (16, 18, 2)])
+def test_input_layout_needs_no_conversion_when_rows_allow(mf, c, w, launches):
+    # mafat_run reads an NHWC image in place (raw rows widened inside the kernel) whenever
+    # a raw image row is a multiple of 16 bytes, 8 channels as they are; otherwise (and for
+    # inputs of more than 8 channels) a layout kernel runs first
+    layers = [("conv", 3, 1, 1, 16)]
+    net = mf.Net(layers, 16, w, c)
+    net.set_params(synth.make_params(layers, c, 3, "bf16"))
+    plan = mf.Plan(net, None, [(1, 1)], dtype=mf.BF16, dry_run=True)
+    assert plan.launches_per_run() == launches
+    assert plan.stats()["group_io_bytes"] == 2 * (16 * w * c + 16 * w * 16)
+    fplan = mf.Plan(net, None, [(1, 1)], dtype=mf.FP32, dry_run=True)
+    assert fplan.launches_per_run() == 1

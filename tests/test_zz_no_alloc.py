@@ -36,7 +36,7 @@ def _setup(mf, layers, h, c, cut, grids, seed, batch=1, **plan_kwargs):
     net = mf.Net(layers, h, h, c)
     net.set_params(params)
     plan = mf.Plan(net, cut, grids, batch=batch, dtype=mf.FP32, **plan_kwargs)
-    xin = torch.from_numpy(mf.to_planar(x)).cuda()
+    xin = torch.from_numpy(x).cuda()  # NHWC
     sh = net.shape(len(layers) - 1)
     return net, plan, xin, (batch, sh[3], sh[4], sh[5])
 
@@ -113,7 +113,7 @@ def test_noalloc_refuses_oversized_bf16_and_overlapping(mf):
     big = mf.Net(layers, 416, 416, 3)
     big.set_params(synth.make_params(layers, 3, 5, "fp32"))
     sh = big.shape(len(layers) - 1)
-    xin = torch.zeros((1, 1, 416, 416, 8), dtype=torch.float32, device="cuda")
+    xin = torch.zeros((1, 416, 416, 3), dtype=torch.float32, device="cuda")
     out = torch.zeros((1, sh[3], sh[4], sh[5]), dtype=torch.float32, device="cuda")
     plan = mf.Plan(big, None, [(3, 3)], dtype=mf.FP32)
     with pytest.raises(mf.MafatError) as e:
