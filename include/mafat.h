@@ -108,6 +108,11 @@ typedef struct {
     int32_t frame_major;        /* batch > 1 with two groups: 1 hands the frames out strictly one after
                                    another; 0 (default) overlaps frame f's second group with frame
                                    f + 1's first (the second group's small maps leave SMs idle) */
+    int32_t no_chain;           /* BF16 plans: 1 runs every convolution as its own stage.  0 (default)
+                                   chains a 3x3 convolution and the 1x1 convolution after it inside one
+                                   work item where both fit one TMEM accumulator buffer: the 3x3's
+                                   activated bf16 output stays in tensor memory and is the 1x1's A
+                                   operand, so it never reaches shared or global memory */
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */
@@ -371,11 +376,14 @@ mafat_status mafat_run_fp32_noalloc(const mafat_plan_t* plan, const void* input,
 mafat_status mafat_noalloc_sync_status(void* stream);
 
 /* Diagnostic with no counterpart in the paper: one 128 x n x 16 bf16 tensor-core
- * product D = A * B^T on one CTA, with the shared-memory descriptor encoding and
- * the accumulator layout the fused kernel uses, to check them.  a_dev [128][16],
- * b_dev [n][16] (bf16, row-major, device), d_dev [128][n] fp32 (device); n in
- * {16, 32, ..., 256}.  Synchronous. */
-mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, void* stream);
+ * product D = A * B^T on one CTA, with the operand and accumulator layouts the fused
+ * kernel uses, to check them: B (and, with a_in_tmem = 0, A) read from shared memory
+ * through the kernel's descriptor encoding; with a_in_tmem = 1, A written to tensor
+ * memory first (lane = row, two bf16 per 32-bit column), as the chained 3x3 -> 1x1
+ * layers pass their intermediate.  a_dev [128][16], b_dev [n][16] (bf16, row-major,
+ * device), d_dev [128][n] fp32 (device); n in {16, 32, ..., 256}.  Synchronous. */
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, int32_t a_in_tmem,
+                             void* stream);
 
 #ifdef __cplusplus
 }

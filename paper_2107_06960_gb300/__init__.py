@@ -35,7 +35,8 @@ class PlanOptions(ctypes.Structure):
     _fields_ = [("struct_size", i32), ("ring_slots", i32), ("wave_tiles", i32), ("max_ctas", i32),
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
                 ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32),
-                ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("frame_major", i32)]
+                ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("frame_major", i32),
+                ("no_chain", i32)]
 
 
 class PlanStats(ctypes.Structure):
@@ -91,7 +92,7 @@ _SIGNATURES = [
     ("mafat_net_destroy", None, [vp]),
     ("mafat_last_error", ctypes.c_char_p, []),
     ("mafat_version", ctypes.c_char_p, []),
-    ("mafat_diag_umma", i32, [vp, vp, vp, i32, vp]),
+    ("mafat_diag_umma", i32, [vp, vp, vp, i32, i32, vp]),
     ("mafat_run_fp32_noalloc", i32, [vp, vp, vp, vp]),
     ("mafat_noalloc_sync_status", i32, [vp]),
 ]
@@ -252,7 +253,7 @@ class Plan:
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
                  force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False,
-                 frame_major=False):
+                 frame_major=False, no_chain=False):
         self.net = net
         # cut: None (one group), the first layer of group 2, or a list of increasing cuts
         cut_list = [] if cut is None else (list(cut) if isinstance(cut, (list, tuple)) else [cut])
@@ -273,6 +274,7 @@ class Plan:
         opt.lookahead_items = lookahead_items
         opt.halo_reuse = int(halo_reuse)
         opt.frame_major = int(frame_major)
+        opt.no_chain = int(no_chain)
         if tile_bounds is not None:
             # per group (rows, cols): the non-uniform tiling; kept alive with the plan
             flat = [v for rows, cols in list(tile_bounds)[:n_groups] for v in list(rows) + list(cols)]
@@ -363,10 +365,10 @@ class Plan:
             pass
 
 
-def diag_umma(a_dev, b_dev, d_dev, n, stream=None):
+def diag_umma(a_dev, b_dev, d_dev, n, a_in_tmem=False, stream=None):
     """One 128 x n x 16 bf16 tensor-core product d = a * b^T with the fused kernel's
-    descriptor encoding and accumulator layout (mafat_diag_umma)."""
-    _check(lib.mafat_diag_umma(_ptr(a_dev), _ptr(b_dev), _ptr(d_dev), n, _stream(stream, a_dev)))
+    operand and accumulator layouts, A from shared or from tensor memory (mafat_diag_umma)."""
+    _check(lib.mafat_diag_umma(_ptr(a_dev), _ptr(b_dev), _ptr(d_dev), n, int(a_in_tmem), _stream(stream, a_dev)))
 
 
 def version():

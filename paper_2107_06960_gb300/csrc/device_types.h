@@ -79,6 +79,15 @@ struct MafatStageDev {
     //                    expands them into the one-octet halo, channels cin..7 zero.
     int32_t in_mode;
     int32_t raw_e;        // MAFAT_IN_GATHER: elements of one raw row in shared memory (multiple of 8)
+    // On-chip chaining of a 3x3 convolution and the 1x1 convolution after it (tensor-core plans):
+    // an item of a `chain` stage computes its pixels for all of the 3x3's channels into TMEM, the
+    // epilogue writes the activated bf16 result back into TMEM as the A operand of the 1x1, and
+    // the 1x1 (the next stage, marked `chained`, which has no tasks of its own) runs from there.
+    // Columns of one 256-column accumulator buffer: [0, n_blk) the 3x3's accumulator,
+    // [chain_a_col, + n_blk / 2) its bf16 result, [chain_out_col, + next stage's n_blk) the 1x1's.
+    int32_t chain;
+    int32_t chained;
+    int32_t chain_a_col, chain_out_col;
 };
 
 enum { MAFAT_IN_PLANAR = 0, MAFAT_IN_GATHER = 1 };

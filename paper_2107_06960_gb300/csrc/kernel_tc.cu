@@ -80,9 +80,10 @@ constexpr int kBarDone = kBarQEmpty + kQDepth;
 constexpr int kBarEpiDone = kBarDone + 1;          // every epilogue thread has stored item e (slot e % 2)
 constexpr int kBarPubDone = kBarEpiDone + 2;       // the publisher has published item e (slot e % 2)
 constexpr int kBarRawFull = kBarPubDone + 2;       // raw NHWC rows have landed in A stage s (gather items)
-constexpr int kNumBars = kBarRawFull + kAStages;
+constexpr int kBarMidFull = kBarRawFull + kAStages; // chain items: the 3x3's bf16 result is in TMEM (buffer b)
+constexpr int kNumBars = kBarMidFull + 2;
 constexpr int kOffRec = 256;                        // kQDepth epilogue records
-constexpr int kRecStride = 128;
+constexpr int kRecStride = 160;
 constexpr int kOffQItems = kOffRec + kQDepth * kRecStride;
 constexpr int kOffTmem = kOffQItems + 4 * kQDepth;
 constexpr int kOffBroken = kOffTmem + 4;
@@ -122,6 +123,26 @@ __device__ __forceinline__ void sb_load_elect(uint32_t bar, uint32_t slot, const
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%1], [%2], %4, [%0];\n\t"
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%5], [%3], %4, [%0];\n\t}" ::"r"(bar),
         "r"(slot), "l"(scale), "l"(bias), "r"(bytes), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4))
+        : "memory");
+}
+
+// The same for a chain item: the 3x3's n1 channels at slot offset 0 and the chained 1x1's n2
+// at slot offset n1 (scale and bias halves alike), all completing on bar.
+__device__ __forceinline__ void sb_load2_elect(uint32_t bar, uint32_t slot, const float* scale1, const float* bias1,
+                                               uint32_t bytes1, const float* scale2, const float* bias2,
+                                               uint32_t bytes2) {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t.reg .b32 tx;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "add.u32 tx, %4, %7;\n\t"
+        "add.u32 tx, tx, tx;\n\t"
+        "@e mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], tx;\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%1], [%2], %4, [%0];\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%8], [%3], %4, [%0];\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%9], [%5], %7, [%0];\n\t"
+        "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%10], [%6], %7, [%0];\n\t}" ::"r"(bar),
+        "r"(slot), "l"(scale1), "l"(bias1), "r"(bytes1), "l"(scale2), "l"(bias2), "r"(bytes2),
+        "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4)), "r"(slot + bytes1), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4) + bytes1)
         : "memory");
 }
 
@@ -281,6 +302,32 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
+// One MMA whose A operand is in tensor memory (a_tmem: column of K elements 0..1 of lane 0;
+// a K=16 step spans 8 columns, two bf16 per 32-bit column, lane = row of A), B in shared
+// memory, issued by one elected lane of the converged warp.
+__device__ __forceinline__ void mma_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t b_hi,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t.reg .b64 db;\n\t"
+        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 p, %5, 0;\n\t"
+        "mov.b64 db, {%2, %3};\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
+}
+
+// Store 16 consecutive 32-bit TMEM columns of this thread's lane (warp w reaches lanes
+// 32(w%4)..+31), then wait until the stores are done.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+        "%14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
 // The MMA warp runs its loop on all 32 lanes and one elected lane issues each MMA
 // (a lone lane in diverged code issues far slower).  The hot loop keeps descriptors
 // as 32-bit halves: the low word holds
@@ -350,10 +397,19 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 // of channel 0), the plane stride, and whether this lane stores at all.
 // What the MMA issuer needs of an item (all small).
 struct MmaRec {
-    int16_t k, cols_box, rows_box, n_chunks, n_bsteps, bpp, n_pieces, kst, paired, b_swz, nbk, pad;
+    int16_t k, cols_box, rows_box, n_chunks, n_bsteps, bpp, n_pieces, kst, paired, b_swz, nbk, chain;
     int32_t key;         // stage * 256 + channel block: identifies a resident weight set
     int32_t blob_elems;  // elements of one weight blob
     int32_t sb;          // offset of the item's first channel in the scale / bias arrays
+    int32_t n_mid;       // MMA N of the item's (first) convolution
+};
+
+// What the MMA issuer needs of a chain item's chained 1x1 (N, input chunks, K steps per blob,
+// swizzled blobs, blobs per piece, pieces, TMEM columns of its A operand and accumulator,
+// blob elements, scale / bias offset).  Read from the queue slot only on the chain path.
+struct ChainRec {
+    int16_t n2, nch2, kst2, swz2, bpp2, np2, a_col, out_col;
+    int32_t blob2, sb2;
 };
 
 // What the MMA issuer, the epilogue and the publisher need of an item, written into its
@@ -377,16 +433,26 @@ struct EpiRec {
     int32_t cout, ch_base;   // channels of the layer; first channel of the item
     int32_t flags;           // bit 0: fused max-pool, bit 1: NHWC output, bit 2: never published (test hook)
     int32_t done_ctr, extra_ctr;
+    int16_t chain;           // 1: chain item (first pass turns the 3x3's result into the 1x1's A operand)
+    int16_t n_mid;           // chain item: columns of the 3x3's accumulator
+    int16_t a_col, out_col;  // chain item: TMEM columns of the 1x1's A operand and of its accumulator
+};
+
+// A queue slot: the record of one item, in parts, so that every role copies only its own.
+struct ItemRec {
+    EpiRec epi;
     MmaRec mma;
+    ChainRec chain;
     GatherRec gather;
 };
-static_assert(sizeof(EpiRec) <= kRecStride, "item record");
+static_assert(sizeof(ItemRec) <= kRecStride, "item record");
 
 struct EpiDst {
     __nv_bfloat16* out;
     size_t pix, plane;
     int nhwc, cout, pool;
     bool store;
+    uint32_t tmem;  // nonzero: the packed bf16 result goes to these TMEM columns instead (chain items)
 };
 
 // Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1, NC = 16 or 32)
@@ -424,6 +490,12 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         }
         pk[i / 2] = pack_bf16x2(v[0], v[1]);
         pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
+    }
+    if constexpr (NC == 32) {
+        if (d.tmem) {  // a chain item's first pass: the 1x1's A operand, two bf16 per column
+            tmem_st16(d.tmem, pk);
+            return;
+        }
     }
     if (!d.pool) {
         if (!d.store) return;
@@ -671,6 +743,46 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     }
 }
 
+// The chained 1x1 of a chain item: A = the 3x3's activated bf16 result in TMEM (columns
+// acc + a_col .., 8 per K=16 step), B = the 1x1's weights streamed through the two
+// buffers piece by piece (never resident), D = TMEM columns acc + out_col .., N = n2.  The
+// K order is the 1x1's packed blob order: input chunk c, K step q = channels (c kst2 + q) 16 ...
+__device__ __forceinline__ void mma_chain_1x1(MmaState& s, uint32_t acc, int n2, int nch2, int kst2, bool swz2,
+                                              int bpp2, int np2, uint32_t blob_bytes2, int a_col, int out_col) {
+    const uint32_t idesc = instr_desc_bf16(n2, 128);
+    const uint32_t b_half = (uint32_t)n2 * 16u;
+    const uint32_t b_hi = swz2 ? desc_hi_sw128(1024u) : (uint32_t)(smem_desc(0u, b_half, 128u) >> 32);
+    const uint32_t b_step = swz2 ? 2u : 2u * (b_half >> 4);
+    const uint32_t blob16 = blob_bytes2 >> 4;
+    const uint32_t d = acc + (uint32_t)out_col;
+    uint32_t a = acc + (uint32_t)a_col;
+    uint32_t accumulate = 0;
+    int g = 0;
+    for (int pc = 0; pc < np2; ++pc) {
+        const int b = s.wb.next;
+        s.wb.next ^= 1;
+        if (s.wb.held(b)) {
+            tc_commit_warp(s.bar(kBarBEmpty + b));
+            s.wb.release(b);
+        }
+        mbar_wait_mma(s.bar(kBarBFull + b), s.wb.loads(b) & 1u, s.ctr, s.pipe_limit, s.broken);
+        s.wb.set_loaded(b, -1, false);
+        tc_fence_after();
+        const uint32_t addr = s.sbase + kOffB + (uint32_t)b * kBPieceBytes;
+        uint32_t b_lo = swz2 ? desc_lo_sw128(addr) : (uint32_t)smem_desc(addr, b_half, 128u);
+        const int nb = min(bpp2, nch2 - g);
+        for (int k = 0; k < nb; ++k, ++g) {
+            for (int q = 0; q < kst2; ++q) {
+                mma_tmem_a(d, a, b_lo + (uint32_t)q * b_step, b_hi, idesc, accumulate);
+                accumulate = 1u;
+                a += 8u;
+            }
+            b_lo += blob16;
+        }
+        tc_commit_warp(s.bar(kBarBEmpty + b));  // the piece is free once these MMAs are done
+    }
+}
+
 // Gather of a 3x3 halo row from raw NHWC elements: the one-octet pixel x of a halo row
 // holds elements S0 + C x .. S0 + C x + C - 1 of the raw row (the rest zero).  One lane
 // builds whole rows: the row's RAW_E elements come in as 16-byte loads, and with C, S0 and
@@ -715,7 +827,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int* q_items = reinterpret_cast<volatile int*>(smem + kOffQItems);
     volatile uint32_t* tmem_slot = reinterpret_cast<volatile uint32_t*>(smem + kOffTmem);
     volatile int* broken = reinterpret_cast<volatile int*>(smem + kOffBroken);
-    EpiRec* recs = reinterpret_cast<EpiRec*>(smem + kOffRec);
+    ItemRec* recs = reinterpret_cast<ItemRec*>(smem + kOffRec);
     auto bar = [&](int i) { return sbase + (uint32_t)(i * 8); };
 
     const int warp = threadIdx.x >> 5;
@@ -743,6 +855,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(bar(kBarQEmpty + i), kEpiWarps + 3);  // epilogue warps, MMA warp, publisher, gather warp
         }
         for (int i = 0; i < kAStages; ++i) mbar_init(bar(kBarRawFull + i), 1);
+        for (int i = 0; i < 2; ++i) mbar_init(bar(kBarMidFull + i), kEpiThreads);
         mbar_init(bar(kBarDone), 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(kBarEpiDone + i), kEpiThreads);
@@ -799,16 +912,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
                 }
                 MafatTaskDev tk;
-                MafatStageDev st;
+                MafatStageDev st, st2;
                 if (ticket >= 0) {  // two independent loads (the item names its stage)
                     tk = p.tasks[it.task];
                     st = p.stages[it.stage];
+                    if (st.chain) st2 = p.stages[it.stage + 1];  // the chained 1x1
                 }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                 q_items[qs] = ticket;
                 if (ticket >= 0) {
-                    EpiRec& rc = recs[qs];
+                    EpiRec& rc = recs[qs].epi;
+                    MmaRec& rm = recs[qs].mma;
+                    GatherRec& rg = recs[qs].gather;
                     rc.out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
                                               : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
                                                                                 : p.scratch) +
@@ -822,33 +938,54 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.out_w = tk.out_w;
                     rc.out_h = tk.out_h;
                     rc.nbk = it.nbk;
-                    rc.n_blk = st.n_blk;
-                    rc.cout = st.cout;
-                    rc.ch_base = it.nb * st.n_blk;
-                    rc.flags = (st.pool ? 1 : 0) | (tk.out_nhwc ? 2 : 0) | ((it.flags & 1) ? 4 : 0);
+                    // what the epilogue stores: the item's own output, or a chain item's 1x1 output
+                    rc.n_blk = st.chain ? st2.n_blk : st.n_blk;
+                    rc.cout = st.chain ? st2.cout : st.cout;
+                    rc.ch_base = st.chain ? 0 : it.nb * st.n_blk;
+                    rc.flags = ((st.chain ? st2.pool : st.pool) ? 1 : 0) | (tk.out_nhwc ? 2 : 0) |
+                               ((it.flags & 1) ? 4 : 0);
                     rc.done_ctr = tk.done_ctr;
                     rc.extra_ctr = it.extra_ctr;
-                    rc.mma.k = (int16_t)st.k;
-                    rc.mma.cols_box = (int16_t)st.cols_box;
-                    rc.mma.rows_box = (int16_t)st.rows_box;
-                    rc.mma.n_chunks = (int16_t)st.n_chunks;
-                    rc.mma.n_bsteps = (int16_t)st.n_bsteps;
-                    rc.mma.bpp = (int16_t)st.bpp;
-                    rc.mma.n_pieces = (int16_t)st.n_pieces;
-                    rc.mma.kst = (int16_t)st.kst;
-                    rc.mma.paired = (int16_t)st.paired;
-                    rc.mma.b_swz = (int16_t)st.b_swz;
-                    rc.mma.nbk = it.nbk;
-                    rc.mma.key = tk.stage * 256 + it.nb;
-                    rc.mma.blob_elems = st.blob_elems;
-                    rc.mma.sb = st.sb_off + it.nb * st.n_blk;
-                    rc.gather.on = 0;
+                    rm.k = (int16_t)st.k;
+                    rm.cols_box = (int16_t)st.cols_box;
+                    rm.rows_box = (int16_t)st.rows_box;
+                    rm.n_chunks = (int16_t)st.n_chunks;
+                    rm.n_bsteps = (int16_t)st.n_bsteps;
+                    rm.bpp = (int16_t)st.bpp;
+                    rm.n_pieces = (int16_t)st.n_pieces;
+                    rm.kst = (int16_t)st.kst;
+                    rm.paired = (int16_t)st.paired;
+                    rm.b_swz = (int16_t)st.b_swz;
+                    rm.nbk = it.nbk;
+                    rm.key = tk.stage * 256 + it.nb;
+                    rm.blob_elems = st.blob_elems;
+                    rm.sb = st.sb_off + it.nb * st.n_blk;
+                    rm.n_mid = st.n_blk;
+                    rm.chain = (int16_t)st.chain;
+                    rc.n_mid = (int16_t)st.n_blk;
+                    rc.chain = (int16_t)st.chain;
+                    if (st.chain) {
+                        ChainRec& rh = recs[qs].chain;
+                        rh.n2 = (int16_t)st2.n_blk;
+                        rh.nch2 = (int16_t)st2.n_chunks;
+                        rh.kst2 = (int16_t)st2.kst;
+                        rh.swz2 = (int16_t)st2.b_swz;
+                        rh.bpp2 = (int16_t)st2.bpp;
+                        rh.np2 = (int16_t)st2.n_pieces;
+                        rh.a_col = (int16_t)st.chain_a_col;
+                        rh.out_col = (int16_t)st.chain_out_col;
+                        rh.blob2 = st2.blob_elems;
+                        rh.sb2 = st2.sb_off;
+                        rc.a_col = (int16_t)st.chain_a_col;
+                        rc.out_col = (int16_t)st.chain_out_col;
+                    }
+                    rg.on = 0;
                     if (tk.in_kind == MAFAT_BUF_USER_IN && st.in_mode == MAFAT_IN_GATHER) {
                         const int e_start = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * st.cin;
-                        rc.gather.on = 1;
-                        rc.gather.c = (int16_t)st.cin;
-                        rc.gather.raw_e = (int16_t)st.raw_e;
-                        rc.gather.s0 = (int16_t)(e_start - (e_start & ~7));
+                        rg.on = 1;
+                        rg.c = (int16_t)st.cin;
+                        rg.raw_e = (int16_t)st.raw_e;
+                        rg.s0 = (int16_t)(e_start - (e_start & ~7));
                     }
                 }
                 mbar_arrive(bar(kBarQFull + qs));  // release: the record is visible to the consumers
@@ -926,6 +1063,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
                 }
 #undef MAFAT_LOAD_PIECE
+                if (st.chain) {
+                    // the chained 1x1's weights follow the 3x3's, streamed piece by piece (never
+                    // resident), in the order the MMA issuer consumes them
+                    const uint16_t* wset2 = p.w_bf16 + st2.w_off;
+                    const int G2 = st2.n_chunks * st2.n_bsteps;
+                    const uint32_t blob_bytes2 = (uint32_t)(st2.blob_elems * 2);
+                    for (int pc = 0; pc < st2.n_pieces; ++pc) {
+                        const int b_ = wb.next;
+                        wb.next ^= 1;
+                        mbar_wait(bar(kBarBEmpty + b_), (wb.loads(b_) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
+                        const int nblob_ = min(st2.bpp, G2 - pc * st2.bpp);
+                        const uint32_t bytes_ = (uint32_t)nblob_ * blob_bytes2;
+                        mbar_arrive_expect_tx(bar(kBarBFull + b_), bytes_);
+                        bulk_load(sbase + kOffB + b_ * kBPieceBytes, wset2 + (size_t)pc * st2.bpp * st2.blob_elems, bytes_,
+                                  bar(kBarBFull + b_));
+                        wb.set_loaded(b_, -1, false);
+                    }
+                }
                 if (!st.lookahead)
                     mbar_wait(bar(kBarAEmpty + (int)(a_cnt % kAStages)), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr,
                               pipe_limit, broken, 64);
@@ -956,6 +1111,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ms.trace = p.trace;
             const uint32_t tmem_u = (uint32_t)wu((int)tmem_base);
             uint32_t q_cnt = 0, acc_cnt = 0;
+            uint32_t mid_ph0 = 0, mid_ph1 = 0;  // MidFull phases consumed, per accumulator buffer
             bool issued = false;
             while (true) {
                 const int qs = (int)(q_cnt % kQDepth);
@@ -965,9 +1121,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 int n_blk = 0;
                 if (ticket >= 0) {
                     mr = recs[qs].mma;
-                    n_blk = recs[qs].n_blk;
+                    n_blk = mr.n_mid;  // N of the item's (first) convolution
                 }
-                mbar_arrive_elect(ms.bar(kBarQEmpty + qs));  // release: the record has been read
+                // release the slot once the record has been read (a chain item's slot is held until
+                // its chained 1x1's fields have been read, on the chain path)
+                const bool chain = ticket >= 0 && wu(mr.chain) != 0;
+                if (!chain) mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
                 MmaJob j;
@@ -995,8 +1154,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // the item's scale and bias go into the accumulator's slot (the epilogue of
                     // the slot's previous item is past it); the accumulator's full barrier then
                     // completes only once they have landed as well
-                    sb_load_elect(ms.bar(kBarAccFull + buf), ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes),
-                                  p.scale + sb, p.bias + sb, j.n_blk * 4u);
+                    const uint32_t slot = ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes);
+                    if (chain) {
+                        const int sb2 = wu(recs[qs].chain.sb2);
+                        sb_load2_elect(ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u,
+                                       p.scale + sb2, p.bias + sb2, (uint32_t)wu(recs[qs].chain.n2) * 4u);
+                    } else {
+                        sb_load_elect(ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u);
+                    }
                 }
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
                 j.idesc = instr_desc_bf16((int)j.n_blk, 128);
@@ -1030,6 +1195,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::trace_put(p.trace, ticket, 8, j.wait_a);
                     mafat_dev::trace_put(p.trace, ticket, 9, j.wait_b);
                 }
+                if (chain) {
+                    // chain item: the 3x3's accumulator goes to the epilogue, which writes its activated
+                    // bf16 result back into TMEM; the chained 1x1 then runs from there
+                    tc_commit_warp(ms.bar(kBarAccFull + buf));
+                    const ChainRec ch = recs[qs].chain;
+                    mbar_arrive_elect(ms.bar(kBarQEmpty + qs));  // the slot is no longer read
+                    const uint32_t mph = buf ? mid_ph1++ : mid_ph0++;
+                    mbar_wait_mma(ms.bar(kBarMidFull + buf), mph & 1u, p.ctr, pipe_limit, broken);
+                    tc_fence_after();
+                    mma_chain_1x1(ms, j.d_tmem, wu(ch.n2), wu(ch.nch2), wu(ch.kst2), wu(ch.swz2) != 0, wu(ch.bpp2),
+                                  wu(ch.np2), (uint32_t)wu(ch.blob2 * 2), wu(ch.a_col), wu(ch.out_col));
+                }
                 tc_commit_warp(ms.bar(kBarAccFull + buf));
                 ++acc_cnt;
             }
@@ -1055,9 +1232,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int ticket = q_items[qs];
                 int done_ctr = 0, extra_ctr = -1, flags = 0;
                 if (ticket >= 0) {
-                    done_ctr = recs[qs].done_ctr;
-                    extra_ctr = recs[qs].extra_ctr;
-                    flags = recs[qs].flags;
+                    done_ctr = recs[qs].epi.done_ctr;
+                    extra_ctr = recs[qs].epi.extra_ctr;
+                    flags = recs[qs].epi.flags;
                 }
                 mbar_arrive(bar(kBarQEmpty + qs));
                 ++q_cnt;
@@ -1147,6 +1324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Warp w reads TMEM lanes 32*(w%4) .. +31 (conv rows 4*(w%4) .. +3 of a block);
         // the two warpgroups (h = w/4) take units of one block x 32 columns in turn.
         uint32_t q_cnt = 0, acc_cnt = 0;
+        uint32_t full_ph0 = 0, full_ph1 = 0;  // AccFull phases consumed, per buffer (chain items take two)
         const int wq = warp & 3, h = warp >> 2;  // lane quarter, warpgroup
         const int r = wq * 4 + (lane >> 3);  // conv row within the block
         const int cc = lane & 7;             // conv column within the block
@@ -1155,59 +1333,81 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
             const int ticket = q_items[qs];
             EpiRec rc;
-            if (ticket >= 0) rc = recs[qs];
+            if (ticket >= 0) rc = recs[qs].epi;
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
             ++q_cnt;
             if (ticket < 0) break;
             const int buf = (int)(acc_cnt & 1u);
             // completes once the item's MMAs are done and its scale / bias have landed
-            mbar_wait(bar(kBarAccFull + buf), (acc_cnt >> 1) & 1u, p.ctr, pipe_limit, broken, 128);
+            mbar_wait(bar(kBarAccFull + buf), (buf ? full_ph1++ : full_ph0++) & 1u, p.ctr, pipe_limit, broken, 128);
             if (p.trace && threadIdx.x == 0) mafat_dev::trace_put(p.trace, ticket, 2, mafat_dev::globaltimer_ns());
             __syncwarp();
             tc_fence_after();
 
             const float* sc = reinterpret_cast<const float*>(smem + kOffSb + buf * kSbSlotBytes);
             const float* bi = sc + MAFAT_MAX_NBLK;
+            const uint32_t acc_lanes = tmem_base + ((uint32_t)(wq * 32) << 16) + (uint32_t)(buf * kAccStride);
             const int X = rc.x0 + cc;
-            const bool pool = (rc.flags & 1) != 0, nhwc = (rc.flags & 2) != 0;
-            // Work split between the warpgroups in units of one block x 32 output columns
-            // (16 when N is an odd multiple of 16), dealt round-robin.
-            const int uw = (rc.n_blk & 31) == 0 ? 32 : 16;
-            const int upb = uw == 32 ? rc.n_blk >> 5 : rc.n_blk >> 4;  // units per block
-            // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
-            for (int b = 0, qi = h;; qi += kEpiGroups) {
-                while (qi >= upb) {
-                    qi -= upb;
-                    ++b;
+            // A chain item takes two passes over the same unit loop: first the 3x3's accumulator
+            // (n_mid columns), activated and rounded as for a stored output, into TMEM at column
+            // a_col as the chained 1x1's A operand; then, once the 1x1's MMAs are done, its
+            // accumulator from column out_col, stored like any output.  Other items take the
+            // second pass only.
+            for (int pass = rc.chain ? 0 : 1; pass < 2; ++pass) {
+                const bool mid = pass == 0;
+                const int n_blk = mid ? rc.n_mid : rc.n_blk;
+                const uint32_t col0 = mid ? 0u : (rc.chain ? (uint32_t)rc.out_col : 0u);
+                const float* psc = sc + (rc.chain && !mid ? rc.n_mid : 0);
+                const float* pbi = bi + (rc.chain && !mid ? rc.n_mid : 0);
+                const bool pool = !mid && (rc.flags & 1) != 0, nhwc = !mid && (rc.flags & 2) != 0;
+                // Work split between the warpgroups in units of one block x 32 output columns
+                // (16 when N is an odd multiple of 16), dealt round-robin.
+                const int uw = (n_blk & 31) == 0 ? 32 : 16;
+                const int upb = uw == 32 ? n_blk >> 5 : n_blk >> 4;  // units per block
+                // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
+                for (int b = 0, qi = h;; qi += kEpiGroups) {
+                    while (qi >= upb) {
+                        qi -= upb;
+                        ++b;
+                    }
+                    if (b >= rc.nbk) break;
+                    const int q = qi * uw;
+                    const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
+                    const bool valid = (Y < rc.ylim) && (X < rc.xlim);
+                    // a pooled stage's conv region starts on even rows and columns and has even
+                    // extents, so a window's four lanes agree on valid
+                    int oy = Y, ox = X;
+                    if (pool) {
+                        oy = Y >> 1;
+                        ox = X >> 1;
+                    }
+                    const size_t pix = (size_t)(oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0);
+                    EpiDst dst;
+                    dst.out = rc.out;
+                    dst.nhwc = nhwc;
+                    dst.pix = nhwc ? pix * rc.cout : pix * 8;
+                    dst.plane = (size_t)rc.out_h * rc.out_w * 8;
+                    dst.cout = rc.cout;
+                    dst.store = valid;
+                    dst.pool = pool;
+                    dst.tmem = mid ? acc_lanes + (uint32_t)(rc.a_col + q / 2) : 0u;
+                    const uint32_t taddr = acc_lanes + col0 + (uint32_t)(b * n_blk + q);
+                    if (uw == 32)
+                        epi_chunk<32>(taddr, psc + q, pbi + q, rc.ch_base + q, dst, lane);
+                    else
+                        epi_chunk<16>(taddr, psc + q, pbi + q, rc.ch_base + q, dst, lane);
                 }
-                if (b >= rc.nbk) break;
-                const int q = qi * uw;
-                const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
-                const bool valid = (Y < rc.ylim) && (X < rc.xlim);
-                // a pooled stage's conv region starts on even rows and columns and has even
-                // extents, so a window's four lanes agree on valid
-                const bool store = valid;
-                int oy = Y, ox = X;
-                if (pool) {
-                    oy = Y >> 1;
-                    ox = X >> 1;
+                if (mid) {
+                    // hand the A operand to the MMA issuer, then wait for the 1x1's accumulator
+                    tmem_st_wait();
+                    tc_fence_before();
+                    mbar_arrive(bar(kBarMidFull + buf));
+                    mbar_wait(bar(kBarAccFull + buf), (buf ? full_ph1++ : full_ph0++) & 1u, p.ctr, pipe_limit, broken,
+                              64);
+                    __syncwarp();
+                    tc_fence_after();
                 }
-                const size_t pix = (size_t)(oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0);
-                EpiDst dst;
-                dst.out = rc.out;
-                dst.nhwc = nhwc;
-                dst.pix = nhwc ? pix * rc.cout : pix * 8;
-                dst.plane = (size_t)rc.out_h * rc.out_w * 8;
-                dst.cout = rc.cout;
-                dst.store = store;
-                dst.pool = pool;
-                const uint32_t taddr = tmem_base + ((uint32_t)(wq * 32) << 16) +
-                                       (uint32_t)(buf * kAccStride + b * rc.n_blk + q);
-                if (uw == 32)
-                    epi_chunk<32>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
-                else
-                    epi_chunk<16>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
             }
             tc_fence_before();
             mbar_arrive(bar(kBarAccEmpty + buf));  // also frees the scale / bias slot
@@ -1240,7 +1440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // stride 128 B, M / N stride 256 B), read through smem_desc as the kernel does.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(128, 1)
-    mafat_diag_umma_kernel(const __nv_bfloat16* a, const __nv_bfloat16* b, float* d, int n) {
+    mafat_diag_umma_kernel(const __nv_bfloat16* a, const __nv_bfloat16* b, float* d, int n, int a_tmem) {
     __shared__ __align__(1024) __nv_bfloat16 sa[128 * 16];
     __shared__ __align__(1024) __nv_bfloat16 sb[256 * 16];
     __shared__ __align__(8) uint64_t done_bar;
@@ -1262,7 +1462,7 @@ __global__ void __launch_bounds__(128, 1)
     if ((tid >> 5) == 0) {
         __syncwarp();  // thread 0 just left a branch of its own; .sync.aligned needs the warp converged
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
-                     "r"(256)
+                     "r"(512)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -1270,11 +1470,33 @@ __global__ void __launch_bounds__(128, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
-    if (tid == 0) {
-        const uint64_t adesc = smem_desc(smem_u32(sa), 128u, 256u);
+    const int warp0 = tid >> 5;
+    if (a_tmem) {
+        // row tid of A (lane tid) into TMEM columns 256..263, two bf16 per column
+        uint32_t v[16];
+        for (int i = 0; i < 8; ++i) {
+            const uint16_t lo = reinterpret_cast<const uint16_t*>(a)[tid * 16 + 2 * i];
+            const uint16_t hi = reinterpret_cast<const uint16_t*>(a)[tid * 16 + 2 * i + 1];
+            v[i] = (uint32_t)lo | ((uint32_t)hi << 16);
+        }
+        for (int i = 8; i < 16; ++i) v[i] = 0u;
+        tmem_st16(tmem + ((uint32_t)(warp0 * 32) << 16) + 256u, v);
+        tmem_st_wait();
+        tc_fence_before();
+    }
+    __syncthreads();
+    tc_fence_after();
+    if (warp0 == 0) {
+        // one converged warp issues (elect.sync inside the issue helpers)
         const uint64_t bdesc = smem_desc(smem_u32(sb), 128u, 256u);
-        mma_bf16(tmem, adesc, bdesc, instr_desc_bf16(n, 128), 0u);
-        tc_commit(smem_u32(&done_bar));
+        if (a_tmem) {
+            mma_tmem_a(tmem, tmem + 256u, (uint32_t)bdesc, (uint32_t)(bdesc >> 32), instr_desc_bf16(n, 128), 0u);
+        } else {
+            const uint64_t adesc = smem_desc(smem_u32(sa), 128u, 256u);
+            mma_lo(tmem, (uint32_t)adesc, (uint32_t)(adesc >> 32), (uint32_t)bdesc, (uint32_t)(bdesc >> 32),
+                   instr_desc_bf16(n, 128), 0u);
+        }
+        tc_commit_warp(smem_u32(&done_bar));
     }
     __syncwarp();
     // bounded wait (1 s) for the product
@@ -1298,7 +1520,7 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_after();
     if (warp == 0) {
         __syncwarp();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(256) : "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(512) : "memory");
     }
 }
 
@@ -1317,7 +1539,7 @@ cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, in
     return cudaGetLastError();
 }
 
-cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, cudaStream_t s) {
-    mafat_diag_umma_kernel<<<1, 128, 0, s>>>((const __nv_bfloat16*)a, (const __nv_bfloat16*)b, d, n);
+cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int a_tmem, cudaStream_t s) {
+    mafat_diag_umma_kernel<<<1, 128, 0, s>>>((const __nv_bfloat16*)a, (const __nv_bfloat16*)b, d, n, a_tmem);
     return cudaGetLastError();
 }

@@ -48,4 +48,4 @@ cudaError_t mafat_launch_fp32(const MafatKParams& p, int grid, cudaStream_t s);
 cudaError_t mafat_launch_to_planar(const void* nhwc, void* planar, int frames, int h, int w, int c, int c8,
                                    int elem_bytes, cudaStream_t s);
 // Diagnostic single-MMA kernel.
-cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, cudaStream_t s);
+cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int a_tmem, cudaStream_t s);

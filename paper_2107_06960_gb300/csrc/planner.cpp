@@ -345,12 +345,26 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // dominates.  Stages with more blocks than CTAs keep the widest block, which
             // reuses every A operand for the most output channels.
             const int cout_pad = (L.c_out + 15) / 16 * 16;
+            // On-chip chaining (tensor-core plans, halo recompute): a 3x3 convolution without a
+            // fused pool whose next layer is a 1x1 convolution of the same group runs both in one
+            // item when the 3x3's accumulator, its bf16 result and the 1x1's accumulator fit one
+            // 256-column TMEM buffer for a block of 128 pixels; the 1x1's stage has no tasks.
+            const bool prev_chain = !t.stages.empty() && t.stage_first[g] < (int)t.stages.size() &&
+                                    t.stages.back().chain;
+            bool chain_here = false;
+            if (cfg.dtype == 0 && !cfg.halo_reuse && !cfg.no_chain && !prev_chain && L.k == 3 && l + 1 <= last &&
+                net.layers[l + 1].type == L_CONV && net.layers[l + 1].k == 1) {
+                const int next_pad = (net.layers[l + 1].c_out + 15) / 16 * 16;
+                chain_here = cout_pad % 64 == 0 && cout_pad + cout_pad / 2 + next_pad <= 256;
+            }
             // With several frames in flight the SMs are kept busy by the next frame anyway, and a
             // 1x1 layer's item reads a whole K = c_in halo for few MMAs: there the narrowest block
             // considered is 128 (608x608, 16 frames: 81.3 against 83.0 us per frame; at one frame
             // the extra parallelism of N = 64 wins, 117.4 against 121.5 us).
             const int min_nb = (cfg.batch > 1 && L.k == 1) ? 128 : 64;
-            if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
+            if (chain_here || prev_chain) {
+                s.n_blk = cout_pad;  // every channel of the pixels in one item
+            } else if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
                 s.n_blk = cfg.fixed_nblk;
             } else {
                 s.n_blk = largest_nblk(cout_pad);
@@ -366,7 +380,9 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // Blocks per item (stacked along rows, one accumulator each, sharing every
             // weight blob): grow while the stage keeps at least one item per CTA.
             s.mb = 1;
-            if (cfg.fixed_mb > 0) {
+            if (chain_here || prev_chain) {
+                // one 128-pixel block per item: the chained pair's three TMEM regions fill a buffer
+            } else if (cfg.fixed_mb > 0) {
                 s.mb = cfg.fixed_mb;
             } else {
                 while (s.mb * 2 * s.n_blk <= 256 && blocks * s.n_nblk / (s.mb * 2) >= n_ctas) s.mb *= 2;
@@ -396,7 +412,20 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             for (;;) {
                 s.rows_box = MAFAT_BLK_ROWS * s.mb + L.k - 1;
                 const int row_bytes = s.cols_box * 16 * s.rows_box;
-                if (s.in_mode == MAFAT_IN_GATHER) {
+                if (s.chain) {
+            const size_t si = (size_t)(&s - t.stages.data());
+            if (si + 1 >= t.stages.size() || !t.stages[si + 1].chained || t.stages[si + 1].k != 1 || s.k != 3 ||
+                s.pool)
+                return "a chain stage must be a 3x3 convolution followed by its chained 1x1";
+            const MafatStageDev& s2 = t.stages[si + 1];
+            if (s.n_nblk != 1 || s2.n_nblk != 1 || s.mb != 1 || s2.cin != s.cout || s.n_blk % 64 != 0)
+                return "chained stages need every channel of one 128-pixel block in one item";
+            if (s.chain_a_col != s.n_blk || s.chain_out_col != s.n_blk + s.n_blk / 2 ||
+                s.chain_out_col + s2.n_blk > 256)
+                return "chained stages exceed one TMEM accumulator buffer";
+        }
+        if (s.chained && (&s == t.stages.data() || !(&s - 1)->chain)) return "a chained stage without its chain stage";
+        if (s.in_mode == MAFAT_IN_GATHER) {
                     // the expanded halo plus the raw rows it is built from share the stage
                     s.chunk8 = 1;
                     if (mafat_raw_offset(s.rows_box, s.cols_box) + s.rows_box * s.raw_e * 2 <= MAFAT_A_STAGE_BYTES ||
@@ -452,6 +481,12 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             t.weight32_elems += (int64_t)L.c_out * L.c_in * L.k * L.k;
             s.sb_off = (int)t.sb_elems;
             t.sb_elems += cout_pad;
+            s.chain = chain_here ? 1 : 0;
+            s.chained = prev_chain ? 1 : 0;
+            if (chain_here) {
+                s.chain_a_col = cout_pad;
+                s.chain_out_col = cout_pad + cout_pad / 2;
+            }
             t.stages.push_back(s);
             stage_pool_layer.push_back(s.pool ? l + 1 : -1);
             if (s.pool) ++l;
@@ -590,10 +625,15 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             for (size_t w0 = 0; w0 < tl.size(); w0 += W) {
                 size_t w1 = std::min(tl.size(), w0 + (size_t)W);
                 std::vector<int> prev_of_tile(w1 - w0, -1);
+                int rel = -1;  // index of the stage among the group's stages that have tasks
                 for (int s = t.stage_first[g]; s <= t.stage_last[g]; ++s) {
                     const MafatStageDev& st = t.stages[s];
+                    if (st.chained) continue;  // runs inside the items of the chain stage before it
+                    ++rel;
+                    // the stage whose output this task writes: its own, or the chained 1x1's
+                    const int s_out = st.chain ? s + 1 : s;
                     const Layer& Lc = net.layers[st.layer];
-                    const std::vector<int> prev_stage_task = prev_of_tile;  // stage s - 1's task of each tile
+                    const std::vector<int> prev_stage_task = prev_of_tile;  // previous task stage of each tile
                     for (size_t q = w0; q < w1; ++q) {
                         const TileInfo& ti = tl[q];
                         int tseq = seq + (int)(q - w0);
@@ -603,9 +643,11 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         tk.frame = f;
                         const Rect& cr = ti.outs[st.layer];
                         const Rect& ir = ti.ins[st.layer];
-                        int ol = stage_pool_layer[s] >= 0 ? stage_pool_layer[s] : st.layer;
+                        int ol = stage_pool_layer[s_out] >= 0 ? stage_pool_layer[s_out] : t.stages[s_out].layer;
                         const Rect& orr = ti.outs[ol];
-                        if (st.pool) {
+                        if (st.chain && !(ti.outs[t.stages[s_out].layer] == cr))
+                            return "internal: chained 1x1 region differs from its 3x3";
+                        if (t.stages[s_out].pool) {
                             // the conv region of a pooled stage is exactly twice the pooled region
                             if (!(cr.y0 == 2 * orr.y0 && cr.y1 == 2 * orr.y1 && cr.x0 == 2 * orr.x0 &&
                                   cr.x1 == 2 * orr.x1))
@@ -617,7 +659,6 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         tk.cw = cr.w();
                         tk.nby = ceil_div(tk.ch, MAFAT_BLK_ROWS);
                         tk.nbx = ceil_div(tk.cw, MAFAT_BLK_COLS);
-                        int rel = s - t.stage_first[g];
                         if (s == t.stage_first[g]) {
                             tk.in_kind = g == 0 ? MAFAT_BUF_USER_IN : g == 1 ? MAFAT_BUF_CUT : MAFAT_BUF_MAP;
                             tk.in_tmap = g >= 2 ? stage_tmap[s] : -1;
@@ -655,7 +696,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             tk.in_tmap = (int)t.tmaps.size();
                             t.tmaps.push_back(req);
                         }
-                        if (s == t.stage_last[g]) {
+                        if (s_out == t.stage_last[g]) {
                             if (g == G - 1) {
                                 tk.out_kind = MAFAT_BUF_USER_OUT;
                                 tk.out_nhwc = 1;
@@ -720,15 +761,18 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         } else {
                             d.prev_task = prev_of_tile[qi];
                         }
-                        if (g + 1 < G && s == t.stage_last[g]) d.bump_ctr = f * (G - 1) + g;
+                        if (g + 1 < G && s_out == t.stage_last[g]) d.bump_ctr = f * (G - 1) + g;
                         prev_of_tile[qi] = (int)t.tasks.size();
                         t.tasks.push_back(tk);
                         deps.push_back(d);
-                        // statistics
-                        double kk = (double)Lc.k * Lc.k;
-                        t.executed_flops += 2.0 * cr.h() * cr.w() * (double)st.cout * st.cin * kk;
-                        t.issued_flops += 2.0 * tk.nby * tk.nbx * (double)(MAFAT_BLK_ROWS * MAFAT_BLK_COLS) *
-                                          (double)st.n_nblk * st.n_blk * st.n_chunks * st.n_bsteps * st.kst * 16.0;
+                        // statistics (a chain task does the work of both of its stages)
+                        for (int sx = s; sx <= s_out; ++sx) {
+                            const MafatStageDev& sw = t.stages[sx];
+                            const double kk = (double)sw.k * sw.k;
+                            t.executed_flops += 2.0 * cr.h() * cr.w() * (double)sw.cout * sw.cin * kk;
+                            t.issued_flops += 2.0 * tk.nby * tk.nbx * (double)(MAFAT_BLK_ROWS * MAFAT_BLK_COLS) *
+                                              (double)sw.n_nblk * sw.n_blk * sw.n_chunks * sw.n_bsteps * sw.kst * 16.0;
+                        }
                     }
                 }
                 for (size_t q = w0; q < w1; ++q) last_task_of_seq.push_back(prev_of_tile[q - w0]);
@@ -948,7 +992,9 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
     for (int ti = 0; ti < n_tasks; ++ti) {
         const MafatTaskDev& k = t.tasks[ti];
         const MafatStageDev& s = t.stages[k.stage];
+        const MafatStageDev& so = s.chain ? t.stages[k.stage + 1] : s;  // the stage whose output it writes
         const Layer& L = net.layers[s.layer];
+        if (s.chained) return "a chained stage has a task";
         if (last_item[ti] - first_item[ti] + 1 != k.n_items) return "task items not contiguous";
         // input buffer extent and coverage of every in-map tap of the conv rectangle
         const int64_t in_elems = k.in_kind == MAFAT_BUF_USER_IN ? (int64_t)s.cin * k.in_h * k.in_w
@@ -970,14 +1016,14 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         }
         // output extent of the valid pixels
         int oy0 = k.cy0, oy1 = k.cy0 + k.ch, ox0 = k.cx0, ox1 = k.cx0 + k.cw;
-        if (s.pool) {
+        if (so.pool) {
             if (k.cy0 % 2 || k.ch % 2 || k.cx0 % 2 || k.cw % 2) return "pooled rectangle not quad aligned";
             oy0 /= 2; oy1 /= 2; ox0 /= 2; ox1 /= 2;
         }
         if (oy0 < k.out_y0 || ox0 < k.out_x0 || oy1 > k.out_y0 + k.out_h || ox1 > k.out_x0 + k.out_w)
             return "output rectangle outside its buffer";
-        int64_t out_elems = k.out_nhwc ? (int64_t)k.out_h * k.out_w * s.cout
-                                       : (int64_t)((s.cout + 7) / 8) * 8 * k.out_h * k.out_w;
+        int64_t out_elems = k.out_nhwc ? (int64_t)k.out_h * k.out_w * so.cout
+                                       : (int64_t)((so.cout + 7) / 8) * 8 * k.out_h * k.out_w;
         if (k.out_off < 0 || k.out_off + out_elems > buf_total(k.out_kind)) return "output buffer outside its allocation";
         if (k.out_kind == MAFAT_BUF_SCRATCH && out_elems > t.slot_buf_elems) return "scratch output above buffer size";
         if (k.done_ctr < MAFAT_CTR_BASE || k.done_ctr >= MAFAT_CTR_BASE + t.n_counters) return "bad done counter";

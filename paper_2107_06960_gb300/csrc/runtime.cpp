@@ -376,6 +376,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.lookahead_items = o.lookahead_items;
     cfg.halo_reuse = o.halo_reuse != 0;
     cfg.frame_major = o.frame_major != 0;
+    cfg.no_chain = o.no_chain != 0;
     if (o.tile_bounds) {
         // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
         const int32_t* b = o.tile_bounds;
@@ -804,10 +805,11 @@ void mafat_plan_destroy(mafat_plan_t* plan) {
 
 void mafat_net_destroy(mafat_net_t* net) { delete net; }
 
-mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, void* stream) {
+mafat_status mafat_diag_umma(const void* a_dev, const void* b_dev, float* d_dev, int32_t n, int32_t a_in_tmem,
+                             void* stream) {
     if (!a_dev || !b_dev || !d_dev) return fail(MAFAT_EINVAL, "null argument");
     if (n < 16 || n > 256 || n % 16 != 0) return fail(MAFAT_EINVAL, "n must be a multiple of 16 in 16..256");
-    cudaError_t e = mafat_launch_diag_umma(a_dev, b_dev, d_dev, n, (cudaStream_t)stream);
+    cudaError_t e = mafat_launch_diag_umma(a_dev, b_dev, d_dev, n, a_in_tmem ? 1 : 0, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "diag launch");
     e = cudaStreamSynchronize((cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "diag sync");

@@ -378,6 +378,46 @@ def test_measured_search_picks_the_fastest_timed_plan(mf):
 
 
 # ---------------------------------------------------------------------------
+# On-chip chaining of a 3x3 and the 1x1 after it (the 3x3's output stays in TMEM)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("cut,grids", [(8, [(3, 3), (2, 2)]), (6, [(2, 2), (2, 1)]), (None, [(3, 2)])])
+def test_bf16_chained_pair_matches_unchained_and_oracle(mf, cut, grids):
+    # YOLOv2 layers 4 -> 5 chained; with the cut after layer 5 the chained 1x1 writes the cut tensor
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 61, "bf16")
+    x = synth.make_input(2, 96, 96, 3, 62, "bf16")
+    c1, o1 = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
+    c0, o0 = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=dict(no_chain=True))
+    assert np.array_equal(o1, o0)
+    if cut is not None:
+        assert np.array_equal(c1, c0)
+    _check_groups(c1, o1, _oracle_groups(layers, params, x, cut), cut, TOL_BF16)
+
+
+@pytest.mark.parametrize("layers", [
+    [("conv", 3, 1, 1, 64), ("conv", 1, 1, 0, 32)],                        # chained 1x1 writes the output
+    [("conv", 3, 1, 1, 64), ("conv", 1, 1, 0, 32), ("max", 2, 2, 0, 0)],   # ... through a fused max-pool
+    [("conv", 3, 1, 1, 64), ("conv", 1, 1, 0, 48), ("conv", 3, 1, 1, 64), ("conv", 1, 1, 0, 16)],
+])
+def test_bf16_chained_pair_small_networks(mf, layers):
+    params = synth.make_params(layers, 16, 63, "bf16")
+    x = synth.make_input(2, 40, 48, 16, 64, "bf16")
+    _, o1 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16)
+    _, o0 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16, plan_kwargs=dict(no_chain=True))
+    assert np.array_equal(o1, o0)
+    _check_groups(None, o1, _oracle_groups(layers, params, x, None), None, TOL_BF16)
+
+
+def test_bf16_608_chained_matches_unchained(mf):
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    c1, o1 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16)
+    c0, o0 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16,
+                      plan_kwargs=dict(no_chain=True))
+    assert np.array_equal(o1, o0) and np.array_equal(c1, c0)
+
+
+# ---------------------------------------------------------------------------
 # Run paths: host buffers, CUDA graphs, repeated runs
 # ---------------------------------------------------------------------------
 
