@@ -7,8 +7,8 @@ tiled 5x5 and group 2 tiled 2x2.  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl mafat|reference] [--workload NAME]
 
---impl reference times the fp64 CPU oracle on the host cores (the only other
-place this script runs oracle code, together with the cpu_baseline leg).
+--impl reference times the CPU oracle (its plain fp32 build) on the host cores (the
+only other place this script runs oracle code, together with the cpu_baseline leg).
 Under torchrun (N > 1) every rank runs an independent replica on its own GPU
 (the method does not shard a frame across devices); rank 0 reports the frames
 of all ranks over the slowest rank's time.
@@ -147,19 +147,46 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
-def cpu_oracle_rate(wl, budget_s=12.0):
-    """The oracle as it stands (fp64, OpenMP over rows) on the host cores: frames/s on whole frames."""
-    import oracle
-    x = wl["input"][0]
-    n, t0 = 0, time.perf_counter()
-    while True:
-        oracle.forward(wl["layers"], wl["params"], x)
-        n += 1
+def _best_of(n, fn):
+    best = None
+    for _ in range(n):
+        t0 = time.perf_counter()
+        fn()
         el = time.perf_counter() - t0
-        if el >= budget_s or n >= 8:
-            break
-    return n / el, oracle.num_threads(), "%d whole %dx%d frame(s), unfused fp64 forward of all %d layers" % (
-        n, wl["h"], wl["w"], len(wl["layers"]))
+        best = el if best is None else min(best, el)
+    return best
+
+
+def cpu_oracle_timings(wl_names=(DEFAULT_WORKLOAD, "yolo16_416_1x3x3"), best_of=3):
+    """The oracle as it stands, in its plain fp32 build (the same loops as the fp64 parity
+    oracle, single precision), on the host cores: for each workload, single-threaded and
+    with every core (OpenMP over output rows), best of `best_of` wall-clock runs.  All-core
+    runs time whole frames; single-threaded runs time a centre crop of 1/16 of the frame's
+    pixels and scale by the crop's share of the frame's FLOPs (the work per pixel is the
+    same everywhere but at the image border)."""
+    import oracle
+    cores = os.cpu_count() or 1
+    rows = []
+    for name in wl_names:
+        w = synth.workload(name)
+        layers, params, x = w["layers"], w["params"], w["input"][0]
+        full = oracle.conv_flops(layers, oracle.layer_shapes(layers, w["h"], w["w"], 3))
+        side = w["h"] // 4
+        y0 = (w["h"] - side) // 2
+        crop = x[y0:y0 + side, y0:y0 + side]
+        frac = oracle.conv_flops(layers, oracle.layer_shapes(layers, side, side, 3)) / full
+        for threads in (1, cores):
+            oracle.set_num_threads(threads, "f32")
+            if threads == 1:
+                t = _best_of(best_of, lambda: oracle.forward(layers, params, crop, precision="f32")) / frac
+                sample = "%dx%d centre crop (%.4f of a frame's FLOPs), scaled" % (side, side, frac)
+            else:
+                t = _best_of(best_of, lambda: oracle.forward(layers, params, x, precision="f32"))
+                sample = "whole %dx%d frame" % (w["h"], w["w"])
+            rows.append({"workload": name, "threads": threads, "s_per_frame": t, "frames_per_s": 1.0 / t,
+                         "gflop_per_s": full / t / 1e9, "sample": sample})
+    oracle.set_num_threads(cores, "f32")
+    return rows, cores
 
 
 def run_reference(args, wl):
@@ -170,9 +197,11 @@ def run_reference(args, wl):
         return
     layers, params = wl["layers"], wl["params"]
     full = oracle.conv_flops(layers, oracle.layer_shapes(layers, wl["h"], wl["w"], 3))
+    cores = os.cpu_count() or 1
+    oracle.set_num_threads(cores, "f32")
     # size the per-step sample so the whole run stays within about two minutes
     t0 = time.perf_counter()
-    oracle.forward(layers, params, wl["input"][0][:152, :152])
+    oracle.forward(layers, params, wl["input"][0][:152, :152], precision="f32")
     t_small = time.perf_counter() - t0
     est_full = t_small * (wl["h"] * wl["w"]) / (152 * 152)
     steps = args.steps + args.warmup
@@ -183,19 +212,20 @@ def run_reference(args, wl):
     x = wl["input"][0][:side, :side]
     frac = oracle.conv_flops(layers, oracle.layer_shapes(layers, side, side, 3)) / full
     for _ in range(args.warmup):
-        oracle.forward(layers, params, x)
+        oracle.forward(layers, params, x, precision="f32")
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        oracle.forward(layers, params, x)
+        oracle.forward(layers, params, x, precision="f32")
     el = time.perf_counter() - t0
     value = frac * args.steps / el
-    sample = "%dx%d crop per step (%.4f of a frame's FLOPs), unfused fp64 forward" % (side, side, frac)
+    sample = "%dx%d crop per step (%.4f of a frame's FLOPs), unfused forward, the oracle's fp32 build" % (
+        side, side, frac)
     line = {
         "impl": "reference", "metric": metric_of(args.workload), "value": value, "unit": "frames/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": args.workload, "input": "%dx%dx3" % (wl["h"], wl["w"]), "batch": wl["batch"]},
-        "cpu_baseline": {"value": value, "unit": "frames/s", "cores": oracle.num_threads(), "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "frames/s", "cores": oracle.num_threads("f32"), "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "frames/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -448,8 +478,13 @@ def main():
 
     cpu = None
     if not args.no_cpu_baseline:
-        v, cores, sample = cpu_oracle_rate(wl)
-        cpu = {"value": v, "unit": "frames/s", "cores": cores, "kind": "oracle", "sample": sample}
+        names = [args.workload] + (["yolo16_416_1x3x3"] if args.workload == DEFAULT_WORKLOAD else [])
+        rows, cores = cpu_oracle_timings(names)
+        head = next(r for r in rows if r["workload"] == args.workload and r["threads"] == cores)
+        cpu = {"value": head["frames_per_s"], "unit": "frames/s", "cores": cores, "kind": "oracle",
+               "precision": "f32 (the oracle's loops built in single precision; parity uses its fp64 build)",
+               "sample": "%s, all %d host cores, best of 3" % (head["sample"], cores),
+               "timings": rows}
 
     line = {
         "metric": metric_of(args.workload), "value": value, "unit": "frames/s", "n_gpus": ws, "steps": args.steps,

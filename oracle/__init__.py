@@ -15,7 +15,9 @@ Contents, each following the paper (MAFAT, arXiv 2107.06960):
                            group (Sec. 4.1, FTP of Sec. 3).
 * ``predict_layer_group`` / ``predict_mem`` -- the memory predictor (Algorithm 1).
 * ``get_config``        -- the configuration search (Algorithm 2).
-* ``forward``           -- layer-by-layer fp64 forward (the plain definition).
+* ``forward``           -- layer-by-layer fp64 forward (the plain definition); the
+                           same loops in fp32 (``precision="f32"``) are the timed CPU
+                           baseline.
 * ``forward_tiled``     -- the same network executed as fused tiles of its layer
                            groups, merged and re-tiled at every cut (Sec. 4).
 
@@ -30,7 +32,7 @@ import os
 
 import numpy as np
 
-from .build import LIB, build_oracle
+from .build import LIB, LIB_F32, build_oracle
 
 CONV = "conv"
 MAX = "max"
@@ -38,35 +40,45 @@ LEAKY_SLOPE = 0.1
 BIAS_MIB = 31.0          # Sec. 4.1: constant bias term of 31 MB
 BYTES_PER_ELEM = 4       # fp32 elements (Darknet); pinned by the 100 MB / 135 MB figures of Sec. 2
 
-_lib = None
+_libs = {}
+_CT = {"f64": (ctypes.c_double, np.float64), "f32": (ctypes.c_float, np.float32)}
 
 
-def _load():
-    global _lib
-    if _lib is None:
-        path = build_oracle()
-        lib = ctypes.CDLL(path)
-        dp = ctypes.POINTER(ctypes.c_double)
+def _load(precision="f64"):
+    """The oracle's C library: "f64" (the parity oracle) or "f32" (the same loops in
+    single precision, the CPU baseline the benchmark times)."""
+    if precision not in _libs:
+        build_oracle()
+        lib = ctypes.CDLL(LIB if precision == "f64" else LIB_F32)
+        real = _CT[precision][0]
+        dp = ctypes.POINTER(real)
         i = ctypes.c_int
-        lib.oracle_conv_full.argtypes = [dp, i, i, i, dp, i, i, i, i, dp, dp, ctypes.c_double, dp]
+        lib.oracle_conv_full.argtypes = [dp, i, i, i, dp, i, i, i, i, dp, dp, real, dp]
         lib.oracle_maxpool_full.argtypes = [dp, i, i, i, i, i, dp]
         lib.oracle_conv_region.argtypes = [dp, i, i, i, i, i, i, i, dp, i, i, i, i, dp, dp,
-                                           ctypes.c_double, i, i, i, i, dp]
+                                           real, i, i, i, i, dp]
         lib.oracle_maxpool_region.argtypes = [dp, i, i, i, i, i, i, i, i, i, i, i, i, i, dp]
         for f in (lib.oracle_conv_full, lib.oracle_maxpool_full, lib.oracle_conv_region,
                   lib.oracle_maxpool_region):
             f.restype = ctypes.c_int
         lib.oracle_num_threads.restype = ctypes.c_int
-        _lib = lib
-    return _lib
+        lib.oracle_set_num_threads.argtypes = [i]
+        lib.oracle_set_num_threads.restype = None
+        _libs[precision] = lib
+    return _libs[precision]
 
 
 def _dp(a):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
 
 
-def num_threads():
-    return _load().oracle_num_threads()
+def num_threads(precision="f64"):
+    return _load(precision).oracle_num_threads()
+
+
+def set_num_threads(n, precision="f64"):
+    """OpenMP threads of the oracle's loops (n >= 1)."""
+    _load(precision).oracle_set_num_threads(int(n))
 
 
 # ---------------------------------------------------------------------------
@@ -235,47 +247,56 @@ def get_config(layers, shapes, limit_mib, predictor=None, cuts=None, tiles=(1, 2
 # Forward passes (fp64)
 # ---------------------------------------------------------------------------
 
-def _conv_full(x, prm, k, s, p):
+def _ptr(a, precision):
+    return a.ctypes.data_as(ctypes.POINTER(_CT[precision][0]))
+
+
+def _conv_full(x, prm, k, s, p, precision="f64"):
     w, scale, bias = prm
     H, W, C = x.shape
     Cout = w.shape[0]
     Ho, Wo = (H + 2 * p - k) // s + 1, (W + 2 * p - k) // s + 1
-    out = np.empty((Ho, Wo, Cout), dtype=np.float64)
-    xx = np.ascontiguousarray(x, dtype=np.float64)
-    ww = np.ascontiguousarray(w, dtype=np.float64)
-    sc = np.ascontiguousarray(scale, dtype=np.float64)
-    bi = np.ascontiguousarray(bias, dtype=np.float64)
-    rc = _load().oracle_conv_full(_dp(xx), H, W, C, _dp(ww), Cout, k, s, p, _dp(sc), _dp(bi),
-                                  LEAKY_SLOPE, _dp(out))
+    dt = _CT[precision][1]
+    out = np.empty((Ho, Wo, Cout), dtype=dt)
+    xx = np.ascontiguousarray(x, dtype=dt)
+    ww = np.ascontiguousarray(w, dtype=dt)
+    sc = np.ascontiguousarray(scale, dtype=dt)
+    bi = np.ascontiguousarray(bias, dtype=dt)
+    q = lambda a: _ptr(a, precision)
+    rc = _load(precision).oracle_conv_full(q(xx), H, W, C, q(ww), Cout, k, s, p, q(sc), q(bi),
+                                           LEAKY_SLOPE, q(out))
     if rc != 0:
         raise ValueError("oracle_conv_full: bad sizes")
     return out
 
 
-def _pool_full(x, k, s):
+def _pool_full(x, k, s, precision="f64"):
     H, W, C = x.shape
     Ho, Wo = (H - k) // s + 1, (W - k) // s + 1
-    out = np.empty((Ho, Wo, C), dtype=np.float64)
-    xx = np.ascontiguousarray(x, dtype=np.float64)
-    if _load().oracle_maxpool_full(_dp(xx), H, W, C, k, s, _dp(out)) != 0:
+    dt = _CT[precision][1]
+    out = np.empty((Ho, Wo, C), dtype=dt)
+    xx = np.ascontiguousarray(x, dtype=dt)
+    if _load(precision).oracle_maxpool_full(_ptr(xx, precision), H, W, C, k, s, _ptr(out, precision)) != 0:
         raise ValueError("oracle_maxpool_full: bad sizes")
     return out
 
 
-def apply_layer(layer, prm, x):
-    """One layer on a full HWC map (fp64)."""
+def apply_layer(layer, prm, x, precision="f64"):
+    """One layer on a full HWC map (fp64, or fp32 with precision="f32")."""
     t, k, s, p, f = layer
     if t == CONV:
-        return _conv_full(x, prm, k, s, p)
-    return _pool_full(x, k, s)
+        return _conv_full(x, prm, k, s, p, precision)
+    return _pool_full(x, k, s, precision)
 
 
-def forward(layers, params, x):
-    """Layer-by-layer forward of one HWC image; returns the list of every layer's output."""
+def forward(layers, params, x, precision="f64"):
+    """Layer-by-layer forward of one HWC image; returns the list of every layer's output.
+    precision="f32" runs the same loops in single precision (every sum and every layer
+    output in fp32): the plain fp32 forward used as the timed CPU baseline."""
     outs = []
-    cur = np.asarray(x, dtype=np.float64)
+    cur = np.asarray(x, dtype=_CT[precision][1])
     for layer, prm in zip(layers, params):
-        cur = apply_layer(layer, prm, cur)
+        cur = apply_layer(layer, prm, cur, precision)
         outs.append(cur)
     return outs
 

@@ -8,7 +8,8 @@
  * (Sec. 2, Sec. 4): a convolution layer followed by folded batch-norm and
  * leaky ReLU, and a max-pool layer.  Feature maps are HWC (channels
  * innermost), weights are [Cout][Cin][k][k] (cross-correlation, as in every
- * CNN framework), everything in double precision:
+ * CNN framework), everything in double precision (single precision in the
+ * fp32 build, see ORACLE_REAL below):
  *
  *   acc[y][x][o] = sum_{c, ky, kx} w[o][c][ky][kx] * in[y*s+ky-p][x*s+kx-p][c]
  *                  (input outside the map counts as 0)
@@ -32,13 +33,21 @@
  */
 #include <stddef.h>
 
+/* Arithmetic type: double (the parity oracle), or float when built with
+ * -DORACLE_REAL=float (the plain fp32 forward the method statement names, built
+ * as a second library and used only to time the CPU baseline; the same loops). */
+#ifndef ORACLE_REAL
+#define ORACLE_REAL double
+#endif
+typedef ORACLE_REAL real_t;
+
 #define IDX3(y, x, c, W, C) ((((size_t)(y)) * (size_t)(W) + (size_t)(x)) * (size_t)(C) + (size_t)(c))
 
 /* Full-map convolution + folded BN + leaky ReLU.  Returns 0, or -1 on bad sizes. */
-int oracle_conv_full(const double* in, int H, int W, int Cin,
-                     const double* w, int Cout, int k, int stride, int pad,
-                     const double* scale, const double* bias, double slope,
-                     double* out)
+int oracle_conv_full(const real_t* in, int H, int W, int Cin,
+                     const real_t* w, int Cout, int k, int stride, int pad,
+                     const real_t* scale, const real_t* bias, real_t slope,
+                     real_t* out)
 {
     if (H <= 0 || W <= 0 || Cin <= 0 || Cout <= 0 || k <= 0 || stride <= 0 || pad < 0) return -1;
     int Ho = (H + 2 * pad - k) / stride + 1;
@@ -48,7 +57,7 @@ int oracle_conv_full(const double* in, int H, int W, int Cin,
     for (int y = 0; y < Ho; ++y) {
         for (int x = 0; x < Wo; ++x) {
             for (int o = 0; o < Cout; ++o) {
-                double acc = 0.0;
+                real_t acc = 0.0;
                 for (int c = 0; c < Cin; ++c) {
                     for (int ky = 0; ky < k; ++ky) {
                         int iy = y * stride + ky - pad;
@@ -56,12 +65,12 @@ int oracle_conv_full(const double* in, int H, int W, int Cin,
                         for (int kx = 0; kx < k; ++kx) {
                             int ix = x * stride + kx - pad;
                             if (ix < 0 || ix >= W) continue;
-                            double wv = w[(((size_t)o * Cin + c) * k + ky) * k + kx];
+                            real_t wv = w[(((size_t)o * Cin + c) * k + ky) * k + kx];
                             acc += wv * in[IDX3(iy, ix, c, W, Cin)];
                         }
                     }
                 }
-                double z = scale[o] * acc + bias[o];
+                real_t z = scale[o] * acc + bias[o];
                 out[IDX3(y, x, o, Wo, Cout)] = z > 0.0 ? z : slope * z;
             }
         }
@@ -70,7 +79,7 @@ int oracle_conv_full(const double* in, int H, int W, int Cin,
 }
 
 /* Full-map max-pool (no padding).  Returns 0, or -1 on bad sizes. */
-int oracle_maxpool_full(const double* in, int H, int W, int C, int k, int stride, double* out)
+int oracle_maxpool_full(const real_t* in, int H, int W, int C, int k, int stride, real_t* out)
 {
     if (H <= 0 || W <= 0 || C <= 0 || k <= 0 || stride <= 0 || H < k || W < k) return -1;
     int Ho = (H - k) / stride + 1;
@@ -79,10 +88,10 @@ int oracle_maxpool_full(const double* in, int H, int W, int C, int k, int stride
     for (int y = 0; y < Ho; ++y)
         for (int x = 0; x < Wo; ++x)
             for (int c = 0; c < C; ++c) {
-                double m = in[IDX3(y * stride, x * stride, c, W, C)];
+                real_t m = in[IDX3(y * stride, x * stride, c, W, C)];
                 for (int dy = 0; dy < k; ++dy)
                     for (int dx = 0; dx < k; ++dx) {
-                        double v = in[IDX3(y * stride + dy, x * stride + dx, c, W, C)];
+                        real_t v = in[IDX3(y * stride + dy, x * stride + dx, c, W, C)];
                         if (v > m) m = v;
                     }
                 out[IDX3(y, x, c, Wo, C)] = m;
@@ -97,11 +106,11 @@ int oracle_maxpool_full(const double* in, int H, int W, int C, int k, int stride
  * Output buffer is out[oh][ow][Cout].  Returns 0, or -1 if a needed in-map
  * input pixel is missing from the region (or on bad sizes).
  */
-int oracle_conv_region(const double* in, int iy0, int ix0, int ih, int iw,
+int oracle_conv_region(const real_t* in, int iy0, int ix0, int ih, int iw,
                        int mh, int mw, int Cin,
-                       const double* w, int Cout, int k, int stride, int pad,
-                       const double* scale, const double* bias, double slope,
-                       int oy0, int ox0, int oh, int ow, double* out)
+                       const real_t* w, int Cout, int k, int stride, int pad,
+                       const real_t* scale, const real_t* bias, real_t slope,
+                       int oy0, int ox0, int oh, int ow, real_t* out)
 {
     if (ih < 0 || iw < 0 || oh < 0 || ow < 0 || Cin <= 0 || Cout <= 0 || k <= 0 || stride <= 0) return -1;
     /* Check first that every needed in-map pixel is in the region. */
@@ -123,7 +132,7 @@ int oracle_conv_region(const double* in, int iy0, int ix0, int ih, int iw,
         for (int xx = 0; xx < ow; ++xx) {
             int x = ox0 + xx;
             for (int o = 0; o < Cout; ++o) {
-                double acc = 0.0;
+                real_t acc = 0.0;
                 for (int c = 0; c < Cin; ++c) {
                     for (int ky = 0; ky < k; ++ky) {
                         int my = y * stride + ky - pad;
@@ -131,12 +140,12 @@ int oracle_conv_region(const double* in, int iy0, int ix0, int ih, int iw,
                         for (int kx = 0; kx < k; ++kx) {
                             int mx = x * stride + kx - pad;
                             if (mx < 0 || mx >= mw) continue;
-                            double wv = w[(((size_t)o * Cin + c) * k + ky) * k + kx];
+                            real_t wv = w[(((size_t)o * Cin + c) * k + ky) * k + kx];
                             acc += wv * in[IDX3(my - iy0, mx - ix0, c, iw, Cin)];
                         }
                     }
                 }
-                double z = scale[o] * acc + bias[o];
+                real_t z = scale[o] * acc + bias[o];
                 out[IDX3(yy, xx, o, ow, Cout)] = z > 0.0 ? z : slope * z;
             }
         }
@@ -145,9 +154,9 @@ int oracle_conv_region(const double* in, int iy0, int ix0, int ih, int iw,
 }
 
 /* Max-pool evaluated on an output rectangle from an input region buffer (as above). */
-int oracle_maxpool_region(const double* in, int iy0, int ix0, int ih, int iw,
+int oracle_maxpool_region(const real_t* in, int iy0, int ix0, int ih, int iw,
                           int mh, int mw, int C, int k, int stride,
-                          int oy0, int ox0, int oh, int ow, double* out)
+                          int oy0, int ox0, int oh, int ow, real_t* out)
 {
     if (ih < 0 || iw < 0 || oh < 0 || ow < 0 || C <= 0 || k <= 0 || stride <= 0) return -1;
     for (int y = oy0; y < oy0 + oh; ++y)
@@ -164,10 +173,10 @@ int oracle_maxpool_region(const double* in, int iy0, int ix0, int ih, int iw,
         for (int xx = 0; xx < ow; ++xx)
             for (int c = 0; c < C; ++c) {
                 int by = (oy0 + yy) * stride - iy0, bx = (ox0 + xx) * stride - ix0;
-                double m = in[IDX3(by, bx, c, iw, C)];
+                real_t m = in[IDX3(by, bx, c, iw, C)];
                 for (int dy = 0; dy < k; ++dy)
                     for (int dx = 0; dx < k; ++dx) {
-                        double v = in[IDX3(by + dy, bx + dx, c, iw, C)];
+                        real_t v = in[IDX3(by + dy, bx + dx, c, iw, C)];
                         if (v > m) m = v;
                     }
                 out[IDX3(yy, xx, c, ow, C)] = m;
@@ -183,5 +192,16 @@ int oracle_num_threads(void)
     return omp_get_max_threads();
 #else
     return 1;
+#endif
+}
+
+/* Set the number of OpenMP threads of the loops above (n >= 1; no effect without OpenMP). */
+void oracle_set_num_threads(int n)
+{
+#ifdef _OPENMP
+    extern void omp_set_num_threads(int);
+    if (n >= 1) omp_set_num_threads(n);
+#else
+    (void)n;
 #endif
 }

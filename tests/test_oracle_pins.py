@@ -217,6 +217,22 @@ def test_yolo16_more_groups_are_bit_identical_to_unfused(cuts, grids):
         assert np.array_equal(a, b)
 
 
+def test_fp32_build_matches_fp64_within_single_precision():
+    # the CPU baseline the benchmark times is the oracle's loops built in fp32; they must
+    # compute the same network, to single-precision accuracy (every sum and layer in fp32)
+    layers = synth.YOLO16
+    params = synth.make_params(layers, 3, 41, "bf16")
+    x = synth.make_input(1, 48, 40, 3, 42, "bf16")[0]
+    a = oracle.forward(layers, params, x)
+    b = oracle.forward(layers, params, x, precision="f32")
+    assert b[-1].dtype == np.float32 and a[-1].dtype == np.float64
+    for l in (0, 6, 15):
+        err = np.abs(b[l] - a[l]).max() / np.abs(a[l]).max()
+        assert err < 2e-5, (l, err)
+    # a dropped term or a wrong index would differ by far more than rounding
+    assert np.abs(b[-1] - a[-1]).max() > 0.0
+
+
 def test_region_that_misses_halo_is_rejected():
     # A region one row short of the receptive field must be refused, not silently padded.
     layers = [_conv_layer(3, 2)]
