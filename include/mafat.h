@@ -108,11 +108,12 @@ typedef struct {
     int32_t frame_major;        /* batch > 1 with two groups: 1 hands the frames out strictly one after
                                    another; 0 (default) overlaps frame f's second group with frame
                                    f + 1's first (the second group's small maps leave SMs idle) */
-    int32_t no_chain;           /* BF16 plans: 1 runs every convolution as its own stage.  0 (default)
-                                   chains a 3x3 convolution and the 1x1 convolution after it inside one
-                                   work item where both fit one TMEM accumulator buffer: the 3x3's
-                                   activated bf16 output stays in tensor memory and is the 1x1's A
-                                   operand, so it never reaches shared or global memory */
+    int32_t chain;              /* BF16 plans: 1 chains a 3x3 convolution and the 1x1 convolution after
+                                   it inside one work item where both fit one TMEM accumulator buffer:
+                                   the 3x3's activated bf16 output stays in tensor memory and is the
+                                   1x1's A operand, so it never reaches shared or global memory.
+                                   0 (default): every convolution is a stage of its own (on GB300 the
+                                   chained form measured slower for the 608x608 YOLOv2 plan) */
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */

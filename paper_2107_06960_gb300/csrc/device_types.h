@@ -88,6 +88,12 @@ struct MafatStageDev {
     int32_t chain;
     int32_t chained;
     int32_t chain_a_col, chain_out_col;
+    // chain stage: what the kernel needs of the chained 1x1 (a copy of its stage's fields, so that
+    // one stage record serves the item): N, output channels, fused pool, input chunks, K steps and
+    // swizzle of its weight blobs, blobs per piece, pieces, blob elements, scale / bias offset,
+    // packed weight offset
+    int32_t c2_n_blk, c2_cout, c2_pool, c2_n_chunks, c2_kst, c2_b_swz, c2_bpp, c2_n_pieces, c2_blob_elems, c2_sb_off;
+    int64_t c2_w_off;
 };
 
 enum { MAFAT_IN_PLANAR = 0, MAFAT_IN_GATHER = 1 };

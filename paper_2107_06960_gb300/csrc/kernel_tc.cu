@@ -449,10 +449,9 @@ static_assert(sizeof(ItemRec) <= kRecStride, "item record");
 
 struct EpiDst {
     __nv_bfloat16* out;
-    size_t pix, plane;
+    uint32_t pix, plane;  // element offsets within the output buffer (a frame's region: < 2^31)
     int nhwc, cout, pool;
     bool store;
-    uint32_t tmem;  // nonzero: the packed bf16 result goes to these TMEM columns instead (chain items)
 };
 
 // Epilogue of NC accumulator columns (output channels ch0 .. ch0+NC-1, NC = 16 or 32)
@@ -491,12 +490,6 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         pk[i / 2] = pack_bf16x2(v[0], v[1]);
         pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
     }
-    if constexpr (NC == 32) {
-        if (d.tmem) {  // a chain item's first pass: the 1x1's A operand, two bf16 per column
-            tmem_st16(d.tmem, pk);
-            return;
-        }
-    }
     if (!d.pool) {
         if (!d.store) return;
 #pragma unroll
@@ -504,7 +497,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
             const int ch = ch0 + 8 * o;
             if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
             const uint4 w = make_uint4(pk[4 * o], pk[4 * o + 1], pk[4 * o + 2], pk[4 * o + 3]);
-            __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+            __nv_bfloat16* p = d.out + (d.nhwc ? d.pix + (uint32_t)ch : (uint32_t)(ch >> 3) * d.plane + d.pix);
             *reinterpret_cast<uint4*>(p) = w;
         }
         return;
@@ -531,7 +524,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         }
         const int ch = ch0 + 8 * (2 * (int)h3 + (int)h0);
         if (!d.store || ch >= d.cout) return;
-        __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+        __nv_bfloat16* p = d.out + (d.nhwc ? d.pix + (uint32_t)ch : (uint32_t)(ch >> 3) * d.plane + d.pix);
         *reinterpret_cast<uint4*>(p) = make_uint4(r2[0], r2[1], r2[2], r2[3]);
     } else {
         // two octets: round 2 is a plain max with lane ^ 8, and lanes with h3 set leave the store
@@ -539,7 +532,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         for (int j = 0; j < 4; ++j) r1[j] = max_bf16x2(r1[j], __shfl_xor_sync(0xffffffffu, r1[j], 8));
         const int ch = ch0 + 8 * (int)h0;
         if (!d.store || h3 || ch >= d.cout) return;
-        __nv_bfloat16* p = d.nhwc ? d.out + d.pix + ch : d.out + (size_t)(ch >> 3) * d.plane + d.pix;
+        __nv_bfloat16* p = d.out + (d.nhwc ? d.pix + (uint32_t)ch : (uint32_t)(ch >> 3) * d.plane + d.pix);
         *reinterpret_cast<uint4*>(p) = make_uint4(r1[0], r1[1], r1[2], r1[3]);
     }
 }
@@ -819,6 +812,9 @@ __device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, in
     }
 }
 
+// kChain: the instance for plans with chain stages; plans without them run the instance
+// compiled without that path.
+template <bool kChain>
 __global__ void __launch_bounds__(kThreads, 1)
     mafat_tc_kernel(const __grid_constant__ MafatKParams p, const __grid_constant__ CUtensorMap in_map) {
     extern __shared__ uint8_t smem_raw[];
@@ -912,11 +908,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
                 }
                 MafatTaskDev tk;
-                MafatStageDev st, st2;
+                MafatStageDev st;
                 if (ticket >= 0) {  // two independent loads (the item names its stage)
                     tk = p.tasks[it.task];
                     st = p.stages[it.stage];
-                    if (st.chain) st2 = p.stages[it.stage + 1];  // the chained 1x1
                 }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
@@ -939,11 +934,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.out_h = tk.out_h;
                     rc.nbk = it.nbk;
                     // what the epilogue stores: the item's own output, or a chain item's 1x1 output
-                    rc.n_blk = st.chain ? st2.n_blk : st.n_blk;
-                    rc.cout = st.chain ? st2.cout : st.cout;
-                    rc.ch_base = st.chain ? 0 : it.nb * st.n_blk;
-                    rc.flags = ((st.chain ? st2.pool : st.pool) ? 1 : 0) | (tk.out_nhwc ? 2 : 0) |
-                               ((it.flags & 1) ? 4 : 0);
+                    const bool chain = kChain && st.chain;
+                    rc.n_blk = chain ? st.c2_n_blk : st.n_blk;
+                    rc.cout = chain ? st.c2_cout : st.cout;
+                    rc.ch_base = chain ? 0 : it.nb * st.n_blk;
+                    rc.flags = ((chain ? st.c2_pool : st.pool) ? 1 : 0) | (tk.out_nhwc ? 2 : 0) | ((it.flags & 1) ? 4 : 0);
                     rc.done_ctr = tk.done_ctr;
                     rc.extra_ctr = it.extra_ctr;
                     rm.k = (int16_t)st.k;
@@ -961,21 +956,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rm.blob_elems = st.blob_elems;
                     rm.sb = st.sb_off + it.nb * st.n_blk;
                     rm.n_mid = st.n_blk;
-                    rm.chain = (int16_t)st.chain;
+                    rm.chain = (int16_t)chain;
                     rc.n_mid = (int16_t)st.n_blk;
-                    rc.chain = (int16_t)st.chain;
-                    if (st.chain) {
+                    rc.chain = (int16_t)chain;
+                    if (chain) {
                         ChainRec& rh = recs[qs].chain;
-                        rh.n2 = (int16_t)st2.n_blk;
-                        rh.nch2 = (int16_t)st2.n_chunks;
-                        rh.kst2 = (int16_t)st2.kst;
-                        rh.swz2 = (int16_t)st2.b_swz;
-                        rh.bpp2 = (int16_t)st2.bpp;
-                        rh.np2 = (int16_t)st2.n_pieces;
+                        rh.n2 = (int16_t)st.c2_n_blk;
+                        rh.nch2 = (int16_t)st.c2_n_chunks;
+                        rh.kst2 = (int16_t)st.c2_kst;
+                        rh.swz2 = (int16_t)st.c2_b_swz;
+                        rh.bpp2 = (int16_t)st.c2_bpp;
+                        rh.np2 = (int16_t)st.c2_n_pieces;
                         rh.a_col = (int16_t)st.chain_a_col;
                         rh.out_col = (int16_t)st.chain_out_col;
-                        rh.blob2 = st2.blob_elems;
-                        rh.sb2 = st2.sb_off;
+                        rh.blob2 = st.c2_blob_elems;
+                        rh.sb2 = st.c2_sb_off;
                         rc.a_col = (int16_t)st.chain_a_col;
                         rc.out_col = (int16_t)st.chain_out_col;
                     }
@@ -1063,21 +1058,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                             if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
                 }
 #undef MAFAT_LOAD_PIECE
-                if (st.chain) {
+                if (kChain && st.chain) {
                     // the chained 1x1's weights follow the 3x3's, streamed piece by piece (never
                     // resident), in the order the MMA issuer consumes them
-                    const uint16_t* wset2 = p.w_bf16 + st2.w_off;
-                    const int G2 = st2.n_chunks * st2.n_bsteps;
-                    const uint32_t blob_bytes2 = (uint32_t)(st2.blob_elems * 2);
-                    for (int pc = 0; pc < st2.n_pieces; ++pc) {
+                    const uint16_t* wset2 = p.w_bf16 + st.c2_w_off;
+                    const int G2 = st.c2_n_chunks;  // one tap per blob
+                    const uint32_t blob_bytes2 = (uint32_t)(st.c2_blob_elems * 2);
+                    for (int pc = 0; pc < st.c2_n_pieces; ++pc) {
                         const int b_ = wb.next;
                         wb.next ^= 1;
                         mbar_wait(bar(kBarBEmpty + b_), (wb.loads(b_) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
-                        const int nblob_ = min(st2.bpp, G2 - pc * st2.bpp);
+                        const int nblob_ = min(st.c2_bpp, G2 - pc * st.c2_bpp);
                         const uint32_t bytes_ = (uint32_t)nblob_ * blob_bytes2;
                         mbar_arrive_expect_tx(bar(kBarBFull + b_), bytes_);
-                        bulk_load(sbase + kOffB + b_ * kBPieceBytes, wset2 + (size_t)pc * st2.bpp * st2.blob_elems, bytes_,
-                                  bar(kBarBFull + b_));
+                        bulk_load(sbase + kOffB + b_ * kBPieceBytes, wset2 + (size_t)pc * st.c2_bpp * st.c2_blob_elems,
+                                  bytes_, bar(kBarBFull + b_));
                         wb.set_loaded(b_, -1, false);
                     }
                 }
@@ -1125,7 +1120,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 // release the slot once the record has been read (a chain item's slot is held until
                 // its chained 1x1's fields have been read, on the chain path)
-                const bool chain = ticket >= 0 && wu(mr.chain) != 0;
+                const bool chain = kChain && ticket >= 0 && wu(mr.chain) != 0;
                 if (!chain) mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
@@ -1348,66 +1343,80 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float* sc = reinterpret_cast<const float*>(smem + kOffSb + buf * kSbSlotBytes);
             const float* bi = sc + MAFAT_MAX_NBLK;
             const uint32_t acc_lanes = tmem_base + ((uint32_t)(wq * 32) << 16) + (uint32_t)(buf * kAccStride);
+            uint32_t col0 = 0;  // accumulator column of what is stored
+            if (kChain && rc.chain) {
+                // Chain item, first pass: the 3x3's accumulator (n_mid columns of one block),
+                // activated and rounded as for a stored output, into TMEM at column a_col as the
+                // chained 1x1's A operand (two bf16 per column), 32 columns per unit, every other
+                // unit to this warpgroup; then, once the 1x1's MMAs are done, its accumulator
+                // (from column out_col) is stored like any output below.
+                for (int q = 32 * h; q < rc.n_mid; q += 32 * kEpiGroups) {
+                    uint32_t raw[32];
+                    tmem_ld32(acc_lanes + (uint32_t)q, raw);
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 4) {
+                        const float4 s4 = *reinterpret_cast<const float4*>(sc + q + i);
+                        const float4 b4 = *reinterpret_cast<const float4*>(bi + q + i);
+                        const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+                        float v[4];
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float z = fmaf(sv[e], __uint_as_float(raw[i + e]), bv[e]);
+                            v[e] = fmaxf(z, 0.1f * z);
+                        }
+                        pk[i / 2] = pack_bf16x2(v[0], v[1]);
+                        pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
+                    }
+                    tmem_st16(acc_lanes + (uint32_t)(rc.a_col + q / 2), pk);
+                }
+                tmem_st_wait();
+                tc_fence_before();
+                mbar_arrive(bar(kBarMidFull + buf));
+                mbar_wait(bar(kBarAccFull + buf), (buf ? full_ph1++ : full_ph0++) & 1u, p.ctr, pipe_limit, broken, 64);
+                __syncwarp();
+                tc_fence_after();
+                col0 = (uint32_t)rc.out_col;
+                sc += rc.n_mid;
+                bi += rc.n_mid;
+            }
             const int X = rc.x0 + cc;
-            // A chain item takes two passes over the same unit loop: first the 3x3's accumulator
-            // (n_mid columns), activated and rounded as for a stored output, into TMEM at column
-            // a_col as the chained 1x1's A operand; then, once the 1x1's MMAs are done, its
-            // accumulator from column out_col, stored like any output.  Other items take the
-            // second pass only.
-            for (int pass = rc.chain ? 0 : 1; pass < 2; ++pass) {
-                const bool mid = pass == 0;
-                const int n_blk = mid ? rc.n_mid : rc.n_blk;
-                const uint32_t col0 = mid ? 0u : (rc.chain ? (uint32_t)rc.out_col : 0u);
-                const float* psc = sc + (rc.chain && !mid ? rc.n_mid : 0);
-                const float* pbi = bi + (rc.chain && !mid ? rc.n_mid : 0);
-                const bool pool = !mid && (rc.flags & 1) != 0, nhwc = !mid && (rc.flags & 2) != 0;
-                // Work split between the warpgroups in units of one block x 32 output columns
-                // (16 when N is an odd multiple of 16), dealt round-robin.
-                const int uw = (n_blk & 31) == 0 ? 32 : 16;
-                const int upb = uw == 32 ? n_blk >> 5 : n_blk >> 4;  // units per block
-                // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
-                for (int b = 0, qi = h;; qi += kEpiGroups) {
-                    while (qi >= upb) {
-                        qi -= upb;
-                        ++b;
-                    }
-                    if (b >= rc.nbk) break;
-                    const int q = qi * uw;
-                    const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
-                    const bool valid = (Y < rc.ylim) && (X < rc.xlim);
-                    // a pooled stage's conv region starts on even rows and columns and has even
-                    // extents, so a window's four lanes agree on valid
-                    int oy = Y, ox = X;
-                    if (pool) {
-                        oy = Y >> 1;
-                        ox = X >> 1;
-                    }
-                    const size_t pix = (size_t)(oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0);
-                    EpiDst dst;
-                    dst.out = rc.out;
-                    dst.nhwc = nhwc;
-                    dst.pix = nhwc ? pix * rc.cout : pix * 8;
-                    dst.plane = (size_t)rc.out_h * rc.out_w * 8;
-                    dst.cout = rc.cout;
-                    dst.store = valid;
-                    dst.pool = pool;
-                    dst.tmem = mid ? acc_lanes + (uint32_t)(rc.a_col + q / 2) : 0u;
-                    const uint32_t taddr = acc_lanes + col0 + (uint32_t)(b * n_blk + q);
-                    if (uw == 32)
-                        epi_chunk<32>(taddr, psc + q, pbi + q, rc.ch_base + q, dst, lane);
-                    else
-                        epi_chunk<16>(taddr, psc + q, pbi + q, rc.ch_base + q, dst, lane);
+            const bool pool = (rc.flags & 1) != 0, nhwc = (rc.flags & 2) != 0;
+            // Work split between the warpgroups in units of one block x 32 output columns
+            // (16 when N is an odd multiple of 16), dealt round-robin.
+            const int uw = (rc.n_blk & 31) == 0 ? 32 : 16;
+            const int upb = uw == 32 ? rc.n_blk >> 5 : rc.n_blk >> 4;  // units per block
+            // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
+            for (int b = 0, qi = h;; qi += kEpiGroups) {
+                while (qi >= upb) {
+                    qi -= upb;
+                    ++b;
                 }
-                if (mid) {
-                    // hand the A operand to the MMA issuer, then wait for the 1x1's accumulator
-                    tmem_st_wait();
-                    tc_fence_before();
-                    mbar_arrive(bar(kBarMidFull + buf));
-                    mbar_wait(bar(kBarAccFull + buf), (buf ? full_ph1++ : full_ph0++) & 1u, p.ctr, pipe_limit, broken,
-                              64);
-                    __syncwarp();
-                    tc_fence_after();
+                if (b >= rc.nbk) break;
+                const int q = qi * uw;
+                const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
+                const bool valid = (Y < rc.ylim) && (X < rc.xlim);
+                // a pooled stage's conv region starts on even rows and columns and has even
+                // extents, so a window's four lanes agree on valid
+                int oy = Y, ox = X;
+                if (pool) {
+                    oy = Y >> 1;
+                    ox = X >> 1;
                 }
+                const uint32_t pix = (uint32_t)((oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0));
+                EpiDst dst;
+                dst.out = rc.out;
+                dst.nhwc = nhwc;
+                dst.pix = nhwc ? pix * (uint32_t)rc.cout : pix * 8u;
+                dst.plane = (uint32_t)(rc.out_h * rc.out_w * 8);
+                dst.cout = rc.cout;
+                dst.store = valid;
+                dst.pool = pool;
+                const uint32_t taddr = acc_lanes + col0 + (uint32_t)(b * rc.n_blk + q);
+                if (uw == 32)
+                    epi_chunk<32>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
+                else
+                    epi_chunk<16>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
             }
             tc_fence_before();
             mbar_arrive(bar(kBarAccEmpty + buf));  // also frees the scale / bias slot
@@ -1528,14 +1537,20 @@ __global__ void __launch_bounds__(128, 1)
 
 size_t mafat_tc_smem_bytes() { return (size_t)kSmemBytes; }
 
-cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(mafat_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, bool chain, cudaStream_t s) {
+    static bool attr_set[2] = {false, false};
+    if (!attr_set[chain]) {
+        cudaError_t e = chain ? cudaFuncSetAttribute(mafat_tc_kernel<true>,
+                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes)
+                              : cudaFuncSetAttribute(mafat_tc_kernel<false>,
+                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_set[chain] = true;
     }
-    mafat_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
+    if (chain)
+        mafat_tc_kernel<true><<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
+    else
+        mafat_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
     return cudaGetLastError();
 }
 

@@ -38,8 +38,9 @@ struct MafatKParams {
     const MafatDepDev* deps;            // task dependency lists (halo reuse)
 };
 
-// bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan.
-cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, cudaStream_t s);
+// bf16 tensor-core kernel (tcgen05 + TMA): one launch runs a whole plan; `chain` selects the
+// instance with the on-chip 3x3 -> 1x1 chaining path (plans that have chain stages).
+cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, bool chain, cudaStream_t s);
 size_t mafat_tc_smem_bytes();
 // fp32 CUDA-core check kernel: same work list, same scheduler.
 cudaError_t mafat_launch_fp32(const MafatKParams& p, int grid, cudaStream_t s);

@@ -345,14 +345,15 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // dominates.  Stages with more blocks than CTAs keep the widest block, which
             // reuses every A operand for the most output channels.
             const int cout_pad = (L.c_out + 15) / 16 * 16;
-            // On-chip chaining (tensor-core plans, halo recompute): a 3x3 convolution without a
-            // fused pool whose next layer is a 1x1 convolution of the same group runs both in one
-            // item when the 3x3's accumulator, its bf16 result and the 1x1's accumulator fit one
-            // 256-column TMEM buffer for a block of 128 pixels; the 1x1's stage has no tasks.
+            // On-chip chaining (option; tensor-core plans, halo recompute): a 3x3 convolution
+            // without a fused pool whose next layer is a 1x1 convolution of the same group runs
+            // both in one item when the 3x3's accumulator, its bf16 result and the 1x1's
+            // accumulator fit one 256-column TMEM buffer for a block of 128 pixels; the 1x1's
+            // stage has no tasks.
             const bool prev_chain = !t.stages.empty() && t.stage_first[g] < (int)t.stages.size() &&
                                     t.stages.back().chain;
             bool chain_here = false;
-            if (cfg.dtype == 0 && !cfg.halo_reuse && !cfg.no_chain && !prev_chain && L.k == 3 && l + 1 <= last &&
+            if (cfg.dtype == 0 && !cfg.halo_reuse && cfg.chain && !prev_chain && L.k == 3 && l + 1 <= last &&
                 net.layers[l + 1].type == L_CONV && net.layers[l + 1].k == 1) {
                 const int next_pad = (net.layers[l + 1].c_out + 15) / 16 * 16;
                 chain_here = cout_pad % 64 == 0 && cout_pad + cout_pad / 2 + next_pad <= 256;
@@ -423,6 +424,11 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             if (s.chain_a_col != s.n_blk || s.chain_out_col != s.n_blk + s.n_blk / 2 ||
                 s.chain_out_col + s2.n_blk > 256)
                 return "chained stages exceed one TMEM accumulator buffer";
+            if (s.c2_n_blk != s2.n_blk || s.c2_cout != s2.cout || s.c2_pool != s2.pool || s.c2_n_chunks != s2.n_chunks ||
+                s.c2_kst != s2.kst || s.c2_b_swz != s2.b_swz || s.c2_bpp != s2.bpp || s.c2_n_pieces != s2.n_pieces ||
+                s.c2_blob_elems != s2.blob_elems || s.c2_sb_off != s2.sb_off || s.c2_w_off != s2.w_off ||
+                s2.n_bsteps != 1)
+                return "chain stage's copy of its 1x1 differs";
         }
         if (s.chained && (&s == t.stages.data() || !(&s - 1)->chain)) return "a chained stage without its chain stage";
         if (s.in_mode == MAFAT_IN_GATHER) {
@@ -492,6 +498,23 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             if (s.pool) ++l;
         }
         t.stage_last[g] = (int)t.stages.size() - 1;
+    }
+    // a chain stage carries the fields of its chained 1x1 that the kernel reads
+    for (size_t si = 0; si + 1 < t.stages.size(); ++si) {
+        MafatStageDev& a = t.stages[si];
+        if (!a.chain) continue;
+        const MafatStageDev& b = t.stages[si + 1];
+        a.c2_n_blk = b.n_blk;
+        a.c2_cout = b.cout;
+        a.c2_pool = b.pool;
+        a.c2_n_chunks = b.n_chunks;
+        a.c2_kst = b.kst;
+        a.c2_b_swz = b.b_swz;
+        a.c2_bpp = b.bpp;
+        a.c2_n_pieces = b.n_pieces;
+        a.c2_blob_elems = b.blob_elems;
+        a.c2_sb_off = b.sb_off;
+        a.c2_w_off = b.w_off;
     }
 
     // ---- geometry of the group inputs / outputs
@@ -1025,6 +1048,7 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         int64_t out_elems = k.out_nhwc ? (int64_t)k.out_h * k.out_w * so.cout
                                        : (int64_t)((so.cout + 7) / 8) * 8 * k.out_h * k.out_w;
         if (k.out_off < 0 || k.out_off + out_elems > buf_total(k.out_kind)) return "output buffer outside its allocation";
+        if (out_elems >= ((int64_t)1 << 31)) return "an output region exceeds 2^31 elements";
         if (k.out_kind == MAFAT_BUF_SCRATCH && out_elems > t.slot_buf_elems) return "scratch output above buffer size";
         if (k.done_ctr < MAFAT_CTR_BASE || k.done_ctr >= MAFAT_CTR_BASE + t.n_counters) return "bad done counter";
     }

@@ -52,6 +52,7 @@ struct mafat_plan_s {
     // multiple of 16 bytes (t.in_convert), made by a small kernel before each launch
     void* d_in_planar = nullptr;
     size_t in_planar_bytes = 0;
+    bool has_chain = false;  // the plan has chain stages (selects the kernel instance)
     // staging for mafat_run_host: the NHWC input batch as copied from the host, the output
     void* d_in_stage = nullptr;
     void* d_out_stage = nullptr;
@@ -244,7 +245,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
             if (!ok) return fail(MAFAT_ECUDA, err);
             p->in_map_ptr = in_dev;
         }
-        e = mafat_launch_tc(kp, p->in_map, p->grid, s);
+        e = mafat_launch_tc(kp, p->in_map, p->grid, p->has_chain, s);
     } else {
         e = mafat_launch_fp32(kp, p->grid, s);
     }
@@ -376,7 +377,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.lookahead_items = o.lookahead_items;
     cfg.halo_reuse = o.halo_reuse != 0;
     cfg.frame_major = o.frame_major != 0;
-    cfg.no_chain = o.no_chain != 0;
+    cfg.chain = o.chain != 0;
     if (o.tile_bounds) {
         // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
         const int32_t* b = o.tile_bounds;
@@ -415,6 +416,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     const mafat::Layer& L0 = net->net.layers[0];
     p->in_bytes = (size_t)t.cfg.batch * L0.c_in * L0.h_in * L0.w_in * p->esz;  // NHWC, as the caller holds it
     p->in_planar_bytes = t.in_convert ? (size_t)t.cfg.batch * t.in_c8 * 8 * L0.h_in * L0.w_in * p->esz : 0;
+    for (const MafatStageDev& st : t.stages) p->has_chain = p->has_chain || st.chain != 0;
     p->out_bytes = (size_t)t.cfg.batch * t.out_h * t.out_w * t.out_c * p->esz;
     p->cut_bytes = (size_t)t.cfg.batch * t.cut_c8 * 8 * t.cut_h * t.cut_w * p->esz;
     p->ctr_bytes = (size_t)(MAFAT_CTR_BASE + t.n_counters) * sizeof(uint32_t);

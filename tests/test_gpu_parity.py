@@ -378,7 +378,7 @@ def test_measured_search_picks_the_fastest_timed_plan(mf):
 
 
 # ---------------------------------------------------------------------------
-# On-chip chaining of a 3x3 and the 1x1 after it (the 3x3's output stays in TMEM)
+# On-chip chaining of a 3x3 and the 1x1 after it (option chain=True: the 3x3's output stays in TMEM)
 # ---------------------------------------------------------------------------
 
 @pytest.mark.parametrize("cut,grids", [(8, [(3, 3), (2, 2)]), (6, [(2, 2), (2, 1)]), (None, [(3, 2)])])
@@ -387,8 +387,8 @@ def test_bf16_chained_pair_matches_unchained_and_oracle(mf, cut, grids):
     layers = synth.YOLO16
     params = synth.make_params(layers, 3, 61, "bf16")
     x = synth.make_input(2, 96, 96, 3, 62, "bf16")
-    c1, o1 = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
-    c0, o0 = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=dict(no_chain=True))
+    c1, o1 = run_plan(mf, layers, params, x, cut, grids, mf.BF16, plan_kwargs=dict(chain=True))
+    c0, o0 = run_plan(mf, layers, params, x, cut, grids, mf.BF16)
     assert np.array_equal(o1, o0)
     if cut is not None:
         assert np.array_equal(c1, c0)
@@ -403,17 +403,17 @@ def test_bf16_chained_pair_matches_unchained_and_oracle(mf, cut, grids):
 def test_bf16_chained_pair_small_networks(mf, layers):
     params = synth.make_params(layers, 16, 63, "bf16")
     x = synth.make_input(2, 40, 48, 16, 64, "bf16")
-    _, o1 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16)
-    _, o0 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16, plan_kwargs=dict(no_chain=True))
+    _, o1 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16, plan_kwargs=dict(chain=True))
+    _, o0 = run_plan(mf, layers, params, x, None, [(2, 3)], mf.BF16)
     assert np.array_equal(o1, o0)
     _check_groups(None, o1, _oracle_groups(layers, params, x, None), None, TOL_BF16)
 
 
 def test_bf16_608_chained_matches_unchained(mf):
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
-    c1, o1 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16)
-    c0, o0 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16,
-                      plan_kwargs=dict(no_chain=True))
+    c1, o1 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16,
+                      plan_kwargs=dict(chain=True))
+    c0, o0 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16)
     assert np.array_equal(o1, o0) and np.array_equal(c1, c0)
 
 

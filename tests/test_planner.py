@@ -374,13 +374,13 @@ def test_input_layout_needs_no_conversion_when_rows_allow(mf, c, w, launches):
 
 
 def test_chained_pairs_in_the_benchmark_plan(mf):
-    # bf16 plans run a 3x3 convolution and the 1x1 after it in one item where both fit one TMEM
-    # accumulator buffer (YOLOv2 layers 4 -> 5: 128 + 64 + 64 columns): one task per tile fewer,
-    # the same regions and the same work
+    # with chain=True, bf16 plans run a 3x3 convolution and the 1x1 after it in one item where
+    # both fit one TMEM accumulator buffer (YOLOv2 layers 4 -> 5: 128 + 64 + 64 columns): one
+    # task per tile fewer, the same regions and the same work
     wl = synth.workload("yolo16_608_5x5_c8_2x2")
     net = _net(mf, wl["layers"], 608)
-    chained = mf.Plan(net, 8, wl["grids"], dry_run=True)
-    plain = mf.Plan(net, 8, wl["grids"], dry_run=True, no_chain=True)
+    chained = mf.Plan(net, 8, wl["grids"], dry_run=True, chain=True)
+    plain = mf.Plan(net, 8, wl["grids"], dry_run=True)
     a, b = chained.stats(), plain.stats()
     assert b["n_tasks"] - a["n_tasks"] == 25  # layer 5 of each group-1 tile
     assert a["executed_flops"] == b["executed_flops"] and a["issued_flops"] == b["issued_flops"]
@@ -388,10 +388,10 @@ def test_chained_pairs_in_the_benchmark_plan(mf):
         for l in (4, 5, 6):
             assert chained.tile_region(0, i, j, l) == plain.tile_region(0, i, j, l)
     # fp32 plans and halo-reuse plans keep every convolution a stage of its own
-    f32 = mf.Plan(net, 8, wl["grids"], dry_run=True, dtype=mf.FP32)
+    f32 = mf.Plan(net, 8, wl["grids"], dry_run=True, dtype=mf.FP32, chain=True)
     assert f32.stats()["n_tasks"] == b["n_tasks"]
-    hr_c = mf.Plan(net, 8, wl["grids"], dry_run=True, halo_reuse=True)
-    hr_p = mf.Plan(net, 8, wl["grids"], dry_run=True, halo_reuse=True, no_chain=True)
+    hr_c = mf.Plan(net, 8, wl["grids"], dry_run=True, halo_reuse=True, chain=True)
+    hr_p = mf.Plan(net, 8, wl["grids"], dry_run=True, halo_reuse=True)
     assert hr_c.stats()["n_tasks"] == hr_p.stats()["n_tasks"]
 
 
@@ -405,6 +405,6 @@ def test_chained_pairs_in_the_benchmark_plan(mf):
 def test_chain_eligibility(mf, layers, chained):
     net = mf.Net(layers, 32, 32, 16)
     net.set_params(synth.make_params(layers, 16, 9, "bf16"))
-    c = mf.Plan(net, None, [(2, 2)], dry_run=True).stats()
-    p = mf.Plan(net, None, [(2, 2)], dry_run=True, no_chain=True).stats()
+    c = mf.Plan(net, None, [(2, 2)], dry_run=True, chain=True).stats()
+    p = mf.Plan(net, None, [(2, 2)], dry_run=True).stats()
     assert p["n_tasks"] - c["n_tasks"] == 4 * chained
