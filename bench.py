@@ -93,7 +93,7 @@ class ClockSampler:
 
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,utilization.gpu")
 
     def __init__(self, gpu_index):
         self.gpu = gpu_index
@@ -104,7 +104,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.QUERY, "--format=csv,noheader,nounits",
-                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "10"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
             # nvidia-smi takes a while to start: wait (bounded) for its first line so that
@@ -128,7 +128,7 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-        sm, smax, reasons = [], [], set()
+        sm, smax, busy, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         # the samples taken after the timed region started (the first line predates it)
         for ln in self.lines[self.n_before:] or self.lines[-1:]:
@@ -140,11 +140,19 @@ class ClockSampler:
                 smax.append(float(f[2]))
             except ValueError:
                 continue
+            try:
+                busy.append(len(f) > 9 and float(f[9]) >= 50.0)
+            except ValueError:
+                busy.append(False)
             for n, v in zip(names, f[5:9]):
                 if v.lower() in ("active", "1"):
                     reasons.add(n)
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "reasons": sorted(reasons), "samples": len(sm)}
+        loaded = [c for c, b in zip(sm, busy) if b]
+        use = loaded or sm
+        return {"sm_mhz": statistics.median(use) if use else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm), "samples_under_load": len(loaded),
+                "span": "every timed leg (device, chained, steady-state, end-to-end); median over samples with "
+                        "GPU utilisation >= 50 %"}
 
 
 def _best_of(n, fn):
@@ -375,7 +383,6 @@ def main():
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
-    clk = clocks.stop()
     plan.sync_status(stream=stream)
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     dev_s = sum(step_ms) / 1e3
@@ -472,6 +479,8 @@ def main():
     for _ in range(sync_steps):
         plan.run_host(xh, oh, stream=stream)
     sync_s = time.perf_counter() - t0
+    # the sampler ran through every timed leg (device, chained, steady-state, end-to-end)
+    clk = clocks.stop()
 
     dev_s_max, e2e_s_max, sync_s_max, ss_s_max = reduce_max(
         pg, [dev_s, e2e_s, sync_s, ss["seconds"] if ss else 0.0], dev)
