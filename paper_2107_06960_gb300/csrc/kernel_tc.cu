@@ -373,6 +373,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&h);
 }
+// Folded BN and leaky ReLU of two accumulator values with the packed fp32 instructions:
+// z = s * acc + b (fma.rn per element) and 0.1 z (mul.rn per element), then
+// max(z, 0.1 z) per element: the same roundings as the scalar form.
+__device__ __forceinline__ void bn_leaky2(float s0, float s1, uint32_t a0, uint32_t a1, float b0, float b1, float& v0,
+                                          float& v1) {
+    float z0, z1, t0, t1;
+    asm("{\n\t.reg .b64 s, a, b, z, t, c;\n\t"
+        "mov.b64 s, {%4, %5};\n\t"
+        "mov.b64 a, {%6, %7};\n\t"
+        "mov.b64 b, {%8, %9};\n\t"
+        "fma.rn.f32x2 z, s, a, b;\n\t"
+        "mov.b64 c, {%10, %10};\n\t"
+        "mul.rn.f32x2 t, z, c;\n\t"
+        "mov.b64 {%0, %1}, z;\n\t"
+        "mov.b64 {%2, %3}, t;\n\t}"
+        : "=f"(z0), "=f"(z1), "=f"(t0), "=f"(t1)
+        : "f"(s0), "f"(s1), "r"(a0), "r"(a1), "f"(b0), "f"(b1), "f"(0.1f));
+    v0 = fmaxf(z0, t0);
+    v1 = fmaxf(z1, t1);
+}
+
 __device__ __forceinline__ uint32_t max_bf16x2(uint32_t a, uint32_t b) {
     __nv_bfloat162 x = *reinterpret_cast<__nv_bfloat162*>(&a), y = *reinterpret_cast<__nv_bfloat162*>(&b);
     __nv_bfloat162 m = __hmax2(x, y);
@@ -480,13 +501,9 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
     for (int i = 0; i < NC; i += 4) {
         const float4 s4 = *reinterpret_cast<const float4*>(sc + i);  // shared memory, same address
         const float4 b4 = *reinterpret_cast<const float4*>(bi + i);  // for the whole warp
-        const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
         float v[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const float z = fmaf(sv[u], __uint_as_float(raw[i + u]), bv[u]);
-            v[u] = fmaxf(z, 0.1f * z);
-        }
+        bn_leaky2(s4.x, s4.y, raw[i], raw[i + 1], b4.x, b4.y, v[0], v[1]);
+        bn_leaky2(s4.z, s4.w, raw[i + 2], raw[i + 3], b4.z, b4.w, v[2], v[3]);
         pk[i / 2] = pack_bf16x2(v[0], v[1]);
         pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
     }
@@ -1358,13 +1375,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int i = 0; i < 32; i += 4) {
                         const float4 s4 = *reinterpret_cast<const float4*>(sc + q + i);
                         const float4 b4 = *reinterpret_cast<const float4*>(bi + q + i);
-                        const float sv[4] = {s4.x, s4.y, s4.z, s4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
                         float v[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float z = fmaf(sv[e], __uint_as_float(raw[i + e]), bv[e]);
-                            v[e] = fmaxf(z, 0.1f * z);
-                        }
+                        bn_leaky2(s4.x, s4.y, raw[i], raw[i + 1], b4.x, b4.y, v[0], v[1]);
+                        bn_leaky2(s4.z, s4.w, raw[i + 2], raw[i + 3], b4.z, b4.w, v[2], v[3]);
                         pk[i / 2] = pack_bf16x2(v[0], v[1]);
                         pk[i / 2 + 1] = pack_bf16x2(v[2], v[3]);
                     }
