@@ -377,6 +377,25 @@ def test_measured_search_picks_the_fastest_timed_plan(mf):
     assert rel_err(out[0], oracle.forward(layers, params, x[0])[-1]) <= TOL_BF16
 
 
+@pytest.mark.parametrize("n_layers,cut,c,h,w,launches", [
+    (8, 4, 3, 40, 56, 1),   # RGB rows of 336 bytes: widened in the kernel
+    (4, 2, 3, 36, 44, 2),   # RGB rows of 264 bytes (not a multiple of 16): the layout kernel first
+    (8, 4, 1, 32, 48, 1),   # one channel
+    (8, 4, 5, 40, 40, 1),   # five channels
+])
+def test_bf16_nhwc_image_batch2(mf, n_layers, cut, c, h, w, launches):
+    # the first layer reads the NHWC image of every frame in place (raw rows widened in the
+    # kernel) or, for rows of another size, through the layout kernel; both at batch 2
+    layers = synth.YOLO16[:n_layers]
+    params = synth.make_params(layers, c, 71 + c, "bf16")
+    x = synth.make_input(2, h, w, c, 72 + w, "bf16")
+    net = mf.Net(layers, h, w, c)
+    net.set_params(params)
+    assert mf.Plan(net, cut, [(2, 3), (2, 2)], batch=2, dry_run=True).launches_per_run() == launches
+    got_cut, out = run_plan(mf, layers, params, x, cut, [(2, 3), (2, 2)], mf.BF16)
+    _check_groups(got_cut, out, _oracle_groups(layers, params, x, cut), cut, TOL_BF16)
+
+
 # ---------------------------------------------------------------------------
 # On-chip chaining of a 3x3 and the 1x1 after it (option chain=True: the 3x3's output stays in TMEM)
 # ---------------------------------------------------------------------------
