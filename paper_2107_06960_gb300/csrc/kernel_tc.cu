@@ -257,9 +257,6 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 // Broadcast from lane 0: marks the value warp-uniform for the compiler.
 __device__ __forceinline__ int wu(int v) { return __shfl_sync(0xffffffffu, v, 0); }
 
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
 // Warp-wide forms for the MMA warp, whose 32 lanes all run the issue loop (so that
 // descriptors stay warp-uniform): elect.sync picks one lane, the same lane every time
 // since the warp is converged, to issue the operation.
@@ -520,7 +517,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         return;
     }
     const bool h0 = (lane & 1) != 0, h3 = (lane & 8) != 0;
-    // round 1, partner lane ^ 1: keep octet 2m + h0 of each pair (2m, 2m + 1)
+    // first exchange, partner lane ^ 1: keep octet 2m + h0 of each pair (2m, 2m + 1)
     uint32_t r1[NC / 4];
 #pragma unroll
     for (int m = 0; m < NO / 2; ++m)
@@ -531,7 +528,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
             r1[4 * m + j] = max_bf16x2(h0 ? hi : lo, got);
         }
     if constexpr (NO == 4) {
-        // round 2, partner lane ^ 8: keep octet 2 * h3 + h0
+        // second exchange, partner lane ^ 8: keep octet 2 * h3 + h0
         uint32_t r2[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -544,7 +541,7 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
         __nv_bfloat16* p = d.out + (d.nhwc ? d.pix + (uint32_t)ch : (uint32_t)(ch >> 3) * d.plane + d.pix);
         *reinterpret_cast<uint4*>(p) = make_uint4(r2[0], r2[1], r2[2], r2[3]);
     } else {
-        // two octets: round 2 is a plain max with lane ^ 8, and lanes with h3 set leave the store
+        // two octets: the second exchange is a plain max with lane ^ 8, and lanes with h3 set leave the store
 #pragma unroll
         for (int j = 0; j < 4; ++j) r1[j] = max_bf16x2(r1[j], __shfl_xor_sync(0xffffffffu, r1[j], 8));
         const int ch = ch0 + 8 * (int)h0;
