@@ -288,17 +288,6 @@ __device__ __forceinline__ uint32_t instr_desc_bf16(int n, int m) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
-// No "memory" clobber: the MMA reads shared memory through its descriptors and
-// writes tensor memory only, and volatile asm statements keep their order.
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                         uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
-}
-
 // One MMA whose A operand is in tensor memory (a_tmem: column of K elements 0..1 of lane 0;
 // a K=16 step spans 8 columns, two bf16 per 32-bit column, lane = row of A), B in shared
 // memory, issued by one elected lane of the converged warp.
