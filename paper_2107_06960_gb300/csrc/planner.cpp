@@ -413,25 +413,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             for (;;) {
                 s.rows_box = MAFAT_BLK_ROWS * s.mb + L.k - 1;
                 const int row_bytes = s.cols_box * 16 * s.rows_box;
-                if (s.chain) {
-            const size_t si = (size_t)(&s - t.stages.data());
-            if (si + 1 >= t.stages.size() || !t.stages[si + 1].chained || t.stages[si + 1].k != 1 || s.k != 3 ||
-                s.pool)
-                return "a chain stage must be a 3x3 convolution followed by its chained 1x1";
-            const MafatStageDev& s2 = t.stages[si + 1];
-            if (s.n_nblk != 1 || s2.n_nblk != 1 || s.mb != 1 || s2.cin != s.cout || s.n_blk % 64 != 0)
-                return "chained stages need every channel of one 128-pixel block in one item";
-            if (s.chain_a_col != s.n_blk || s.chain_out_col != s.n_blk + s.n_blk / 2 ||
-                s.chain_out_col + s2.n_blk > 256)
-                return "chained stages exceed one TMEM accumulator buffer";
-            if (s.c2_n_blk != s2.n_blk || s.c2_cout != s2.cout || s.c2_pool != s2.pool || s.c2_n_chunks != s2.n_chunks ||
-                s.c2_kst != s2.kst || s.c2_b_swz != s2.b_swz || s.c2_bpp != s2.bpp || s.c2_n_pieces != s2.n_pieces ||
-                s.c2_blob_elems != s2.blob_elems || s.c2_sb_off != s2.sb_off || s.c2_w_off != s2.w_off ||
-                s2.n_bsteps != 1)
-                return "chain stage's copy of its 1x1 differs";
-        }
-        if (s.chained && (&s == t.stages.data() || !(&s - 1)->chain)) return "a chained stage without its chain stage";
-        if (s.in_mode == MAFAT_IN_GATHER) {
+                if (s.in_mode == MAFAT_IN_GATHER) {
                     // the expanded halo plus the raw rows it is built from share the stage
                     s.chunk8 = 1;
                     if (mafat_raw_offset(s.rows_box, s.cols_box) + s.rows_box * s.raw_e * 2 <= MAFAT_A_STAGE_BYTES ||
@@ -994,6 +976,24 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
             return "K steps per blob must be 1, 2 or 4 (1 when taps are paired)";
         if (s.b_swz && (s.kst != 4 || s.paired || (s.blob_elems * 2) % 1024 != 0))
             return "swizzled blobs need 64 channels and whole 1024-byte atoms";
+        if (s.chain) {
+            const size_t si = (size_t)(&s - t.stages.data());
+            if (si + 1 >= t.stages.size() || !t.stages[si + 1].chained || t.stages[si + 1].k != 1 || s.k != 3 ||
+                s.pool)
+                return "a chain stage must be a 3x3 convolution followed by its chained 1x1";
+            const MafatStageDev& s2 = t.stages[si + 1];
+            if (s.n_nblk != 1 || s2.n_nblk != 1 || s.mb != 1 || s2.cin != s.cout || s.n_blk % 64 != 0)
+                return "chained stages need every channel of one 128-pixel block in one item";
+            if (s.chain_a_col != s.n_blk || s.chain_out_col != s.n_blk + s.n_blk / 2 ||
+                s.chain_out_col + s2.n_blk > 256)
+                return "chained stages exceed one TMEM accumulator buffer";
+            if (s.c2_n_blk != s2.n_blk || s.c2_cout != s2.cout || s.c2_pool != s2.pool || s.c2_n_chunks != s2.n_chunks ||
+                s.c2_kst != s2.kst || s.c2_b_swz != s2.b_swz || s.c2_bpp != s2.bpp || s.c2_n_pieces != s2.n_pieces ||
+                s.c2_blob_elems != s2.blob_elems || s.c2_sb_off != s2.sb_off || s.c2_w_off != s2.w_off ||
+                s2.n_bsteps != 1)
+                return "chain stage's copy of its 1x1 differs";
+        }
+        if (s.chained && (&s == t.stages.data() || !(&s - 1)->chain)) return "a chained stage without its chain stage";
         if (s.in_mode == MAFAT_IN_GATHER) {
             const Layer& L = net.layers[s.layer];
             if (s.layer != 0 || !s.paired || L.c_in >= 8 || (int64_t)L.w_in * L.c_in % 8 != 0)
