@@ -114,6 +114,12 @@ typedef struct {
                                    1x1's A operand, so it never reaches shared or global memory.
                                    0 (default): every convolution is a stage of its own (on GB300 the
                                    chained form measured slower for the 608x608 YOLOv2 plan) */
+    int32_t rect_blocks;        /* 1: every work item's pixel blocks are 16x8 rectangles.  0 (default):
+                                   a convolution without a fused max-pool whose tile regions are at
+                                   most 32 - k + 1 pixels wide reads each region as its rows laid end
+                                   to end with a pitch of a multiple of 8 pixels, cut into runs of
+                                   128 pixels, where that takes fewer blocks (e.g. a 19x19 region: 4
+                                   blocks instead of 6); results are identical either way */
 } mafat_plan_options;
 
 /* Statistics of a plan (all per batch unless stated). */

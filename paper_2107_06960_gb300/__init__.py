@@ -36,7 +36,7 @@ class PlanOptions(ctypes.Structure):
                 ("wait_timeout_ns", i64), ("test_unpublished_task", i32), ("dry_run", i32),
                 ("trace", i32), ("force_nblk", i32), ("force_mb", i32), ("lookahead_items", i32),
                 ("tile_bounds", ctypes.POINTER(i32)), ("halo_reuse", i32), ("frame_major", i32),
-                ("chain", i32)]
+                ("chain", i32), ("rect_blocks", i32)]
 
 
 class PlanStats(ctypes.Structure):
@@ -253,7 +253,7 @@ class Plan:
     def __init__(self, net, cut=None, grids=((1, 1),), batch=1, dtype=BF16, ring_slots=0, wave_tiles=0,
                  max_ctas=0, wait_timeout_ns=0, test_unpublished_task=-1, dry_run=False, trace=False,
                  force_nblk=0, force_mb=0, lookahead_items=0, tile_bounds=None, halo_reuse=False,
-                 frame_major=False, chain=False):
+                 frame_major=False, chain=False, rect_blocks=False):
         self.net = net
         # cut: None (one group), the first layer of group 2, or a list of increasing cuts
         cut_list = [] if cut is None else (list(cut) if isinstance(cut, (list, tuple)) else [cut])
@@ -275,6 +275,7 @@ class Plan:
         opt.halo_reuse = int(halo_reuse)
         opt.frame_major = int(frame_major)
         opt.chain = int(chain)
+        opt.rect_blocks = int(rect_blocks)
         if tile_bounds is not None:
             # per group (rows, cols): the non-uniform tiling; kept alive with the plan
             flat = [v for rows, cols in list(tile_bounds)[:n_groups] for v in list(rows) + list(cols)]

@@ -9,10 +9,12 @@
 //                       (the tile's region from the Grid back-traversal,
 //                       Sec. 4.1) and where the result goes;
 //   * MafatItemDev   -- the work list in hand-out order: one item is up to
-//                       `mb` 16 x 8 blocks of conv output pixels (stacked
-//                       along rows) x one block of output channels of a
-//                       task, with up to two completion counters it must
-//                       wait for.
+//                       `mb` blocks of 128 conv output pixels x one block of
+//                       output channels of a task, with up to two completion
+//                       counters it must wait for.  A block is a 16 x 8
+//                       rectangle (stacked along rows), or, in a `flat`
+//                       stage, a run of 128 pixels of the task's region read
+//                       row after row with a row pitch of `cols_box` pixels.
 //
 // Activations are stored in "octet-planar" layout [C/8][H][W][8]: 8 channels of
 // one pixel are 16 bytes (bf16) or 32 bytes (fp32) and consecutive pixels of a
@@ -62,6 +64,16 @@ struct MafatStageDev {
     int32_t b_swz;        // 1: blobs in the 128-byte swizzled K-major layout (kst == 4), 0: no swizzle
     int32_t mb;           // M blocks per item (stacked along rows, one TMEM accumulator each)
     int32_t rows_box, cols_box;  // A halo box (pixels): 16*mb + k - 1 rows, 8 + k - 1 columns
+                                 // (flat stage: mafat_flat_rows(mb, pitch, k) rows, pitch columns)
+    // Flattened M blocks (convolutions without a fused pool, tensor maps of at most 32 pixels a
+    // row): the task's conv region of ch x cw pixels is read as ch rows of `pitch` = cols_box
+    // pixels (a multiple of 8, at least cw + k - 1) laid end to end, and block b is pixels
+    // 128 b .. 128 b + 127 of that sequence, pixel p being (p / pitch, p % pitch); pixels in
+    // columns cw .. pitch - 1 are computed and dropped.  The A halo of an item is the same
+    // rows laid out the same way, so that 8 consecutive pixels are one core matrix wherever a
+    // row ends, and tap (ky, kx) is an offset of ky * pitch + kx pixels.  A region 19 pixels
+    // wide takes 4 such blocks for 19 rows instead of 6 rectangles.
+    int32_t flat;
     int64_t w_off;        // element offset of this stage's packed bf16 weights
     int32_t blob_elems;   // elements of one blob (n_blk * 16 * kst)
     int32_t set_bytes;    // bytes of the weights of one output-channel block (all chunks and blobs)
@@ -98,6 +110,12 @@ struct MafatStageDev {
 
 enum { MAFAT_IN_PLANAR = 0, MAFAT_IN_GATHER = 1 };
 
+// Rows of the A box of a flat stage's item: its 128 * mb pixels start anywhere in a row of
+// `pitch` pixels, and the last of them reads (k - 1) rows and (k - 1) pixels further on.
+inline MAFAT_HD int mafat_flat_rows(int mb, int pitch, int k) {
+    return (128 * mb + pitch - 1 + (k - 1) * (pitch + 1) + pitch - 1) / pitch;
+}
+
 // Byte offset of the raw rows inside an A stage (MAFAT_IN_GATHER): after the expanded
 // one-octet halo of rows_box x cols_box pixels, on a 128-byte boundary.
 inline MAFAT_HD int mafat_raw_offset(int rows_box, int cols_box) {
@@ -115,7 +133,7 @@ struct MafatTaskDev {
     int32_t in_y0, in_x0; // map position of buffer pixel (0, 0)
     // conv output rectangle computed by this task (map coordinates, before pooling)
     int32_t cy0, cx0, ch, cw;
-    int32_t nby, nbx;     // M blocks along rows / columns
+    int32_t nby, nbx;     // M blocks along rows / columns (flat stage: blocks of the region, 1)
     // output buffer
     int32_t out_kind;     // MAFAT_BUF_*
     int32_t out_nhwc;     // 1: NHWC (user output), 0: octet-planar
@@ -129,7 +147,7 @@ struct MafatTaskDev {
 
 struct MafatItemDev {
     int32_t task;
-    int16_t by, bx;       // M block
+    int16_t by, bx;       // M block (flat stage: index of the first block in the region, 0)
     int16_t nb;           // output-channel block
     int16_t nbk;          // M blocks of this item (rows by .. by+nbk-1)
     int16_t flags;        // bit 0: do not publish completion (test hook)

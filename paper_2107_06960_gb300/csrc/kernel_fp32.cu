@@ -4,8 +4,9 @@
 // with fp32 activations, weights and accumulation, so that the tiling, the
 // region arithmetic and the dependency chain can be checked against the
 // oracle at a tight tolerance.  One CTA of 128 threads computes one item: a
-// 16 x 8 block of conv output pixels (thread = pixel) for one block of output
-// channels, 8 channels at a time:
+// block of 128 conv output pixels (thread = pixel; a 16 x 8 rectangle, or a run
+// of a flat stage's region) for one block of output channels, 8 channels at a
+// time:
 //   acc[o] = sum_{c, ky, kx} w[o][c][ky][kx] * in[y + ky - p][x + kx - p][c]
 //   z = scale[o] * acc + bias[o];  out = z > 0 ? z : 0.1 z
 // followed, for a fused max-pool, by the 2x2 maximum over neighbouring lanes.
@@ -51,12 +52,19 @@ __global__ void __launch_bounds__(128) mafat_fp32_kernel(const __grid_constant__
                               : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
                                                                 : p.scratch) + tk.out_off;
         const float* w = p.w_f32 + st.w32_off;
-        const int X = tk.cx0 + it.bx * MAFAT_BLK_COLS + c;
         const int k = st.k, kk = st.k * st.k;
         const int o_end = min((it.nb + 1) * st.n_blk, st.cout);
         for (int blk = 0; blk < it.nbk; ++blk)
         for (int o0 = it.nb * st.n_blk; o0 < o_end; o0 += 8) {
-            const int Y = tk.cy0 + (it.by + blk) * MAFAT_BLK_ROWS + r;
+            // pixel of this thread: (r, c) of a 16 x 8 block, or in a flat stage pixel
+            // 128 (by + blk) + tid of the region read row after row, cols_box pixels a row
+            int Y = tk.cy0 + (it.by + blk) * MAFAT_BLK_ROWS + r, X = tk.cx0 + it.bx * MAFAT_BLK_COLS + c;
+            if (st.flat) {
+                const int pf = (it.by + blk) * 128 + tid;
+                const int yy = pf / st.cols_box;
+                Y = tk.cy0 + yy;
+                X = tk.cx0 + (pf - yy * st.cols_box);
+            }
             const bool valid = (Y < tk.cy0 + tk.ch) && (X < tk.cx0 + tk.cw);
             float acc[8];
 #pragma unroll

@@ -409,6 +409,7 @@ struct MmaRec {
     int32_t blob_elems;  // elements of one weight blob
     int32_t sb;          // offset of the item's first channel in the scale / bias arrays
     int32_t n_mid;       // MMA N of the item's (first) convolution
+    int16_t flat_off;    // flat stage: A box pixel of the item's first pixel (< pitch); -1: 16x8 blocks
 };
 
 // What the MMA issuer needs of a chain item's chained 1x1 (N, input chunks, K steps per blob,
@@ -443,6 +444,8 @@ struct EpiRec {
     int16_t chain;           // 1: chain item (first pass turns the 3x3's result into the 1x1's A operand)
     int16_t n_mid;           // chain item: columns of the 3x3's accumulator
     int16_t a_col, out_col;  // chain item: TMEM columns of the 1x1's A operand and of its accumulator
+    int16_t pitch;           // flat stage: row pitch of the region (pixels); 0: 16x8 blocks
+    int16_t flat_by;         // flat stage: the item's first block in the region
 };
 
 // A queue slot: the record of one item, in parts, so that every role copies only its own.
@@ -610,6 +613,7 @@ struct MmaState {
 struct MmaJob {
     uint32_t d_tmem, idesc;
     uint32_t a_plane, a_row, a_step, blk16;  // A: octet-plane and row strides (bytes), K step and block (16-B units)
+    uint32_t a_off16;                        // A: first pixel of the item in the box (16-B units; flat stages)
     uint32_t b_hi, b_half, b_step, blob_bytes, n_blk;
     int k, cols_box, n_chunks, n_bsteps, bpp, P, G, key, ticket, cur_b;
     bool bswz;
@@ -673,7 +677,7 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
         const uint32_t a_base = s.sbase + kOffA + (uint32_t)as * kAStageBytes;
         const uint64_t a_desc0 = smem_desc(a_base, j.a_plane, j.a_row);
         const uint32_t a_hi = (uint32_t)(a_desc0 >> 32);
-        uint32_t a_lo = (uint32_t)a_desc0;  // tap (ky, kx) of the plain form: + ky * cols_box + kx
+        uint32_t a_lo = (uint32_t)a_desc0 + j.a_off16;  // tap (ky, kx) of the plain form: + ky * cols_box + kx
         int kx = 0;
         // paired form: offset (16-byte units) and column of tap 2t, advanced by two taps per blob
         const uint32_t a_base16 = (a_base & 0x3FFFFu) >> 4;
@@ -916,6 +920,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tk = p.tasks[it.task];
                     st = p.stages[it.stage];
                 }
+                // a flat stage's item starts at pixel 128 by of its region read row by row: its A box
+                // starts at that pixel's row, the pixel being flat_off pixels into the box
+                int y_lo = 0, flat_off = -1;
+                if (ticket >= 0 && st.flat) {
+                    const int p0 = it.by * 128;
+                    y_lo = p0 / st.cols_box;
+                    flat_off = p0 - y_lo * st.cols_box;
+                }
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                 q_items[qs] = ticket;
@@ -929,7 +941,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                              tk.out_off;
                     rc.x0 = tk.cx0 + it.bx * MAFAT_BLK_COLS;
                     rc.xlim = tk.cx0 + tk.cw;
-                    rc.y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS;
+                    rc.y0 = flat_off >= 0 ? tk.cy0 : tk.cy0 + it.by * MAFAT_BLK_ROWS;
+                    rc.pitch = (int16_t)(flat_off >= 0 ? st.cols_box : 0);
+                    rc.flat_by = it.by;
                     rc.ylim = tk.cy0 + tk.ch;
                     rc.out_y0 = tk.out_y0;
                     rc.out_x0 = tk.out_x0;
@@ -959,6 +973,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rm.blob_elems = st.blob_elems;
                     rm.sb = st.sb_off + it.nb * st.n_blk;
                     rm.n_mid = st.n_blk;
+                    rm.flat_off = (int16_t)flat_off;
                     rm.chain = (int16_t)chain;
                     rc.n_mid = (int16_t)st.n_blk;
                     rc.chain = (int16_t)chain;
@@ -1017,7 +1032,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int in_mode = tk.in_kind == MAFAT_BUF_USER_IN ? st.in_mode : MAFAT_IN_PLANAR;
                 const int px0 = tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0;  // first halo column
                 const int x0 = px0 * 8;
-                const int y0 = tk.cy0 + it.by * MAFAT_BLK_ROWS - st.pad - tk.in_y0;
+                const int y0 = tk.cy0 + (flat_off >= 0 ? y_lo : it.by * MAFAT_BLK_ROWS) - st.pad - tk.in_y0;
                 const uint32_t a_bytes = (uint32_t)(st.chunk8 * st.rows_box * st.cols_box * 16);
                 bool waited = false;
                 if (it.dep0 >= 0 && !(it.dep0 == ok_idx0 && it.dep0_target <= ok_tgt0)) {
@@ -1163,9 +1178,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
                 j.idesc = instr_desc_bf16((int)j.n_blk, 128);
-                j.a_row = (uint32_t)(j.cols_box * 16);
+                // 8-pixel groups of a block: one halo row apart in a 16x8 block, adjacent in a flat one
+                const int flat_off = wu(mr.flat_off);
+                j.a_row = flat_off >= 0 ? 128u : (uint32_t)(j.cols_box * 16);
                 j.b_half = j.n_blk * 16u;
-                j.blk16 = (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);  // one block down, 16-B units
+                j.blk16 = flat_off >= 0 ? 128u : (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);  // next block, 16-B units
+                j.a_off16 = flat_off >= 0 ? (uint32_t)flat_off : 0u;
                 j.a_step = 2u * (j.a_plane >> 4);                   // next K=16 step: two octet planes
                 // B descriptor: 128-byte swizzled blobs (64 channels per row) or no-swizzle core matrices
                 j.b_hi = j.bswz ? desc_hi_sw128(1024u) : (uint32_t)(smem_desc(0u, j.b_half, 128u) >> 32);
@@ -1393,14 +1411,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (b >= rc.nbk) break;
                 const int q = qi * uw;
-                const int Y = rc.y0 + b * MAFAT_BLK_ROWS + r;
-                const bool valid = (Y < rc.ylim) && (X < rc.xlim);
+                int Y = rc.y0 + b * MAFAT_BLK_ROWS + r, Xb = X;
+                if (rc.pitch > 0) {
+                    // flat stage (never pooled): pixel 128 (flat_by + b) + 32 wq + lane of the
+                    // region read row after row, rc.pitch pixels a row
+                    const int pf = (rc.flat_by + b) * 128 + wq * 32 + lane;
+                    const int yy = pf / rc.pitch;
+                    Y = rc.y0 + yy;
+                    Xb = rc.x0 + (pf - yy * rc.pitch);
+                }
+                const bool valid = (Y < rc.ylim) && (Xb < rc.xlim);
                 // a pooled stage's conv region starts on even rows and columns and has even
                 // extents, so a window's four lanes agree on valid
-                int oy = Y, ox = X;
+                int oy = Y, ox = Xb;
                 if (pool) {
                     oy = Y >> 1;
-                    ox = X >> 1;
+                    ox = Xb >> 1;
                 }
                 const uint32_t pix = (uint32_t)((oy - rc.out_y0) * rc.out_w + (ox - rc.out_x0));
                 EpiDst dst;

@@ -358,11 +358,31 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                 const int next_pad = (net.layers[l + 1].c_out + 15) / 16 * 16;
                 chain_here = cout_pad % 64 == 0 && cout_pad + cout_pad / 2 + next_pad <= 256;
             }
-            // With several frames in flight the SMs are kept busy by the next frame anyway, and a
-            // 1x1 layer's item reads a whole K = c_in halo for few MMAs: there the narrowest block
-            // considered is 128 (608x608, 16 frames: 81.3 against 83.0 us per frame; at one frame
-            // the extra parallelism of N = 64 wins, 117.4 against 121.5 us).
-            const int min_nb = (cfg.batch > 1 && L.k == 1) ? 128 : 64;
+            // Flattened M blocks (MafatStageDev::flat) where they take fewer blocks than 16 x 8
+            // rectangles: convolutions without a fused pool (a pool window's four pixels are
+            // lanes of one warp only in a rectangle), of more than 8 input channels (the
+            // paired-tap form of one-octet inputs keeps rectangles) and outside a chained pair,
+            // whose widest region needs a pitch of at most 32 pixels (a tensor-map box row
+            // holds at most 256 elements, 8 per pixel).
+            int flat_pitch = 0;
+            if (!cfg.rect_blocks && !s.pool && s.cin8 > 1 && !chain_here && !prev_chain) {
+                int pitch = 0;
+                for (const TileInfo& ti : tiles[g])
+                    if (!ti.outs[l].empty()) pitch = std::max(pitch, (ti.outs[l].w() + L.k - 1 + 7) / 8 * 8);
+                int64_t flat_blocks = 0;
+                for (const TileInfo& ti : tiles[g]) flat_blocks += ((int64_t)ti.outs[l].h() * pitch + 127) / 128;
+                if (pitch > 0 && pitch <= 32 && flat_blocks < blocks) {
+                    flat_pitch = pitch;
+                    blocks = flat_blocks;
+                }
+            }
+            s.flat = flat_pitch > 0 ? 1 : 0;
+            // With several frames in flight the SMs are kept busy by the next frame anyway, and an
+            // item reads its whole K = c_in * k * k halo for n_blk channels: there the narrowest
+            // block considered is 128 (608x608, 16 frames: 1x1 layers at N = 64 -> 128, 83.0 ->
+            // 81.3 us per frame; then the flat 3x3 layers after the cut too, 83.5 -> 79.7 us; at
+            // one frame the extra parallelism of N = 64 wins, 117.4 against 121.5 us).
+            const int min_nb = cfg.batch > 1 ? 128 : 64;
             if (chain_here || prev_chain) {
                 s.n_blk = cout_pad;  // every channel of the pixels in one item
             } else if (cfg.fixed_nblk > 0 && cout_pad % cfg.fixed_nblk == 0) {
@@ -393,7 +413,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // form of 8-input-channel layers (narrow N, many small items: their epilogue's
             // fixed cost per item dominates)
             s.mb = std::min(s.mb, s.cin8 == 1 ? MAFAT_MAX_MB_PAIRED : MAFAT_MAX_MB);
-            s.cols_box = MAFAT_BLK_COLS + L.k - 1;
+            s.cols_box = s.flat ? flat_pitch : MAFAT_BLK_COLS + L.k - 1;
             // How the caller's NHWC input reaches the first stage's A halo (tensor-core plans; the
             // fp32 kernel reads NHWC directly).  An image of fewer than 8 channels is read in place
             // as raw rows, which a TMA box needs to be a multiple of 16 bytes; 8 channels are one
@@ -411,7 +431,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             }
             // input octets per A chunk: the largest that fits the A stage with mb blocks
             for (;;) {
-                s.rows_box = MAFAT_BLK_ROWS * s.mb + L.k - 1;
+                s.rows_box = s.flat ? mafat_flat_rows(s.mb, s.cols_box, L.k) : MAFAT_BLK_ROWS * s.mb + L.k - 1;
                 const int row_bytes = s.cols_box * 16 * s.rows_box;
                 if (s.in_mode == MAFAT_IN_GATHER) {
                     // the expanded halo plus the raw rows it is built from share the stage
@@ -662,8 +682,8 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                         tk.cx0 = cr.x0;
                         tk.ch = cr.h();
                         tk.cw = cr.w();
-                        tk.nby = ceil_div(tk.ch, MAFAT_BLK_ROWS);
-                        tk.nbx = ceil_div(tk.cw, MAFAT_BLK_COLS);
+                        tk.nby = st.flat ? ceil_div(tk.ch * st.cols_box, 128) : ceil_div(tk.ch, MAFAT_BLK_ROWS);
+                        tk.nbx = st.flat ? 1 : ceil_div(tk.cw, MAFAT_BLK_COLS);
                         if (s == t.stage_first[g]) {
                             tk.in_kind = g == 0 ? MAFAT_BUF_USER_IN : g == 1 ? MAFAT_BUF_CUT : MAFAT_BUF_MAP;
                             tk.in_tmap = g >= 2 ? stage_tmap[s] : -1;
@@ -967,7 +987,15 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if ((s.cols_box * 16) % 16 != 0) return "TMA inner box not a multiple of 16 bytes";
         if (s.n_blk % 16 != 0 || s.n_blk < 16 || s.n_blk > MAFAT_MAX_NBLK) return "bad MMA N";
         if (s.mb < 1 || s.mb * s.n_blk > 256) return "blocks of an item exceed one TMEM accumulator buffer";
-        if (s.rows_box != MAFAT_BLK_ROWS * s.mb + s.k - 1) return "A box rows do not cover the item";
+        if (s.rows_box != (s.flat ? mafat_flat_rows(s.mb, s.cols_box, s.k) : MAFAT_BLK_ROWS * s.mb + s.k - 1))
+            return "A box rows do not cover the item";
+        if (s.flat) {
+            if (s.pool || s.chain || s.chained || s.paired || s.cin8 < 2 || s.in_mode != MAFAT_IN_PLANAR)
+                return "flat blocks on a pooled, chained, paired-tap or gathered stage";
+            if (s.cols_box % 8 != 0 || s.cols_box < 8) return "flat pitch not a multiple of 8 pixels";
+        } else if (s.cols_box != MAFAT_BLK_COLS + s.k - 1) {
+            return "A box columns do not cover a 16x8 block's taps";
+        }
         if (s.w_off + (int64_t)s.n_nblk * s.n_chunks * s.n_bsteps * s.blob_elems > t.weight_elems)
             return "weight blobs outside the packed weights";
         if (s.n_chunks * s.chunk8 != s.cin8) return "chunks do not cover the input channels";
@@ -1019,6 +1047,9 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         const Layer& L = net.layers[s.layer];
         if (s.chained) return "a chained stage has a task";
         if (last_item[ti] - first_item[ti] + 1 != k.n_items) return "task items not contiguous";
+        if (s.flat ? (k.cw + s.k - 1 > s.cols_box || k.nbx != 1 || k.nby != ceil_div(k.ch * s.cols_box, 128))
+                   : (k.nby != ceil_div(k.ch, MAFAT_BLK_ROWS) || k.nbx != ceil_div(k.cw, MAFAT_BLK_COLS)))
+            return "task blocks do not tile its conv rectangle";
         // input buffer extent and coverage of every in-map tap of the conv rectangle
         const int64_t in_elems = k.in_kind == MAFAT_BUF_USER_IN ? (int64_t)s.cin * k.in_h * k.in_w
                                                                  : (int64_t)s.cin8 * 8 * k.in_h * k.in_w;
@@ -1061,6 +1092,14 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if (it.by >= k.nby || it.bx >= k.nbx || it.nb >= s.n_nblk || it.by < 0 || it.bx < 0 || it.nb < 0)
             return "item block out of range";
         if (it.nbk < 1 || it.nbk > s.mb || it.by + it.nbk > k.nby) return "item block count out of range";
+        if (s.flat) {
+            // every pixel the item's MMAs read (its blocks' 128 pixels at every tap offset) lies
+            // inside the A box that starts at the row of its first pixel
+            const int64_t p0 = (int64_t)it.by * 128, y_lo = p0 / s.cols_box;
+            const int64_t last = p0 - y_lo * s.cols_box + 128 * it.nbk - 1 + (int64_t)(s.k - 1) * (s.cols_box + 1);
+            if (last >= (int64_t)s.rows_box * s.cols_box) return "flat item reads past its A box";
+            if (it.bx != 0) return "flat item with a block column";
+        }
         const int deps[2] = {it.dep0, it.dep1};
         const int tgts[2] = {it.dep0_target, it.dep1_target};
         for (int d = 0; d < 2; ++d) {

@@ -94,6 +94,7 @@ struct PlanConfig {
     int lookahead_items = 0;  // stages with at least this many items take tickets early (0: 5/4 n_ctas, < 0: never)
     bool frame_major = false; // batch > 1: hand frames out one after another, never overlapped
     bool chain = false;       // chain a 3x3 and the 1x1 after it on chip where both fit a TMEM buffer
+    bool rect_blocks = false; // 16x8 rectangular M blocks only (no flattened blocks, MafatStageDev::flat)
     // explicit tile bounds per group (empty: even): rows[g] has grid_n[g] + 1 entries, cols[g] grid_m[g] + 1
     std::vector<int> row_bounds[MAFAT_MAX_GROUPS], col_bounds[MAFAT_MAX_GROUPS];
 };

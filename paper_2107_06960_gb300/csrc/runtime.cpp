@@ -378,6 +378,7 @@ mafat_status mafat_plan_ex(const mafat_net_t* net, int32_t n_groups, const int32
     cfg.halo_reuse = o.halo_reuse != 0;
     cfg.frame_major = o.frame_major != 0;
     cfg.chain = o.chain != 0;
+    cfg.rect_blocks = o.rect_blocks != 0;
     if (o.tile_bounds) {
         // per group: grid_n + 1 row bounds, then grid_m + 1 column bounds
         const int32_t* b = o.tile_bounds;

@@ -128,6 +128,71 @@ def test_bf16_single_layer(mf, cin, cout, k, pool, h, w, grid):
         bad.sum(), bad.size, float(np.abs(got - ref).max()))
 
 
+def _issued(mf, layers, h, w, c, cut, grids, dtype, **kw):
+    net = mf.Net(layers, h, w, c)
+    net.set_params(synth.make_params(layers, c, 1, "fp32"))
+    return mf.Plan(net, cut, grids, dtype=dtype, dry_run=True, **kw).stats()["issued_flops"]
+
+
+@pytest.mark.parametrize("cin,cout,k,h,w,grid,mb", [
+    (64, 64, 3, 40, 14, (1, 1), 0),     # pitch 16: 5 runs of 128 pixels instead of 6 rectangles
+    (256, 512, 3, 38, 38, (2, 2), 0),   # the benchmark's 38x38 3x3 layers: 19x19 regions, pitch 24
+    (512, 256, 1, 38, 38, (2, 2), 0),   # and its 1x1 layers, pitch 24
+    (128, 64, 1, 33, 31, (1, 1), 0),    # pitch 32, a ragged last run
+    (32, 48, 3, 70, 30, (1, 1), 0),     # pitch 32, output channels padded to the MMA N
+    (32, 48, 3, 70, 30, (1, 1), 4),     # four runs per item (one accumulator each)
+    (64, 32, 3, 99, 14, (3, 1), 2),     # two runs per item, 5 runs per task (3 + 2)
+])
+def test_bf16_flat_blocks_match_rectangles_and_oracle(mf, cin, cout, k, h, w, grid, mb):
+    # A convolution without a pool whose regions are narrow reads them as flattened rows
+    # (rect_blocks=False, the default); 16x8 rectangles (rect_blocks=True) compute every
+    # pixel with the same products in the same order, so the outputs are bit-identical.
+    layers = [("conv", k, 1, (k - 1) // 2, cout)]
+    kw = dict(force_mb=mb) if mb else {}
+    assert (_issued(mf, layers, h, w, cin, None, [grid], mf.BF16, **kw) <
+            _issued(mf, layers, h, w, cin, None, [grid], mf.BF16, rect_blocks=True, **kw)), "no flat stage"
+    params = synth.make_params(layers, cin, 3000 + cin + cout + k, "bf16")
+    x = synth.make_input(1, h, w, cin, 4000 + cin, "bf16")
+    _, flat = run_plan(mf, layers, params, x, None, [grid], mf.BF16, plan_kwargs=kw)
+    _, rect = run_plan(mf, layers, params, x, None, [grid], mf.BF16, plan_kwargs=dict(rect_blocks=True, **kw))
+    assert np.array_equal(flat, rect)
+    ref = _oracle_groups(layers, params, x, None)[0][-1]
+    bound = 2.0 ** -8 * np.abs(ref) + 2.0 ** -12 * np.abs(ref).max()
+    bad = np.abs(flat[0] - ref) > bound
+    assert not bad.any(), "%d of %d elements out of bound; worst %.3g" % (
+        bad.sum(), bad.size, float(np.abs(flat[0] - ref).max()))
+
+
+def test_fp32_flat_blocks_match_rectangles_and_oracle(mf):
+    # a 3x3, a 1x1 and a 3x3 on 2x2 tiles of 38x38: 20, 20 and 19-pixel regions run
+    # flattened (pitch 24), the later ones from the tile buffers of the scratch ring, in the
+    # fp32 check kernel as in the bf16 one
+    layers = [("conv", 3, 1, 1, 64), ("conv", 1, 1, 0, 32), ("conv", 3, 1, 1, 32)]
+    assert (_issued(mf, layers, 38, 38, 16, None, [(2, 2)], mf.FP32) <
+            _issued(mf, layers, 38, 38, 16, None, [(2, 2)], mf.FP32, rect_blocks=True))
+    params = synth.make_params(layers, 16, 71, "fp32")
+    x = synth.make_input(2, 38, 38, 16, 72, "fp32")
+    _, flat = run_plan(mf, layers, params, x, None, [(2, 2)], mf.FP32)
+    _, rect = run_plan(mf, layers, params, x, None, [(2, 2)], mf.FP32, plan_kwargs=dict(rect_blocks=True))
+    assert np.array_equal(flat, rect)
+    _check_groups(None, flat, _oracle_groups(layers, params, x, None), None, TOL_FP32)
+    pb = synth.make_params(layers, 16, 73, "bf16")
+    xb = synth.make_input(2, 38, 38, 16, 74, "bf16")
+    _, fb = run_plan(mf, layers, pb, xb, None, [(2, 2)], mf.BF16)
+    _, rb = run_plan(mf, layers, pb, xb, None, [(2, 2)], mf.BF16, plan_kwargs=dict(rect_blocks=True))
+    assert np.array_equal(fb, rb)
+    _check_groups(None, fb, _oracle_groups(layers, pb, xb, None), None, TOL_BF16)
+
+
+def test_bf16_608_flat_matches_rectangles(mf):
+    # the benchmark plan: layers 12-15 (19-20 pixel regions after the cut) run flattened
+    wl = synth.workload("yolo16_608_5x5_c8_2x2")
+    c1, o1 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16)
+    c0, o0 = run_plan(mf, wl["layers"], wl["params"], wl["input"], 8, wl["grids"], mf.BF16,
+                      plan_kwargs=dict(rect_blocks=True))
+    assert np.array_equal(o1, o0) and np.array_equal(c1, c0)
+
+
 # ---------------------------------------------------------------------------
 # bf16 tensor-core path: whole YOLOv2 front-end
 # ---------------------------------------------------------------------------

@@ -138,6 +138,33 @@ def test_headline_plan_numbers(mf):
     assert abs(st["executed_flops"] / st["useful_flops"] - 1.137) < 0.01
 
 
+def test_flat_blocks_cut_block_padding(mf):
+    # 38x38 on a 2x2 grid gives 19x19 conv regions: 2 x 3 rectangles of 16x8 pixels, or the
+    # region's rows laid end to end at a pitch of 24 pixels (19 + 2 halo, rounded up to 8):
+    # 19 * 24 = 456 pixels, 4 runs of 128
+    conv = [("conv", 3, 1, 1, 512)]
+    net = mf.Net(conv, 38, 38, 256)
+    net.set_params(synth.make_params(conv, 256, 1, "bf16"))
+    flat = mf.Plan(net, None, [(2, 2)], dry_run=True).stats()
+    rect = mf.Plan(net, None, [(2, 2)], dry_run=True, rect_blocks=True).stats()
+    mac = 2 * 128 * 512 * 256 * 9
+    assert flat["issued_flops"] == 4 * 4 * mac and rect["issued_flops"] == 4 * 6 * mac
+    assert flat["executed_flops"] == rect["executed_flops"] == 38 * 38 * 512 * 256 * 9 * 2
+    # a convolution with a fused pool keeps its rectangles (a window's pixels must share a warp)
+    pooled = [("conv", 3, 1, 1, 64), ("max", 2, 2, 0, 0)]
+    net = mf.Net(pooled, 76, 76, 128)
+    net.set_params(synth.make_params(pooled, 128, 1, "bf16"))
+    assert (mf.Plan(net, None, [(2, 2)], dry_run=True).stats()["issued_flops"] ==
+            mf.Plan(net, None, [(2, 2)], dry_run=True, rect_blocks=True).stats()["issued_flops"])
+    # the benchmark plan: layers 12-15 (19-20 pixel regions) go from 24 blocks to 16 each
+    wl = synth.WORKLOADS["yolo16_608_5x5_c8_2x2"]
+    net = _net(mf, wl["layers"], 608)
+    a = mf.Plan(net, 8, wl["grids"], dry_run=True).stats()["issued_flops"]
+    b = mf.Plan(net, 8, wl["grids"], dry_run=True, rect_blocks=True).stats()["issued_flops"]
+    saved = 8 * 128 * 2 * (2 * 512 * 256 * 9 + 2 * 256 * 512)
+    assert b - a == saved
+
+
 def test_plan_validation_errors(mf):
     layers = synth.YOLO16
     net = _net(mf, layers, 64)
