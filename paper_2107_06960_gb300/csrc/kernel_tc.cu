@@ -727,9 +727,11 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
             ++g;
             if (--rem == 0) {
                 // end of the buffer's blobs for this item: a streamed piece is released as soon
-                // as its last blob has been issued, and the next piece (if any) is waited for
+                // as its last blob has been issued, and the next piece (if any) is waited for;
+                // a piece that ends with the chunk is followed only after the A stage is
+                // released below, so that the producer can refill the stage meanwhile
                 if (j.P > 1) tc_commit_warp(s.bar(kBarBEmpty + j.cur_b));
-                if (g < j.G) {
+                if (g < j.G && t + 1 < j.n_bsteps) {
                     const uint64_t tp0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
                     mma_begin_piece(s, j);
                     if (s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
@@ -740,6 +742,13 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
         }
         tc_commit_warp(s.bar(kBarAEmpty + as));
         ++s.a_cnt;
+        if (rem == 0 && g < j.G) {
+            const uint64_t tp0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+            mma_begin_piece(s, j);
+            if (s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
+            rem = min(j.bpp, j.G - g);
+            b_lo = b_lo_of(s, j, j.cur_b);
+        }
     }
 }
 
@@ -1004,6 +1013,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_arrive(bar(kBarQFull + qs));  // release: the record is visible to the consumers
                 ++q_cnt;
                 if (ticket < 0) break;
+                // the tensor map of the item's input (a table in global memory, cold after the
+                // launch) into the TMA unit's descriptor cache while the item waits for its inputs
+                if (tk.in_kind != MAFAT_BUF_USER_IN) {
+                    const CUtensorMap* pm = tk.in_kind == MAFAT_BUF_CUT ? p.tmaps + p.cut_tmap : p.tmaps + tk.in_tmap;
+                    asm volatile("prefetch.tensormap [%0];" ::"l"(pm) : "memory");
+                }
                 const int key = tk.stage * 256 + it.nb;
                 const int P = st.n_pieces, G = st.n_chunks * st.n_bsteps;
                 const uint32_t blob_bytes = (uint32_t)(st.blob_elems * 2);
@@ -1159,6 +1174,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int kst = wu(mr.kst), nbk = wu(mr.nbk), paired = wu(mr.paired);
                 const int sb = wu(mr.sb);
                 j.cur_b = j.P == 1 ? ms.wb.resident(j.key) : -1;
+                if (j.P > 1) {
+                    // a streamed set takes both buffers: a resident set held in the one its
+                    // second piece goes to is released now (its MMAs are long done), not when
+                    // that piece is needed, so that the producer can load the piece meanwhile
+                    const int o = ms.wb.next ^ 1;
+                    if (ms.wb.held(o)) {
+                        tc_commit_warp(ms.bar(kBarBEmpty + o));
+                        ms.wb.release(o);
+                    }
+                }
                 if (j.cur_b < 0) mma_begin_piece(ms, j);
                 const int buf = (int)(acc_cnt & 1u);
                 mbar_wait_mma(ms.bar(kBarAccEmpty + buf), ((acc_cnt >> 1) & 1u) ^ 1u, p.ctr, pipe_limit, broken);
