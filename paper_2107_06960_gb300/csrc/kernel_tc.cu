@@ -1069,6 +1069,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (waited) mafat_dev::fence_proxy_async_global();
                 if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
+                int next_pc = 1;  // the next weight piece to load (piece 0 went first)
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
                     const uint32_t a_dst = sbase + kOffA + as * kAStageBytes;
@@ -1086,9 +1087,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tma_load_4d(a_dst, map, x0, y0, c * st.chunk8, c3, bar(kBarAFull + as));
                     }
                     ++a_cnt;
-                    if (P > 1)
-                        for (int g = c * st.n_bsteps; g < (c + 1) * st.n_bsteps; ++g)
-                            if (g > 0 && g % st.bpp == 0) MAFAT_LOAD_PIECE(g / st.bpp);
+                    // the pieces that start inside this chunk (piece pc starts at blob pc * bpp);
+                    // no division: on this single thread, a runtime modulo per blob cost ~1.5 us
+                    // per chunk of a 3x3 256->512 item
+                    while (next_pc < P && next_pc * st.bpp < (c + 1) * st.n_bsteps) {
+                        MAFAT_LOAD_PIECE(next_pc);
+                        ++next_pc;
+                    }
                 }
 #undef MAFAT_LOAD_PIECE
                 if (kChain && st.chain) {
