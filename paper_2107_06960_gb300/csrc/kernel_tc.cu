@@ -591,11 +591,6 @@ __device__ __forceinline__ void prefetch_l2_share(const void* base, int64_t byte
     }
 }
 
-// Byte offset of tap t inside an A halo buffer.
-__device__ __forceinline__ uint32_t tap_off(int t, int k, int cols) {
-    return (uint32_t)(((t / k) * cols + (t % k)) * 16);
-}
-
 // ----------------------------------------------------------------------------- MMA warp
 // State of the MMA warp that lives across items.
 struct MmaState {
@@ -688,14 +683,16 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
             if (PAIRED) {
                 // taps (2t, 2t+1) as the two K halves: LBO = their distance (in the low word's
                 // bits 16-29; the high word, SBO = one halo row, is the plain form's); for an odd
-                // tap count the last blob pairs zero weights with the last tap
+                // tap count (3x3: a 1x1 layer needs more than 8 input channels) the last blob
+                // pairs zero weights with the last tap, the walk's current position, and both
+                // halves read that tap (LBO 0)
                 uint32_t pa, pb;
                 if (2 * t + 1 < taps) {
                     pa = oa16;
                     pb = xa + 1 == j.k ? oa16 + (uint32_t)(j.cols_box - j.k + 1) : oa16 + 1u;
                 } else {
-                    pa = tap_off(taps - 2, j.k, j.cols_box) >> 4;
-                    pb = tap_off(taps - 1, j.k, j.cols_box) >> 4;
+                    pa = oa16;
+                    pb = oa16;
                 }
                 a_lo_t = (a_base16 + pa) | ((pb - pa) << 16);
                 a_hi_t = a_hi;

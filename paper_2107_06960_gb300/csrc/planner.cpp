@@ -1133,7 +1133,8 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
 //    at unit u ^ (n%8) of the row; the tensor core undoes the XOR from the address bits.
 //  - regular stages: blob = tap (ky, kx), K half h of step j = input octet chunk*chunk8 + 2j + h;
 //  - paired stages (8 input channels): blob p holds taps (a, b) = (2p, 2p+1), or for an odd
-//    tap count the last blob holds (zero weights, last tap); K half 0 = tap a, half 1 = tap b.
+//    tap count the last blob holds (zero weights, last tap); K half 0 = tap a, half 1 = tap b
+//    (the kernel points both halves of that last blob at the last tap).
 void pack_weights_bf16(const Net& net, const PlanTables& t, std::vector<uint16_t>& out) {
     out.assign((size_t)t.weight_elems, 0);
     for (const MafatStageDev& s : t.stages) {
