@@ -399,17 +399,20 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Where one thread's epilogue results go: its pixel's element offset in the
-// output buffer (octet-planar: offset inside an 8-channel plane; NHWC: offset
-// of channel 0), the plane stride, and whether this lane stores at all.
-// What the MMA issuer needs of an item (all small).
-struct MmaRec {
-    int16_t k, cols_box, rows_box, n_chunks, n_bsteps, bpp, n_pieces, kst, paired, b_swz, nbk, chain;
-    int32_t key;         // stage * 256 + channel block: identifies a resident weight set
-    int32_t blob_elems;  // elements of one weight blob
-    int32_t sb;          // offset of the item's first channel in the scale / bias arrays
-    int32_t n_mid;       // MMA N of the item's (first) convolution
-    int16_t flat_off;    // flat stage: A box pixel of the item's first pixel (< pitch); -1: 16x8 blocks
+// What the MMA issuer needs of an item, packed in 32-bit words that it reads with three
+// 16-byte shared-memory loads and broadcasts word by word (while the tensor core streams its
+// operands, shared memory is busy: field-by-field loads and broadcasts cost ~0.5 us an item):
+//   w[0] key: stage * 256 + channel block, identifies a resident weight set
+//   w[1] sb: offset of the item's first channel in the scale / bias arrays
+//   w[2] bytes of one weight blob
+//   w[3] n_mid: MMA N of the item's (first) convolution
+//   w[4] k | K steps per blob << 8 | blocks << 16 | paired << 24 | swizzled B << 25 | chain << 26
+//   w[5] A box columns | rows << 16
+//   w[6] input chunks | blobs per chunk << 16
+//   w[7] blobs per weight piece | pieces << 16
+//   w[8] flat stage: A box pixel of the item's first pixel + 1 (0: 16x8 blocks) | box pixels << 16
+struct __align__(16) MmaRec {
+    uint32_t w[12];
 };
 
 // What the MMA issuer needs of a chain item's chained 1x1 (N, input chunks, K steps per blob,
@@ -456,7 +459,11 @@ struct ItemRec {
     GatherRec gather;
 };
 static_assert(sizeof(ItemRec) <= kRecStride, "item record");
+static_assert(kRecStride % 16 == 0 && offsetof(ItemRec, mma) % 16 == 0, "16-byte loads of the MMA record");
 
+// Where one thread's epilogue results go: its pixel's element offset in the
+// output buffer (octet-planar: offset inside an 8-channel plane; NHWC: offset
+// of channel 0), the plane stride, and whether this lane stores at all.
 struct EpiDst {
     __nv_bfloat16* out;
     uint32_t pix, plane;  // element offsets within the output buffer (a frame's region: < 2^31)
@@ -964,23 +971,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.flags = ((chain ? st.c2_pool : st.pool) ? 1 : 0) | (tk.out_nhwc ? 2 : 0) | ((it.flags & 1) ? 4 : 0);
                     rc.done_ctr = tk.done_ctr;
                     rc.extra_ctr = it.extra_ctr;
-                    rm.k = (int16_t)st.k;
-                    rm.cols_box = (int16_t)st.cols_box;
-                    rm.rows_box = (int16_t)st.rows_box;
-                    rm.n_chunks = (int16_t)st.n_chunks;
-                    rm.n_bsteps = (int16_t)st.n_bsteps;
-                    rm.bpp = (int16_t)st.bpp;
-                    rm.n_pieces = (int16_t)st.n_pieces;
-                    rm.kst = (int16_t)st.kst;
-                    rm.paired = (int16_t)st.paired;
-                    rm.b_swz = (int16_t)st.b_swz;
-                    rm.nbk = it.nbk;
-                    rm.key = tk.stage * 256 + it.nb;
-                    rm.blob_elems = st.blob_elems;
-                    rm.sb = st.sb_off + it.nb * st.n_blk;
-                    rm.n_mid = st.n_blk;
-                    rm.flat_off = (int16_t)flat_off;
-                    rm.chain = (int16_t)chain;
+                    {
+                        uint4* w = reinterpret_cast<uint4*>(rm.w);
+                        w[0] = make_uint4((uint32_t)(tk.stage * 256 + it.nb), (uint32_t)(st.sb_off + it.nb * st.n_blk),
+                                          (uint32_t)(st.blob_elems * 2), (uint32_t)st.n_blk);
+                        w[1] = make_uint4((uint32_t)st.k | ((uint32_t)st.kst << 8) | ((uint32_t)it.nbk << 16) |
+                                              ((uint32_t)st.paired << 24) | ((uint32_t)st.b_swz << 25) |
+                                              ((uint32_t)chain << 26),
+                                          (uint32_t)st.cols_box | ((uint32_t)st.rows_box << 16),
+                                          (uint32_t)st.n_chunks | ((uint32_t)st.n_bsteps << 16),
+                                          (uint32_t)st.bpp | ((uint32_t)st.n_pieces << 16));
+                        w[2] = make_uint4((uint32_t)(flat_off + 1) | ((uint32_t)(st.rows_box * st.cols_box) << 16), 0u, 0u,
+                                          0u);
+                    }
                     rc.n_mid = (int16_t)st.n_blk;
                     rc.chain = (int16_t)chain;
                     if (chain) {
@@ -1147,34 +1150,38 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int qs = (int)(q_cnt % kQDepth);
                 mbar_wait_mma(ms.bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken);
                 const int ticket = wu(q_items[qs]);
-                MmaRec mr;
-                int n_blk = 0;
+                uint4 m0 = make_uint4(0u, 0u, 0u, 0u), m1 = m0, m2 = m0;
                 if (ticket >= 0) {
-                    mr = recs[qs].mma;
-                    n_blk = mr.n_mid;  // N of the item's (first) convolution
+                    const uint4* src = reinterpret_cast<const uint4*>(recs[qs].mma.w);
+                    m0 = src[0];
+                    m1 = src[1];
+                    m2 = src[2];
                 }
+                const uint32_t w4 = (uint32_t)wu((int)m1.x);
                 // release the slot once the record has been read (a chain item's slot is held until
                 // its chained 1x1's fields have been read, on the chain path)
-                const bool chain = kChain && ticket >= 0 && wu(mr.chain) != 0;
+                const bool chain = kChain && ticket >= 0 && ((w4 >> 26) & 1u) != 0;
                 if (!chain) mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
                 MmaJob j;
                 j.ticket = ticket;
-                j.k = wu(mr.k);
-                j.cols_box = wu(mr.cols_box);
-                j.n_blk = (uint32_t)wu(n_blk);
-                j.n_chunks = wu(mr.n_chunks);
-                j.n_bsteps = wu(mr.n_bsteps);
-                j.bpp = wu(mr.bpp);
-                j.P = wu(mr.n_pieces);
+                const uint32_t w5 = (uint32_t)wu((int)m1.y), w6 = (uint32_t)wu((int)m1.z), w7 = (uint32_t)wu((int)m1.w);
+                const uint32_t w8 = (uint32_t)wu((int)m2.x);
+                j.k = (int)(w4 & 0xFFu);
+                j.cols_box = (int)(w5 & 0xFFFFu);
+                j.n_blk = (uint32_t)wu((int)m0.w);
+                j.n_chunks = (int)(w6 & 0xFFFFu);
+                j.n_bsteps = (int)(w6 >> 16);
+                j.bpp = (int)(w7 & 0xFFFFu);
+                j.P = (int)(w7 >> 16);
                 j.G = j.n_chunks * j.n_bsteps;
-                j.key = wu(mr.key);
-                j.blob_bytes = (uint32_t)wu(mr.blob_elems * 2);
-                j.a_plane = (uint32_t)wu(mr.rows_box * mr.cols_box * 16);
-                j.bswz = wu(mr.b_swz) != 0;
-                const int kst = wu(mr.kst), nbk = wu(mr.nbk), paired = wu(mr.paired);
-                const int sb = wu(mr.sb);
+                j.key = wu((int)m0.x);
+                j.blob_bytes = (uint32_t)wu((int)m0.z);
+                j.a_plane = (w8 >> 16) * 16u;
+                j.bswz = ((w4 >> 25) & 1u) != 0;
+                const int kst = (int)((w4 >> 8) & 0xFFu), nbk = (int)((w4 >> 16) & 0xFFu), paired = (int)((w4 >> 24) & 1u);
+                const int sb = wu((int)m0.y);
                 j.cur_b = j.P == 1 ? ms.wb.resident(j.key) : -1;
                 if (j.P > 1) {
                     // a streamed set takes both buffers: a resident set held in the one its
@@ -1206,7 +1213,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
                 j.idesc = instr_desc_bf16((int)j.n_blk, 128);
                 // 8-pixel groups of a block: one halo row apart in a 16x8 block, adjacent in a flat one
-                const int flat_off = wu(mr.flat_off);
+                const int flat_off = (int)(w8 & 0xFFFFu) - 1;
                 j.a_row = flat_off >= 0 ? 128u : (uint32_t)(j.cols_box * 16);
                 j.b_half = j.n_blk * 16u;
                 j.blk16 = flat_off >= 0 ? 128u : (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);  // next block, 16-B units
@@ -1308,9 +1315,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             int n_chunks = 0, rows = 0, cols = 0;
             if (ticket >= 0) {
                 g = recs[qs].gather;
-                n_chunks = recs[qs].mma.n_chunks;
-                rows = recs[qs].mma.rows_box;
-                cols = recs[qs].mma.cols_box;
+                const uint32_t w5 = recs[qs].mma.w[5], w6 = recs[qs].mma.w[6];
+                n_chunks = (int)(w6 & 0xFFFFu);
+                rows = (int)(w5 >> 16);
+                cols = (int)(w5 & 0xFFFFu);
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
