@@ -400,8 +400,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 }
 
 // What the MMA issuer needs of an item, packed in 32-bit words that it reads with three
-// 16-byte shared-memory loads and broadcasts word by word (while the tensor core streams its
-// operands, shared memory is busy: field-by-field loads and broadcasts cost ~0.5 us an item):
+// 16-byte shared-memory loads and broadcasts word by word (the read is on the MMA warp's
+// path between items, while the tensor core keeps shared memory busy with its operands):
 //   w[0] key: stage * 256 + channel block, identifies a resident weight set
 //   w[1] sb: offset of the item's first channel in the scale / bias arrays
 //   w[2] bytes of one weight blob
