@@ -163,6 +163,43 @@ def test_bf16_flat_blocks_match_rectangles_and_oracle(mf, cin, cout, k, h, w, gr
         bad.sum(), bad.size, float(np.abs(flat[0] - ref).max()))
 
 
+def test_bf16_flat_blocks_random_shapes(mf):
+    # seeded random single convolutions (1x1 and 3x3, channel counts, map sizes, grids and
+    # forced blocks per item) among those that the planner runs in flat blocks: bit-identical
+    # to 16x8 rectangles and within the per-element bf16 bound of the oracle
+    rng = np.random.default_rng(2107)
+    done = 0
+    for _ in range(2000):
+        if done == 10:
+            break
+        cin = int(rng.choice([16, 32, 64, 128]))
+        cout = int(rng.choice([16, 48, 64, 96, 128]))
+        k = int(rng.choice([1, 3]))
+        h, w = int(rng.integers(8, 72)), int(rng.integers(5, 40))
+        grid = [(1, 1), (2, 1), (1, 2), (2, 2), (3, 2)][int(rng.integers(0, 5))]
+        mb = int(rng.choice([0, 0, 2, 4]))
+        layers = [("conv", k, 1, (k - 1) // 2, cout)]
+        kw = dict(force_mb=mb) if mb else {}
+        try:
+            flat_work = _issued(mf, layers, h, w, cin, None, [grid], mf.BF16, **kw)
+            rect_work = _issued(mf, layers, h, w, cin, None, [grid], mf.BF16, rect_blocks=True, **kw)
+        except mf.MafatError:
+            continue  # a shape the planner refuses (e.g. more blocks per item than fit)
+        if flat_work >= rect_work:
+            continue
+        params = synth.make_params(layers, cin, 5000 + done, "bf16")
+        x = synth.make_input(1, h, w, cin, 6000 + done, "bf16")
+        _, flat = run_plan(mf, layers, params, x, None, [grid], mf.BF16, plan_kwargs=kw)
+        _, rect = run_plan(mf, layers, params, x, None, [grid], mf.BF16, plan_kwargs=dict(rect_blocks=True, **kw))
+        case = (cin, cout, k, h, w, grid, mb)
+        assert np.array_equal(flat, rect), case
+        ref = _oracle_groups(layers, params, x, None)[0][-1]
+        bound = 2.0 ** -8 * np.abs(ref) + 2.0 ** -12 * np.abs(ref).max()
+        assert not (np.abs(flat[0] - ref) > bound).any(), case
+        done += 1
+    assert done == 10
+
+
 def test_fp32_flat_blocks_match_rectangles_and_oracle(mf):
     # a 3x3, a 1x1 and a 3x3 on 2x2 tiles of 38x38: 20, 20 and 19-pixel regions run
     # flattened (pitch 24), the later ones from the tile buffers of the scratch ring, in the
