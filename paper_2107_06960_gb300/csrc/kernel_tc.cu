@@ -656,7 +656,7 @@ __device__ __forceinline__ uint32_t b_lo_of(const MmaState& s, const MmaJob& j, 
 // sharing the SM, a loop that rebuilt the B descriptor and tested the piece bounds
 // twice per blob issued N=64 MMAs every ~87 cycles; this form every ~52 (the shared
 // memory bound of a 128x64x16 MMA is ~49).
-template <int KST, int NBK, bool PAIRED>
+template <int KST, int NBK, bool PAIRED, bool TR>
 __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     uint32_t accumulate = 0;
     int g = 0;                        // blob index within the weight set
@@ -666,9 +666,9 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     const int taps = j.k * j.k;
     for (int c = 0; c < j.n_chunks; ++c) {
         const int as = (int)(s.a_cnt % kAStages);
-        const uint64_t tw0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+        const uint64_t tw0 = (TR && s.trace) ? mafat_dev::globaltimer_ns() : 0;
         mbar_wait_mma(s.bar(kBarAFull + as), (s.a_cnt / kAStages) & 1u, s.ctr, s.pipe_limit, s.broken);
-        if (s.trace) {  // every lane stores (one value wins): no branch on the lane
+        if (TR && s.trace) {  // every lane stores (one value wins): no branch on the lane
             const uint64_t tw1 = mafat_dev::globaltimer_ns();
             if (c > 0)
                 j.wait_a += tw1 - tw0;
@@ -736,9 +736,9 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
                 // released below, so that the producer can refill the stage meanwhile
                 if (j.P > 1) tc_commit_warp(s.bar(kBarBEmpty + j.cur_b));
                 if (g < j.G && t + 1 < j.n_bsteps) {
-                    const uint64_t tp0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+                    const uint64_t tp0 = (TR && s.trace) ? mafat_dev::globaltimer_ns() : 0;
                     mma_begin_piece(s, j);
-                    if (s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
+                    if (TR && s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
                     rem = min(j.bpp, j.G - g);
                     b_lo = b_lo_of(s, j, j.cur_b);
                 }
@@ -747,9 +747,9 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
         tc_commit_warp(s.bar(kBarAEmpty + as));
         ++s.a_cnt;
         if (rem == 0 && g < j.G) {
-            const uint64_t tp0 = s.trace ? mafat_dev::globaltimer_ns() : 0;
+            const uint64_t tp0 = (TR && s.trace) ? mafat_dev::globaltimer_ns() : 0;
             mma_begin_piece(s, j);
-            if (s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
+            if (TR && s.trace) j.wait_b += mafat_dev::globaltimer_ns() - tp0;
             rem = min(j.bpp, j.G - g);
             b_lo = b_lo_of(s, j, j.cur_b);
         }
@@ -833,8 +833,10 @@ __device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, in
 }
 
 // kChain: the instance for plans with chain stages; plans without them run the instance
-// compiled without that path.
-template <bool kChain>
+// compiled without that path.  kTrace: the instance that records the per-item trace (plans
+// made with trace = 1); the others carry none of its code (measured on GB300: with the
+// trace code present but switched off, the 608x608 frame took 2.4 us longer).
+template <bool kChain, bool kTrace>
 __global__ void __launch_bounds__(kThreads, 1)
     mafat_tc_kernel(const __grid_constant__ MafatKParams p, const __grid_constant__ CUtensorMap in_map) {
     extern __shared__ uint8_t smem_raw[];
@@ -849,6 +851,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int64_t pipe_limit = 4 * p.timeout_ns + 1000000000LL;
+    unsigned long long* const trace = kTrace ? p.trace : nullptr;
     // the producer's first item record, in flight while the CTA sets up
     MafatItemDev it_first{};
     if (warp == kProducerWarp && lane == 0 && (int)blockIdx.x < p.n_items) it_first = p.items[blockIdx.x];
@@ -923,9 +926,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             while (true) {
                 const int ticket = next < p.n_items ? next : -1;
                 const MafatItemDev it = it_next;
-                if (ticket >= 0 && p.trace) {
-                    mafat_dev::trace_put(p.trace, ticket, 0, mafat_dev::globaltimer_ns());
-                    mafat_dev::trace_put(p.trace, ticket, 4, mafat_dev::smid());
+                if (ticket >= 0 && trace) {
+                    mafat_dev::trace_put(trace, ticket, 0, mafat_dev::globaltimer_ns());
+                    mafat_dev::trace_put(trace, ticket, 4, mafat_dev::smid());
                 }
                 MafatTaskDev tk;
                 MafatStageDev st;
@@ -1068,7 +1071,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     waited = true;
                 }
                 if (waited) mafat_dev::fence_proxy_async_global();
-                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 1, mafat_dev::globaltimer_ns());
+                if (trace) mafat_dev::trace_put(trace, ticket, 1, mafat_dev::globaltimer_ns());
                 int next_pc = 1;  // the next weight piece to load (piece 0 went first)
                 for (int c = 0; c < st.n_chunks; ++c) {
                     const int as = (int)(a_cnt % kAStages);
@@ -1141,7 +1144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ms.ctr = p.ctr;
             ms.pipe_limit = pipe_limit;
             ms.broken = broken;
-            ms.trace = p.trace;
+            ms.trace = trace;
             const uint32_t tmem_u = (uint32_t)wu((int)tmem_base);
             uint32_t q_cnt = 0, acc_cnt = 0;
             uint32_t mid_ph0 = 0, mid_ph1 = 0;  // MidFull phases consumed, per accumulator buffer
@@ -1227,7 +1230,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // one jump per item into the instance for its shape
                 switch ((paired << 8) | (kst << 4) | nbk) {
 #define MAFAT_MMA_CASE(PA, K, B) \
-    case ((PA) << 8) | ((K) << 4) | (B): mma_item<K, B, PA>(ms, j); break;
+    case ((PA) << 8) | ((K) << 4) | (B): mma_item<K, B, PA, kTrace>(ms, j); break;
                     MAFAT_MMA_CASE(0, 4, 1) MAFAT_MMA_CASE(0, 4, 2) MAFAT_MMA_CASE(0, 4, 3) MAFAT_MMA_CASE(0, 4, 4)
                     MAFAT_MMA_CASE(0, 2, 1) MAFAT_MMA_CASE(0, 2, 2) MAFAT_MMA_CASE(0, 2, 3) MAFAT_MMA_CASE(0, 2, 4)
                     MAFAT_MMA_CASE(0, 1, 1) MAFAT_MMA_CASE(0, 1, 2) MAFAT_MMA_CASE(0, 1, 3) MAFAT_MMA_CASE(0, 1, 4)
@@ -1240,10 +1243,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                 }
                 issued = true;
-                if (p.trace) {
-                    mafat_dev::trace_put(p.trace, ticket, 7, mafat_dev::globaltimer_ns());
-                    mafat_dev::trace_put(p.trace, ticket, 8, j.wait_a);
-                    mafat_dev::trace_put(p.trace, ticket, 9, j.wait_b);
+                if (trace) {
+                    mafat_dev::trace_put(trace, ticket, 7, mafat_dev::globaltimer_ns());
+                    mafat_dev::trace_put(trace, ticket, 8, j.wait_a);
+                    mafat_dev::trace_put(trace, ticket, 9, j.wait_b);
                 }
                 if (chain) {
                     // chain item: the 3x3's accumulator goes to the epilogue, which writes its activated
@@ -1292,7 +1295,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int es = (int)(e_cnt & 1u);
                 mbar_wait(bar(kBarEpiDone + es), (e_cnt >> 1) & 1u, p.ctr, pipe_limit, broken, 32);
                 if (!(flags & 4)) mafat_dev::publish_counters(p.ctr, done_ctr, extra_ctr);
-                if (p.trace) mafat_dev::trace_put(p.trace, ticket, 3, mafat_dev::globaltimer_ns());
+                if (trace) mafat_dev::trace_put(trace, ticket, 3, mafat_dev::globaltimer_ns());
                 mbar_arrive(bar(kBarPubDone + es));
                 ++e_cnt;
             }
@@ -1392,7 +1395,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int buf = (int)(acc_cnt & 1u);
             // completes once the item's MMAs are done and its scale / bias have landed
             mbar_wait(bar(kBarAccFull + buf), (buf ? full_ph1++ : full_ph0++) & 1u, p.ctr, pipe_limit, broken, 128);
-            if (p.trace && threadIdx.x == 0) mafat_dev::trace_put(p.trace, ticket, 2, mafat_dev::globaltimer_ns());
+            if (trace && threadIdx.x == 0) mafat_dev::trace_put(trace, ticket, 2, mafat_dev::globaltimer_ns());
             __syncwarp();
             tc_fence_after();
 
@@ -1597,21 +1600,29 @@ __global__ void __launch_bounds__(128, 1)
 
 size_t mafat_tc_smem_bytes() { return (size_t)kSmemBytes; }
 
-cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, bool chain, cudaStream_t s) {
-    static bool attr_set[2] = {false, false};
-    if (!attr_set[chain]) {
-        cudaError_t e = chain ? cudaFuncSetAttribute(mafat_tc_kernel<true>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes)
-                              : cudaFuncSetAttribute(mafat_tc_kernel<false>,
-                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+namespace {
+template <bool kChain, bool kTrace>
+cudaError_t launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, cudaStream_t s) {
+    // the large dynamic shared memory is opted into once per device
+    static bool attr_set[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+        e = cudaFuncSetAttribute(mafat_tc_kernel<kChain, kTrace>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmemBytes);
         if (e != cudaSuccess) return e;
-        attr_set[chain] = true;
+        if (dev >= 0 && dev < 64) attr_set[dev] = true;
     }
-    if (chain)
-        mafat_tc_kernel<true><<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
-    else
-        mafat_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
+    mafat_tc_kernel<kChain, kTrace><<<grid, kThreads, kSmemBytes, s>>>(p, in_map);
     return cudaGetLastError();
+}
+}  // namespace
+
+cudaError_t mafat_launch_tc(const MafatKParams& p, const CUtensorMap& in_map, int grid, bool chain, cudaStream_t s) {
+    const bool trace = p.trace != nullptr;
+    if (chain) return trace ? launch_tc<true, true>(p, in_map, grid, s) : launch_tc<true, false>(p, in_map, grid, s);
+    return trace ? launch_tc<false, true>(p, in_map, grid, s) : launch_tc<false, false>(p, in_map, grid, s);
 }
 
 cudaError_t mafat_launch_diag_umma(const void* a, const void* b, float* d, int n, int a_tmem, cudaStream_t s) {
