@@ -756,6 +756,32 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     }
 }
 
+// Widening of raw rows of c < 8 channels (other than the RGB fast path), pixel by pixel
+// (idx = r * cols + x dealt to the lanes); out of line, as it is off the common path.
+__device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage, int rows, int cols, int raw_e,
+                                            int s0, int c, int lane) {
+    const uint16_t* raw = reinterpret_cast<const uint16_t*>(raw_b);
+    uint4* dst = reinterpret_cast<uint4*>(stage);
+    int r = 0, x = lane;
+    while (x >= cols) {
+        x -= cols;
+        ++r;
+    }
+    for (int idx = lane; idx < rows * cols; idx += 32) {
+        const uint16_t* src = raw + r * raw_e + s0 + x * c;
+        uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int ch = 0; ch < 7; ++ch)
+            if (ch < c) w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
+        dst[idx] = make_uint4(w[0], w[1], w[2], w[3]);
+        x += 32;
+        while (x >= cols) {
+            x -= cols;
+            ++r;
+        }
+    }
+}
+
 // The chained 1x1 of a chain item: A = the 3x3's activated bf16 result in TMEM (columns
 // acc + a_col .., 8 per K=16 step), B = the 1x1's weights streamed through the two
 // buffers piece by piece (never resident), D = TMEM columns acc + out_col .., N = n2.  The
@@ -1344,27 +1370,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         default: break;
                     }
                 } else {
-                    // other channel counts: pixel by pixel (idx = r * cols + x dealt to the lanes)
-                    const uint16_t* raw = reinterpret_cast<const uint16_t*>(raw_b);
-                    uint4* dst = reinterpret_cast<uint4*>(stage);
-                    int r = 0, x = lane;
-                    while (x >= cols) {
-                        x -= cols;
-                        ++r;
-                    }
-                    for (int idx = lane; idx < rows * cols; idx += 32) {
-                        const uint16_t* src = raw + r * g.raw_e + g.s0 + x * g.c;
-                        uint32_t w[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                        for (int ch = 0; ch < 7; ++ch)
-                            if (ch < g.c) w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
-                        dst[idx] = make_uint4(w[0], w[1], w[2], w[3]);
-                        x += 32;
-                        while (x >= cols) {
-                            x -= cols;
-                            ++r;
-                        }
-                    }
+                    gather_generic(raw_b, stage, rows, cols, g.raw_e, g.s0, g.c, lane);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
