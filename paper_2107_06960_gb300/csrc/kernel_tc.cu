@@ -109,31 +109,31 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-// One elected lane of the converged warp adds 2 x bytes to the current phase of bar's
-// expected transactions (without arriving) and copies bytes of scale and of bias into
-// the slot (bias at slot + MAFAT_MAX_NBLK floats), completing on bar.  No branch on the
-// lane: the MMA warp stays converged.
-__device__ __forceinline__ void sb_load_elect(uint32_t bar, uint32_t slot, const float* scale, const float* bias,
-                                              uint32_t bytes) {
+// The lane with el = 1 (one lane of the converged warp, from elect_one) adds 2 x bytes to
+// the current phase of bar's expected transactions (without arriving) and copies bytes of
+// scale and of bias into the slot (bias at slot + MAFAT_MAX_NBLK floats), completing on
+// bar.  No branch on the lane: the MMA warp stays converged.
+__device__ __forceinline__ void sb_load_el(uint32_t el, uint32_t bar, uint32_t slot, const float* scale,
+                                           const float* bias, uint32_t bytes) {
     asm volatile(
         "{\n\t.reg .pred e;\n\t.reg .b32 tx;\n\t"
-        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 e, %6, 0;\n\t"
         "add.u32 tx, %4, %4;\n\t"
         "@e mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], tx;\n\t"
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%1], [%2], %4, [%0];\n\t"
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%5], [%3], %4, [%0];\n\t}" ::"r"(bar),
-        "r"(slot), "l"(scale), "l"(bias), "r"(bytes), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4))
+        "r"(slot), "l"(scale), "l"(bias), "r"(bytes), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4)), "r"(el)
         : "memory");
 }
 
 // The same for a chain item: the 3x3's n1 channels at slot offset 0 and the chained 1x1's n2
 // at slot offset n1 (scale and bias halves alike), all completing on bar.
-__device__ __forceinline__ void sb_load2_elect(uint32_t bar, uint32_t slot, const float* scale1, const float* bias1,
-                                               uint32_t bytes1, const float* scale2, const float* bias2,
-                                               uint32_t bytes2) {
+__device__ __forceinline__ void sb_load2_el(uint32_t el, uint32_t bar, uint32_t slot, const float* scale1,
+                                            const float* bias1, uint32_t bytes1, const float* scale2,
+                                            const float* bias2, uint32_t bytes2) {
     asm volatile(
         "{\n\t.reg .pred e;\n\t.reg .b32 tx;\n\t"
-        "elect.sync _|e, 0xffffffff;\n\t"
+        "setp.ne.b32 e, %11, 0;\n\t"
         "add.u32 tx, %4, %7;\n\t"
         "add.u32 tx, tx, tx;\n\t"
         "@e mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], tx;\n\t"
@@ -142,7 +142,8 @@ __device__ __forceinline__ void sb_load2_elect(uint32_t bar, uint32_t slot, cons
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%9], [%5], %7, [%0];\n\t"
         "@e cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%10], [%6], %7, [%0];\n\t}" ::"r"(bar),
         "r"(slot), "l"(scale1), "l"(bias1), "r"(bytes1), "l"(scale2), "l"(bias2), "r"(bytes2),
-        "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4)), "r"(slot + bytes1), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4) + bytes1)
+        "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4)), "r"(slot + bytes1), "r"(slot + (uint32_t)(MAFAT_MAX_NBLK * 4) + bytes1),
+        "r"(el)
         : "memory");
 }
 
@@ -220,10 +221,11 @@ __device__ __forceinline__ void mbar_wait_mma(uint32_t bar, uint32_t parity, uin
     }
 }
 
-__device__ __forceinline__ void mbar_arrive_elect(uint32_t bar) {
+// An arrive on bar by the lane with el = 1 (from elect_one).
+__device__ __forceinline__ void mbar_arrive_el(uint32_t el, uint32_t bar) {
     asm volatile(
-        "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
-        "@e mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}" ::"r"(bar)
+        "{\n\t.reg .pred e;\n\tsetp.ne.b32 e, %1, 0;\n\t"
+        "@e mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}" ::"r"(bar), "r"(el)
         : "memory");
 }
 
@@ -266,6 +268,26 @@ __device__ __forceinline__ void tc_commit_warp(uint32_t bar) {
         "elect.sync _|e, 0xffffffff;\n\t"
         "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(bar)
         : "memory");
+}
+
+// tcgen05.commit and the A-in-tensor-memory MMA with the issuing lane chosen beforehand
+// (el from elect_one), as mma_el.
+__device__ __forceinline__ void tc_commit_el(uint32_t el, uint32_t bar) {
+    asm volatile(
+        "{\n\t.reg .pred e;\n\t"
+        "setp.ne.b32 e, %0, 0;\n\t"
+        "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%1];\n\t}" ::"r"(el), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void mma_tmem_a_el(uint32_t el, uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo,
+                                              uint32_t b_hi, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t.reg .b64 db;\n\t"
+        "setp.ne.b32 e, %0, 0;\n\t"
+        "setp.ne.b32 p, %6, 0;\n\t"
+        "mov.b64 db, {%3, %4};\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%1], [%2], db, %5, p;\n\t}" ::"r"(el), "r"(d_tmem),
+        "r"(a_tmem), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
 }
 
 // Shared-memory matrix descriptor, no swizzle: start >> 4 in bits 0-13, LBO >> 4
@@ -329,6 +351,28 @@ __device__ __forceinline__ void mma_lo(uint32_t d_tmem, uint32_t a_lo, uint32_t 
         "mov.b64 da, {%1, %2};\n\t"
         "mov.b64 db, {%3, %4};\n\t"
         "@e tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %5, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
+}
+
+// Picks one lane of the converged warp (the same lane on every call) as 1, the others 0.
+__device__ __forceinline__ uint32_t elect_one() {
+    uint32_t el;
+    asm volatile("{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\tselp.u32 %0, 1, 0, e;\n\t}" : "=r"(el));
+    return el;
+}
+
+// mma_lo with the issuing lane chosen beforehand (el from elect_one, taken once when the
+// MMA warp starts): measured on GB300, an elect.sync per MMA cost ~3.5 % of the one-frame
+// launch against this form.
+__device__ __forceinline__ void mma_el(uint32_t el, uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo,
+                                       uint32_t b_hi, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p, e;\n\t.reg .b64 da, db;\n\t"
+        "setp.ne.b32 e, %0, 0;\n\t"
+        "setp.ne.b32 p, %7, 0;\n\t"
+        "mov.b64 da, {%2, %3};\n\t"
+        "mov.b64 db, {%4, %5};\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%1], da, db, %6, p;\n\t}" ::"r"(el), "r"(d_tmem),
         "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(idesc), "r"(accumulate));
 }
 
@@ -608,6 +652,7 @@ struct MmaState {
     int64_t pipe_limit;
     volatile int* broken;
     unsigned long long* trace;
+    uint32_t el;                    // 1 on the lane that issues tensor-core operations
     __device__ __forceinline__ uint32_t bar(int i) const { return sbase + (uint32_t)(i * 8); }
 };
 
@@ -628,7 +673,7 @@ __device__ __forceinline__ void mma_begin_piece(MmaState& s, MmaJob& j) {
     const int b = s.wb.next;
     s.wb.next ^= 1;
     if (s.wb.held(b)) {
-        tc_commit_warp(s.bar(kBarBEmpty + b));
+        tc_commit_el(s.el, s.bar(kBarBEmpty + b));
         s.wb.release(b);
     }
     mbar_wait_mma(s.bar(kBarBFull + b), s.wb.loads(b) & 1u, s.ctr, s.pipe_limit, s.broken);
@@ -713,12 +758,16 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
                 a_lo_t = a_lo;
                 a_hi_t = a_hi;
             }
+            {
+                const uint32_t el = s.el;
 #pragma unroll
-            for (int q = 0; q < KST; ++q)
+                for (int q = 0; q < KST; ++q)
 #pragma unroll
-                for (int b = 0; b < NBK; ++b)
-                    mma_lo(j.d_tmem + (uint32_t)b * j.n_blk, a_lo_t + (uint32_t)q * j.a_step + (uint32_t)b * j.blk16,
-                           a_hi_t, b_lo + (uint32_t)q * j.b_step, j.b_hi, j.idesc, q == 0 ? accumulate : 1u);
+                    for (int b = 0; b < NBK; ++b)
+                        mma_el(el, j.d_tmem + (uint32_t)b * j.n_blk,
+                               a_lo_t + (uint32_t)q * j.a_step + (uint32_t)b * j.blk16, a_hi_t,
+                               b_lo + (uint32_t)q * j.b_step, j.b_hi, j.idesc, q == 0 ? accumulate : 1u);
+            }
             accumulate = 1;
             b_lo += blob16;
             if (!PAIRED) {
@@ -734,7 +783,7 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
                 // as its last blob has been issued, and the next piece (if any) is waited for;
                 // a piece that ends with the chunk is followed only after the A stage is
                 // released below, so that the producer can refill the stage meanwhile
-                if (j.P > 1) tc_commit_warp(s.bar(kBarBEmpty + j.cur_b));
+                if (j.P > 1) tc_commit_el(s.el, s.bar(kBarBEmpty + j.cur_b));
                 if (g < j.G && t + 1 < j.n_bsteps) {
                     const uint64_t tp0 = (TR && s.trace) ? mafat_dev::globaltimer_ns() : 0;
                     mma_begin_piece(s, j);
@@ -744,7 +793,7 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
                 }
             }
         }
-        tc_commit_warp(s.bar(kBarAEmpty + as));
+        tc_commit_el(s.el, s.bar(kBarAEmpty + as));
         ++s.a_cnt;
         if (rem == 0 && g < j.G) {
             const uint64_t tp0 = (TR && s.trace) ? mafat_dev::globaltimer_ns() : 0;
@@ -801,7 +850,7 @@ __device__ __forceinline__ void mma_chain_1x1(MmaState& s, uint32_t acc, int n2,
         const int b = s.wb.next;
         s.wb.next ^= 1;
         if (s.wb.held(b)) {
-            tc_commit_warp(s.bar(kBarBEmpty + b));
+            tc_commit_el(s.el, s.bar(kBarBEmpty + b));
             s.wb.release(b);
         }
         mbar_wait_mma(s.bar(kBarBFull + b), s.wb.loads(b) & 1u, s.ctr, s.pipe_limit, s.broken);
@@ -812,13 +861,13 @@ __device__ __forceinline__ void mma_chain_1x1(MmaState& s, uint32_t acc, int n2,
         const int nb = min(bpp2, nch2 - g);
         for (int k = 0; k < nb; ++k, ++g) {
             for (int q = 0; q < kst2; ++q) {
-                mma_tmem_a(d, a, b_lo + (uint32_t)q * b_step, b_hi, idesc, accumulate);
+                mma_tmem_a_el(s.el, d, a, b_lo + (uint32_t)q * b_step, b_hi, idesc, accumulate);
                 accumulate = 1u;
                 a += 8u;
             }
             b_lo += blob16;
         }
-        tc_commit_warp(s.bar(kBarBEmpty + b));  // the piece is free once these MMAs are done
+        tc_commit_el(s.el, s.bar(kBarBEmpty + b));  // the piece is free once these MMAs are done
     }
 }
 
@@ -1171,6 +1220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ms.pipe_limit = pipe_limit;
             ms.broken = broken;
             ms.trace = trace;
+            ms.el = elect_one();
             const uint32_t tmem_u = (uint32_t)wu((int)tmem_base);
             uint32_t q_cnt = 0, acc_cnt = 0;
             uint32_t mid_ph0 = 0, mid_ph1 = 0;  // MidFull phases consumed, per accumulator buffer
@@ -1190,7 +1240,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // release the slot once the record has been read (a chain item's slot is held until
                 // its chained 1x1's fields have been read, on the chain path)
                 const bool chain = kChain && ticket >= 0 && ((w4 >> 26) & 1u) != 0;
-                if (!chain) mbar_arrive_elect(ms.bar(kBarQEmpty + qs));
+                if (!chain) mbar_arrive_el(ms.el, ms.bar(kBarQEmpty + qs));
                 ++q_cnt;
                 if (ticket < 0) break;
                 MmaJob j;
@@ -1218,7 +1268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // that piece is needed, so that the producer can load the piece meanwhile
                     const int o = ms.wb.next ^ 1;
                     if (ms.wb.held(o)) {
-                        tc_commit_warp(ms.bar(kBarBEmpty + o));
+                        tc_commit_el(ms.el, ms.bar(kBarBEmpty + o));
                         ms.wb.release(o);
                     }
                 }
@@ -1233,10 +1283,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t slot = ms.sbase + (uint32_t)(kOffSb + buf * kSbSlotBytes);
                     if (chain) {
                         const int sb2 = wu(recs[qs].chain.sb2);
-                        sb_load2_elect(ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u,
+                        sb_load2_el(ms.el, ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u,
                                        p.scale + sb2, p.bias + sb2, (uint32_t)wu(recs[qs].chain.n2) * 4u);
                     } else {
-                        sb_load_elect(ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u);
+                        sb_load_el(ms.el, ms.bar(kBarAccFull + buf), slot, p.scale + sb, p.bias + sb, j.n_blk * 4u);
                     }
                 }
                 j.d_tmem = tmem_u + (uint32_t)(buf * kAccStride);
@@ -1277,21 +1327,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (chain) {
                     // chain item: the 3x3's accumulator goes to the epilogue, which writes its activated
                     // bf16 result back into TMEM; the chained 1x1 then runs from there
-                    tc_commit_warp(ms.bar(kBarAccFull + buf));
+                    tc_commit_el(ms.el, ms.bar(kBarAccFull + buf));
                     const ChainRec ch = recs[qs].chain;
-                    mbar_arrive_elect(ms.bar(kBarQEmpty + qs));  // the slot is no longer read
+                    mbar_arrive_el(ms.el, ms.bar(kBarQEmpty + qs));  // the slot is no longer read
                     const uint32_t mph = buf ? mid_ph1++ : mid_ph0++;
                     mbar_wait_mma(ms.bar(kBarMidFull + buf), mph & 1u, p.ctr, pipe_limit, broken);
                     tc_fence_after();
                     mma_chain_1x1(ms, j.d_tmem, wu(ch.n2), wu(ch.nch2), wu(ch.kst2), wu(ch.swz2) != 0, wu(ch.bpp2),
                                   wu(ch.np2), (uint32_t)wu(ch.blob2 * 2), wu(ch.a_col), wu(ch.out_col));
                 }
-                tc_commit_warp(ms.bar(kBarAccFull + buf));
+                tc_commit_el(ms.el, ms.bar(kBarAccFull + buf));
                 ++acc_cnt;
             }
             // Every MMA this warp issued has completed before TMEM is released.
             if (issued) {
-                tc_commit_warp(ms.bar(kBarDone));
+                tc_commit_el(ms.el, ms.bar(kBarDone));
                 mbar_wait_mma(ms.bar(kBarDone), 0u, p.ctr, pipe_limit, broken);
             }
         }
