@@ -91,6 +91,13 @@ struct MafatStageDev {
     //                    expands them into the one-octet halo, channels cin..7 zero.
     int32_t in_mode;
     int32_t raw_e;        // MAFAT_IN_GATHER: elements of one raw row in shared memory (multiple of 8)
+    // Pixel pairs (a gathered 3x3 stage of at most 4 input channels): 16-byte halo slot q holds
+    // the channels of pixels q and q + 1, 4 channels (8 bytes) each, the unused ones zero.  A
+    // core-matrix row of slot q then spans taps kx and kx + 1 of one kernel row, and one K = 16
+    // step covers a whole kernel row: its K halves are slots kx = 0 (taps 0, 1) and kx = 2 (tap
+    // 2 and a zero tap), LBO two slots apart.  A 3x3 convolution takes 3 K steps instead of the
+    // 5 of tap pairs over 8-channel pixels (K 48 against 80 for 27 useful values).
+    int32_t pix_pair;
     // On-chip chaining of a 3x3 convolution and the 1x1 convolution after it (tensor-core plans):
     // an item of a `chain` stage computes its pixels for all of the 3x3's channels into TMEM, the
     // epilogue writes the activated bf16 result back into TMEM as the A operand of the 1x1, and

@@ -450,7 +450,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 //   w[1] sb: offset of the item's first channel in the scale / bias arrays
 //   w[2] bytes of one weight blob
 //   w[3] n_mid: MMA N of the item's (first) convolution
-//   w[4] k | K steps per blob << 8 | blocks << 16 | paired << 24 | swizzled B << 25 | chain << 26
+//   w[4] k | K steps per blob << 8 | blocks << 16 | paired << 24 | swizzled B << 25 | chain << 26 |
+//        pixel pairs << 27
 //   w[5] A box columns | rows << 16
 //   w[6] input chunks | blobs per chunk << 16
 //   w[7] blobs per weight piece | pieces << 16
@@ -472,7 +473,8 @@ struct ChainRec {
 // none of them reads a work table from global memory on its critical path.
 // What the gather warp needs of an item that reads raw NHWC rows (MAFAT_IN_GATHER).
 struct GatherRec {
-    int16_t on;              // 1: this item's A halo is built from raw rows by the gather warp
+    int16_t on;              // 1: this item's A halo is built from raw rows by the gather warp,
+                             // one pixel per 16-byte slot; 2: two pixels per slot (pixel pairs)
     int16_t c;               // channels of the input (1..7)
     int16_t raw_e;           // elements of one raw row in shared memory
     int16_t s0;              // element of the first halo pixel's channel 0 within a raw row
@@ -664,6 +666,7 @@ struct MmaJob {
     uint32_t b_hi, b_half, b_step, blob_bytes, n_blk;
     int k, cols_box, n_chunks, n_bsteps, bpp, P, G, key, ticket, cur_b;
     bool bswz;
+    bool pp;   // paired form with pixel pairs: blob t is kernel row t (K halves at kx = 0 and 2)
     uint64_t wait_a, wait_b;
 };
 
@@ -726,9 +729,10 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
         const uint32_t a_hi = (uint32_t)(a_desc0 >> 32);
         uint32_t a_lo = (uint32_t)a_desc0 + j.a_off16;  // tap (ky, kx) of the plain form: + ky * cols_box + kx
         int kx = 0;
-        // paired form: offset (16-byte units) and column of tap 2t, advanced by two taps per blob
+        // paired form: offset (16-byte units) and column of tap 2t, advanced by two taps per blob;
+        // with pixel pairs, the offset of kernel row t's slot kx = 0, advanced by a halo row
         const uint32_t a_base16 = (a_base & 0x3FFFFu) >> 4;
-        uint32_t oa16 = 0;
+        uint32_t oa16 = 0, or16 = 0;
         int xa = 0;
         for (int t = 0; t < j.n_bsteps; ++t) {
             uint32_t a_lo_t, a_hi_t;
@@ -746,6 +750,10 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
                     pa = oa16;
                     pb = oa16;
                 }
+                // pixel pairs: the row's slots kx = 0 (taps 0, 1) and kx = 2 (tap 2, zero weights)
+                pa = j.pp ? or16 : pa;
+                pb = j.pp ? or16 + 2u : pb;
+                or16 += (uint32_t)j.cols_box;
                 a_lo_t = (a_base16 + pa) | ((pb - pa) << 16);
                 a_hi_t = a_hi;
                 oa16 += 2u;
@@ -805,10 +813,12 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
     }
 }
 
-// Widening of raw rows of c < 8 channels (other than the RGB fast path), pixel by pixel
-// (idx = r * cols + x dealt to the lanes); out of line, as it is off the common path.
+// Widening of raw rows of c < 8 channels (other than the RGB fast path), slot by slot
+// (idx = r * cols + x dealt to the lanes); out of line, as it is off the common path.  With
+// pixel pairs (pp, c <= 4) slot x holds pixel x in its first 8 bytes and pixel x + 1 in the
+// last 8.
 __device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage, int rows, int cols, int raw_e,
-                                            int s0, int c, int lane) {
+                                            int s0, int c, bool pp, int lane) {
     const uint16_t* raw = reinterpret_cast<const uint16_t*>(raw_b);
     uint4* dst = reinterpret_cast<uint4*>(stage);
     int r = 0, x = lane;
@@ -819,9 +829,18 @@ __device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage
     for (int idx = lane; idx < rows * cols; idx += 32) {
         const uint16_t* src = raw + r * raw_e + s0 + x * c;
         uint32_t w[4] = {0u, 0u, 0u, 0u};
+        if (pp) {
 #pragma unroll
-        for (int ch = 0; ch < 7; ++ch)
-            if (ch < c) w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
+            for (int ch = 0; ch < 4; ++ch)
+                if (ch < c) {
+                    w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
+                    w[2 + (ch >> 1)] |= (uint32_t)src[c + ch] << (16 * (ch & 1));
+                }
+        } else {
+#pragma unroll
+            for (int ch = 0; ch < 7; ++ch)
+                if (ch < c) w[ch >> 1] |= (uint32_t)src[ch] << (16 * (ch & 1));
+        }
         dst[idx] = make_uint4(w[0], w[1], w[2], w[3]);
         x += 32;
         while (x >= cols) {
@@ -871,16 +890,17 @@ __device__ __forceinline__ void mma_chain_1x1(MmaState& s, uint32_t acc, int n2,
     }
 }
 
-// Gather of a 3x3 halo row from raw NHWC elements: the one-octet pixel x of a halo row
-// holds elements S0 + C x .. S0 + C x + C - 1 of the raw row (the rest zero).  One lane
-// builds whole rows: the row's RAW_E elements come in as 16-byte loads, and with C, S0 and
-// the row length fixed at compile time every pixel is a few byte permutes and one 16-byte
+// Gather of a 3x3 halo row from raw NHWC elements: the 16-byte slot x of a halo row holds
+// elements S0 + C x .. S0 + C x + C - 1 of the raw row (the rest zero), or with pixel pairs
+// (PP, C <= 4) those of pixel x in its first 8 bytes and of pixel x + 1 in its last 8.  One
+// lane builds whole rows: the row's RAW_E elements come in as 16-byte loads, and with C, S0
+// and the row length fixed at compile time every slot is a few byte permutes and one 16-byte
 // store.  The rows of a halo are dealt to the lanes in turn.
-template <int C, int S0, int RAW_E>
+template <int C, int S0, int RAW_E, bool PP>
 __device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, int rows, int lane) {
     constexpr int kCols = MAFAT_BLK_COLS + 2;  // a gathered stage is a 3x3 convolution
     constexpr int kWords = RAW_E / 2;
-    static_assert(RAW_E % 8 == 0 && S0 + C * kCols <= RAW_E, "raw row");
+    static_assert(RAW_E % 8 == 0 && S0 + C * (kCols + (PP ? 1 : 0)) <= RAW_E && (!PP || C <= 4), "raw row");
     for (int r = lane; r < rows; r += 32) {
         uint32_t w[kWords];
         const uint4* src = reinterpret_cast<const uint4*>(raw + (size_t)r * RAW_E * 2);
@@ -897,11 +917,13 @@ __device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, in
         for (int x = 0; x < kCols; ++x) {
             uint32_t o[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-            for (int ch = 0; ch < C; ++ch) {
-                const int i = S0 + C * x + ch;
-                const uint32_t e = (w[i >> 1] >> (16 * (i & 1))) & 0xFFFFu;
-                o[ch >> 1] |= e << (16 * (ch & 1));
-            }
+            for (int px = 0; px < (PP ? 2 : 1); ++px)
+#pragma unroll
+                for (int ch = 0; ch < C; ++ch) {
+                    const int i = S0 + C * (x + px) + ch;
+                    const uint32_t e = (w[i >> 1] >> (16 * (i & 1))) & 0xFFFFu;
+                    o[2 * px + (ch >> 1)] |= e << (16 * (ch & 1));
+                }
             out[x] = make_uint4(o[0], o[1], o[2], o[3]);
         }
     }
@@ -1055,7 +1077,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                           (uint32_t)(st.blob_elems * 2), (uint32_t)st.n_blk);
                         w[1] = make_uint4((uint32_t)st.k | ((uint32_t)st.kst << 8) | ((uint32_t)it.nbk << 16) |
                                               ((uint32_t)st.paired << 24) | ((uint32_t)st.b_swz << 25) |
-                                              ((uint32_t)chain << 26),
+                                              ((uint32_t)chain << 26) | ((uint32_t)st.pix_pair << 27),
                                           (uint32_t)st.cols_box | ((uint32_t)st.rows_box << 16),
                                           (uint32_t)st.n_chunks | ((uint32_t)st.n_bsteps << 16),
                                           (uint32_t)st.bpp | ((uint32_t)st.n_pieces << 16));
@@ -1082,7 +1104,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rg.on = 0;
                     if (tk.in_kind == MAFAT_BUF_USER_IN && st.in_mode == MAFAT_IN_GATHER) {
                         const int e_start = (tk.cx0 + it.bx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * st.cin;
-                        rg.on = 1;
+                        rg.on = (int16_t)(st.pix_pair ? 2 : 1);
                         rg.c = (int16_t)st.cin;
                         rg.raw_e = (int16_t)st.raw_e;
                         rg.s0 = (int16_t)(e_start - (e_start & ~7));
@@ -1259,6 +1281,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 j.blob_bytes = (uint32_t)wu((int)m0.z);
                 j.a_plane = (w8 >> 16) * 16u;
                 j.bswz = ((w4 >> 25) & 1u) != 0;
+                j.pp = ((w4 >> 27) & 1u) != 0;
                 const int kst = (int)((w4 >> 8) & 0xFFu), nbk = (int)((w4 >> 16) & 0xFFu), paired = (int)((w4 >> 24) & 1u);
                 const int sb = wu((int)m0.y);
                 j.cur_b = j.P == 1 ? ms.wb.resident(j.key) : -1;
@@ -1409,18 +1432,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait(bar(kBarRawFull + as), uses & 1u, p.ctr, pipe_limit, broken, 32);
                 uint8_t* stage = smem + kOffA + as * kAStageBytes;
                 const uint8_t* raw_b = stage + mafat_raw_offset(rows, cols);
-                if (g.c == 3 && g.raw_e == 40 && cols == MAFAT_BLK_COLS + 2) {
-                    // RGB: the common case, one instance per alignment of the first element
+                if (g.on == 2 && g.c == 3 && g.raw_e == 40 && cols == MAFAT_BLK_COLS + 2) {
+                    // RGB in pixel pairs: the common case, one instance per alignment of the first element
                     switch (g.s0) {
 #define MAFAT_GATHER_CASE(S) \
-    case S: gather_rows<3, S, 40>(raw_b, stage, rows, lane); break;
+    case S: gather_rows<3, S, 40, true>(raw_b, stage, rows, lane); break;
                         MAFAT_GATHER_CASE(0) MAFAT_GATHER_CASE(1) MAFAT_GATHER_CASE(2) MAFAT_GATHER_CASE(3)
                         MAFAT_GATHER_CASE(4) MAFAT_GATHER_CASE(5) MAFAT_GATHER_CASE(6) MAFAT_GATHER_CASE(7)
 #undef MAFAT_GATHER_CASE
                         default: break;
                     }
                 } else {
-                    gather_generic(raw_b, stage, rows, cols, g.raw_e, g.s0, g.c, lane);
+                    gather_generic(raw_b, stage, rows, cols, g.raw_e, g.s0, g.c, g.on == 2, lane);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();

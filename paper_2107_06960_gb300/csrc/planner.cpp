@@ -421,10 +421,13 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             // i.e. not an image) are converted to octet-planar by a small kernel before the launch.
             s.in_mode = MAFAT_IN_PLANAR;
             s.raw_e = 0;
+            s.pix_pair = 0;
             if (l == 0 && cfg.dtype == 0) {
                 if (L.c_in < 8 && ((int64_t)L.w_in * L.c_in) % 8 == 0) {
                     s.in_mode = MAFAT_IN_GATHER;
-                    s.raw_e = (L.c_in * s.cols_box + 7 + 7) / 8 * 8;  // up to 7 leading elements of alignment
+                    // up to 7 leading elements of alignment; pixel pairs read one pixel more
+                    s.pix_pair = (L.c_in <= 4 && L.k == 3) ? 1 : 0;
+                    s.raw_e = (L.c_in * (s.cols_box + s.pix_pair) + 7 + 7) / 8 * 8;
                 } else if (L.c_in != 8) {
                     t.in_convert = 1;
                 }
@@ -459,7 +462,7 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             if (s.cin8 == 1) {
                 s.paired = 1;
                 s.n_chunks = 1;
-                s.n_bsteps = ceil_div(L.k * L.k, 2);
+                s.n_bsteps = s.pix_pair ? L.k : ceil_div(L.k * L.k, 2);  // a kernel row, or two taps, per K step
                 s.kst = 1;
             } else {
                 s.paired = 0;
@@ -1022,12 +1025,15 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
                 return "chain stage's copy of its 1x1 differs";
         }
         if (s.chained && (&s == t.stages.data() || !(&s - 1)->chain)) return "a chained stage without its chain stage";
+        if (s.pix_pair && s.in_mode != MAFAT_IN_GATHER) return "pixel pairs on a stage that is not gathered";
         if (s.in_mode == MAFAT_IN_GATHER) {
             const Layer& L = net.layers[s.layer];
             if (s.layer != 0 || !s.paired || L.c_in >= 8 || (int64_t)L.w_in * L.c_in % 8 != 0)
                 return "raw-row gather on a stage that does not read a narrow NHWC input";
-            if (s.raw_e % 8 != 0 || s.raw_e > 256 || s.raw_e < 7 + L.c_in * s.cols_box)
+            if (s.raw_e % 8 != 0 || s.raw_e > 256 || s.raw_e < 7 + L.c_in * (s.cols_box + s.pix_pair))
                 return "raw row does not hold the halo's elements";
+            if (s.pix_pair && (L.c_in > 4 || s.k != 3 || s.n_bsteps != 3 || s.cols_box != MAFAT_BLK_COLS + 2))
+                return "pixel pairs on a stage that is not a 3x3 convolution of at most 4 gathered channels";
             if (mafat_raw_offset(s.rows_box, s.cols_box) + (int64_t)s.rows_box * s.raw_e * 2 > MAFAT_A_STAGE_BYTES)
                 return "raw rows exceed their A stage";
         }
@@ -1134,7 +1140,10 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
 //  - regular stages: blob = tap (ky, kx), K half h of step j = input octet chunk*chunk8 + 2j + h;
 //  - paired stages (8 input channels): blob p holds taps (a, b) = (2p, 2p+1), or for an odd
 //    tap count the last blob holds (zero weights, last tap); K half 0 = tap a, half 1 = tap b
-//    (the kernel points both halves of that last blob at the last tap).
+//    (the kernel points both halves of that last blob at the last tap);
+//  - pixel-pair stages (3x3, at most 4 input channels): blob p is kernel row ky = p; K half h
+//    holds taps kx = 2h (elements 0-3, its channels) and 2h + 1 (elements 4-7; kx = 3 is a
+//    zero tap), matching a halo slot that holds two neighbouring pixels of 4 channels.
 void pack_weights_bf16(const Net& net, const PlanTables& t, std::vector<uint16_t>& out) {
     out.assign((size_t)t.weight_elems, 0);
     for (const MafatStageDev& s : t.stages) {
@@ -1152,7 +1161,11 @@ void pack_weights_bf16(const Net& net, const PlanTables& t, std::vector<uint16_t
                                 for (int e = 0; e < 8; ++e) {
                                     int o = nb * s.n_blk + nn;
                                     int ci, tap;
-                                    if (s.paired) {
+                                    if (s.pix_pair) {
+                                        const int kx = 2 * h + (e >> 2);
+                                        tap = kx < k ? b * k + kx : -1;
+                                        ci = e & 3;
+                                    } else if (s.paired) {
                                         int a = 2 * b, bb = 2 * b + 1;
                                         if (bb >= taps) {
                                             a = -1;  // zero weights paired with the last tap
