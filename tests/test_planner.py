@@ -165,6 +165,23 @@ def test_flat_blocks_cut_block_padding(mf):
     assert b - a == saved
 
 
+@pytest.mark.parametrize("c, k_issued", [(1, 48), (3, 48), (4, 48), (5, 80), (8, 80)])
+def test_first_layer_k_steps(mf, c, k_issued):
+    # A 3x3 first layer of c < 8 channels read from the NHWC image: up to 4 channels go in
+    # pixel pairs (a 16-byte halo slot holds two pixels, one K = 16 step covers a kernel row:
+    # 3 steps, K 48); 5-7 channels pair taps over 8-channel pixels (5 steps, K 80), and so do
+    # 8-channel inputs read as one octet plane.  64x64 on one tile: 4 x 8 blocks of 16x8.
+    conv = [("conv", 3, 1, 1, 32)]
+    net = mf.Net(conv, 64, 64, c)
+    net.set_params(synth.make_params(conv, c, 1, "bf16"))
+    st = mf.Plan(net, None, [(1, 1)], dry_run=True).stats()
+    assert st["issued_flops"] == 2 * (4 * 8 * 128) * 32 * k_issued
+    assert st["executed_flops"] == 2 * 64 * 64 * 32 * c * 9
+    # the fp32 check mode has no tensor-core packing: issued = executed
+    st32 = mf.Plan(net, None, [(1, 1)], dtype=mf.FP32, dry_run=True).stats()
+    assert st32["executed_flops"] == st["executed_flops"]
+
+
 def test_plan_validation_errors(mf):
     layers = synth.YOLO16
     net = _net(mf, layers, 64)
