@@ -98,6 +98,13 @@ struct MafatStageDev {
     // 2 and a zero tap), LBO two slots apart.  A 3x3 convolution takes 3 K steps instead of the
     // 5 of tap pairs over 8-channel pixels (K 48 against 80 for 27 useful values).
     int32_t pix_pair;
+    // Per-block halos (every gathered stage): the A stage holds one (16 + k - 1) x cols_box halo
+    // per block of the item, block after block, so that an item's blocks need not be stacked in
+    // one block column: they are any run of the task's blocks in column-major order (linear
+    // index bx * nby + by; the item's `by` is its first block's index, `bx` is 0).  The
+    // widening builds each block's halo from raw rows loaded block by block.  A 137-row tile
+    // region (9 block rows) then takes items of 8 blocks instead of 5 + 4 per block column.
+    int32_t blk_halo;
     // On-chip chaining of a 3x3 convolution and the 1x1 convolution after it (tensor-core plans):
     // an item of a `chain` stage computes its pixels for all of the 3x3's channels into TMEM, the
     // epilogue writes the activated bf16 result back into TMEM as the A operand of the 1x1, and
@@ -127,6 +134,12 @@ inline MAFAT_HD int mafat_flat_rows(int mb, int pitch, int k) {
 // one-octet halo of rows_box x cols_box pixels, on a 128-byte boundary.
 inline MAFAT_HD int mafat_raw_offset(int rows_box, int cols_box) {
     return (rows_box * cols_box * 16 + 127) & ~127;
+}
+
+// Bytes between the raw rows of consecutive blocks of a per-block-halo item (one TMA box of
+// 16 + k - 1 rows of raw_e elements each, on 128-byte boundaries).
+inline MAFAT_HD int mafat_raw_blk_stride(int k, int raw_e) {
+    return ((MAFAT_BLK_ROWS + k - 1) * raw_e * 2 + 127) & ~127;
 }
 
 struct MafatTaskDev {

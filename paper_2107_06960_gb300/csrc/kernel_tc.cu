@@ -451,7 +451,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 //   w[2] bytes of one weight blob
 //   w[3] n_mid: MMA N of the item's (first) convolution
 //   w[4] k | K steps per blob << 8 | blocks << 16 | paired << 24 | swizzled B << 25 | chain << 26 |
-//        pixel pairs << 27
+//        pixel pairs << 27 | per-block halos << 28
 //   w[5] A box columns | rows << 16
 //   w[6] input chunks | blobs per chunk << 16
 //   w[7] blobs per weight piece | pieces << 16
@@ -486,7 +486,9 @@ struct EpiRec {
     int32_t y0, ylim;        // conv row of the item's first block row; end of the task's rows
     int32_t out_y0, out_x0;  // map position of output buffer pixel (0, 0)
     int32_t out_w, out_h;    // output buffer extent (pixels, after pooling)
-    int32_t nbk, n_blk;      // blocks of the item; output channels per item (accumulator columns per block)
+    int16_t nbk;             // blocks of the item
+    int16_t nby;             // per-block-halo item: block rows of its task (0: blocks stacked from y0)
+    int32_t n_blk;           // output channels per item (accumulator columns per block)
     int32_t cout, ch_base;   // channels of the layer; first channel of the item
     int32_t flags;           // bit 0: fused max-pool, bit 1: NHWC output, bit 2: never published (test hook)
     int32_t done_ctr, extra_ctr;
@@ -494,7 +496,8 @@ struct EpiRec {
     int16_t n_mid;           // chain item: columns of the 3x3's accumulator
     int16_t a_col, out_col;  // chain item: TMEM columns of the 1x1's A operand and of its accumulator
     int16_t pitch;           // flat stage: row pitch of the region (pixels); 0: 16x8 blocks
-    int16_t flat_by;         // flat stage: the item's first block in the region
+    int16_t flat_by;         // flat stage: the item's first block in the region; per-block-halo item:
+                             // its first block's index in the task's column-major block order
 };
 
 // A queue slot: the record of one item, in parts, so that every role copies only its own.
@@ -816,10 +819,10 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
 // Widening of raw rows of c < 8 channels (other than the RGB fast path), slot by slot
 // (idx = r * cols + x dealt to the lanes); out of line, as it is off the common path.  With
 // pixel pairs (pp, c <= 4) slot x holds pixel x in its first 8 bytes and pixel x + 1 in the
-// last 8.
+// last 8.  The item's blocks have a halo of hr rows each, and their raw rows come block by
+// block, blk_stride bytes apart.
 __device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage, int rows, int cols, int raw_e,
-                                            int s0, int c, bool pp, int lane) {
-    const uint16_t* raw = reinterpret_cast<const uint16_t*>(raw_b);
+                                            int s0, int c, bool pp, int hr, int blk_stride, int lane) {
     uint4* dst = reinterpret_cast<uint4*>(stage);
     int r = 0, x = lane;
     while (x >= cols) {
@@ -827,7 +830,9 @@ __device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage
         ++r;
     }
     for (int idx = lane; idx < rows * cols; idx += 32) {
-        const uint16_t* src = raw + r * raw_e + s0 + x * c;
+        // widened row r is row r % hr of block r / hr, whose raw rows start blk_stride bytes apart
+        const uint16_t* src = reinterpret_cast<const uint16_t*>(raw_b + (r / hr) * blk_stride) + (r % hr) * raw_e +
+                              s0 + x * c;
         uint32_t w[4] = {0u, 0u, 0u, 0u};
         if (pp) {
 #pragma unroll
@@ -895,15 +900,18 @@ __device__ __forceinline__ void mma_chain_1x1(MmaState& s, uint32_t acc, int n2,
 // (PP, C <= 4) those of pixel x in its first 8 bytes and of pixel x + 1 in its last 8.  One
 // lane builds whole rows: the row's RAW_E elements come in as 16-byte loads, and with C, S0
 // and the row length fixed at compile time every slot is a few byte permutes and one 16-byte
-// store.  The rows of a halo are dealt to the lanes in turn.
+// store.  The rows of a halo are dealt to the lanes in turn.  Row r of the item is row r % 18
+// of its block r / 18, whose raw rows start on a 128-byte boundary.
 template <int C, int S0, int RAW_E, bool PP>
 __device__ __forceinline__ void gather_rows(const uint8_t* raw, uint8_t* dst, int rows, int lane) {
     constexpr int kCols = MAFAT_BLK_COLS + 2;  // a gathered stage is a 3x3 convolution
     constexpr int kWords = RAW_E / 2;
     static_assert(RAW_E % 8 == 0 && S0 + C * (kCols + (PP ? 1 : 0)) <= RAW_E && (!PP || C <= 4), "raw row");
+    constexpr int kHR = MAFAT_BLK_ROWS + 2;                          // halo rows of one block
+    constexpr int kStride = (kHR * RAW_E * 2 + 127) / 128 * 128;     // raw bytes of one block
     for (int r = lane; r < rows; r += 32) {
         uint32_t w[kWords];
-        const uint4* src = reinterpret_cast<const uint4*>(raw + (size_t)r * RAW_E * 2);
+        const uint4* src = reinterpret_cast<const uint4*>(raw + (r / kHR) * kStride + (r % kHR) * RAW_E * 2);
 #pragma unroll
         for (int q = 0; q < kWords / 4; ++q) {
             const uint4 v = src[q];
@@ -1054,7 +1062,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                              tk.out_off;
                     rc.x0 = tk.cx0 + it.bx * MAFAT_BLK_COLS;
                     rc.xlim = tk.cx0 + tk.cw;
-                    rc.y0 = flat_off >= 0 ? tk.cy0 : tk.cy0 + it.by * MAFAT_BLK_ROWS;
+                    rc.y0 = (flat_off >= 0 || st.blk_halo) ? tk.cy0 : tk.cy0 + it.by * MAFAT_BLK_ROWS;
+                    rc.nby = (int16_t)(st.blk_halo ? tk.nby : 0);
                     rc.pitch = (int16_t)(flat_off >= 0 ? st.cols_box : 0);
                     rc.flat_by = it.by;
                     rc.ylim = tk.cy0 + tk.ch;
@@ -1062,7 +1071,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.out_x0 = tk.out_x0;
                     rc.out_w = tk.out_w;
                     rc.out_h = tk.out_h;
-                    rc.nbk = it.nbk;
+                    rc.nbk = (int16_t)it.nbk;
                     // what the epilogue stores: the item's own output, or a chain item's 1x1 output
                     const bool chain = kChain && st.chain;
                     rc.n_blk = chain ? st.c2_n_blk : st.n_blk;
@@ -1077,7 +1086,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                                           (uint32_t)(st.blob_elems * 2), (uint32_t)st.n_blk);
                         w[1] = make_uint4((uint32_t)st.k | ((uint32_t)st.kst << 8) | ((uint32_t)it.nbk << 16) |
                                               ((uint32_t)st.paired << 24) | ((uint32_t)st.b_swz << 25) |
-                                              ((uint32_t)chain << 26) | ((uint32_t)st.pix_pair << 27),
+                                              ((uint32_t)chain << 26) | ((uint32_t)st.pix_pair << 27) |
+                                              ((uint32_t)st.blk_halo << 28),
                                           (uint32_t)st.cols_box | ((uint32_t)st.rows_box << 16),
                                           (uint32_t)st.n_chunks | ((uint32_t)st.n_bsteps << 16),
                                           (uint32_t)st.bpp | ((uint32_t)st.n_pieces << 16));
@@ -1175,13 +1185,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint32_t a_dst = sbase + kOffA + as * kAStageBytes;
                     mbar_wait(bar(kBarAEmpty + as), ((a_cnt / kAStages) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                     if (in_mode == MAFAT_IN_GATHER) {
-                        // raw NHWC rows from the 16-byte aligned element at or before the halo's
-                        // first one into the stage's tail; the gather warp builds the halo from
-                        // them and completes the stage's full barrier itself
-                        const int e_start = px0 * st.cin;
-                        mbar_arrive_expect_tx(bar(kBarRawFull + as), (uint32_t)(st.rows_box * st.raw_e * 2));
-                        tma_load_3d(a_dst + (uint32_t)mafat_raw_offset(st.rows_box, st.cols_box), map,
-                                    e_start & ~7, y0, c3, bar(kBarRawFull + as));
+                        // raw NHWC rows of each block's halo, from the 16-byte aligned element at
+                        // or before the halo's first one, into the stage's tail block after block;
+                        // the gather warp builds the halos from them and completes the stage's
+                        // full barrier itself.  The item's blocks run down its task's block
+                        // columns (column-major order from block it.by).
+                        const int hr = MAFAT_BLK_ROWS + st.k - 1;
+                        const uint32_t stride = (uint32_t)mafat_raw_blk_stride(st.k, st.raw_e);
+                        uint32_t dst = a_dst + (uint32_t)mafat_raw_offset(st.rows_box, st.cols_box);
+                        mbar_arrive_expect_tx(bar(kBarRawFull + as), (uint32_t)(it.nbk * hr * st.raw_e * 2));
+                        int bxx = it.by / tk.nby, byy = it.by - bxx * tk.nby;
+                        for (int j = 0; j < it.nbk; ++j, dst += stride) {
+                            const int e = (tk.cx0 + bxx * MAFAT_BLK_COLS - st.pad - tk.in_x0) * st.cin;
+                            tma_load_3d(dst, map, e & ~7, tk.cy0 + byy * MAFAT_BLK_ROWS - st.pad - tk.in_y0, c3,
+                                        bar(kBarRawFull + as));
+                            if (++byy == tk.nby) {
+                                byy = 0;
+                                ++bxx;
+                            }
+                        }
                     } else {
                         mbar_arrive_expect_tx(bar(kBarAFull + as), a_bytes);
                         tma_load_4d(a_dst, map, x0, y0, c * st.chunk8, c3, bar(kBarAFull + as));
@@ -1318,7 +1340,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int flat_off = (int)(w8 & 0xFFFFu) - 1;
                 j.a_row = flat_off >= 0 ? 128u : (uint32_t)(j.cols_box * 16);
                 j.b_half = j.n_blk * 16u;
-                j.blk16 = flat_off >= 0 ? 128u : (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);  // next block, 16-B units
+                // next block (16-B units): one halo row apart in stacked 16x8 blocks; a block-halo apart
+                // with per-block halos; 128 pixels on in a flat stage
+                j.blk16 = flat_off >= 0             ? 128u
+                          : ((w4 >> 28) & 1u) != 0u ? (uint32_t)((MAFAT_BLK_ROWS + j.k - 1) * j.cols_box)
+                                                    : (uint32_t)(MAFAT_BLK_ROWS * j.cols_box);
                 j.a_off16 = flat_off >= 0 ? (uint32_t)flat_off : 0u;
                 j.a_step = 2u * (j.a_plane >> 4);                   // next K=16 step: two octet planes
                 // B descriptor: 128-byte swizzled blobs (64 channels per row) or no-swizzle core matrices
@@ -1414,13 +1440,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_wait(bar(kBarQFull + qs), (q_cnt / kQDepth) & 1u, p.ctr, pipe_limit, broken, 256);
             const int ticket = q_items[qs];
             GatherRec g{};
-            int n_chunks = 0, rows = 0, cols = 0;
+            int n_chunks = 0, rows_box = 0, rows = 0, cols = 0, hr = 0;
             if (ticket >= 0) {
                 g = recs[qs].gather;
-                const uint32_t w5 = recs[qs].mma.w[5], w6 = recs[qs].mma.w[6];
+                const uint32_t w4 = recs[qs].mma.w[4], w5 = recs[qs].mma.w[5], w6 = recs[qs].mma.w[6];
                 n_chunks = (int)(w6 & 0xFFFFu);
-                rows = (int)(w5 >> 16);
+                rows_box = (int)(w5 >> 16);
                 cols = (int)(w5 & 0xFFFFu);
+                // a gathered item holds one halo of hr rows per block, block after block
+                hr = MAFAT_BLK_ROWS + (int)(w4 & 0xFFu) - 1;
+                rows = (int)((w4 >> 16) & 0xFFu) * hr;
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarQEmpty + qs));
@@ -1431,7 +1460,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t uses = as ? raw_uses1++ : raw_uses0++;
                 mbar_wait(bar(kBarRawFull + as), uses & 1u, p.ctr, pipe_limit, broken, 32);
                 uint8_t* stage = smem + kOffA + as * kAStageBytes;
-                const uint8_t* raw_b = stage + mafat_raw_offset(rows, cols);
+                // the raw rows start after the widened halos of the stage's largest item
+                const uint8_t* raw_b = stage + mafat_raw_offset(rows_box, cols);
                 if (g.on == 2 && g.c == 3 && g.raw_e == 40 && cols == MAFAT_BLK_COLS + 2) {
                     // RGB in pixel pairs: the common case, one instance per alignment of the first element
                     switch (g.s0) {
@@ -1443,7 +1473,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         default: break;
                     }
                 } else {
-                    gather_generic(raw_b, stage, rows, cols, g.raw_e, g.s0, g.c, g.on == 2, lane);
+                    gather_generic(raw_b, stage, rows, cols, g.raw_e, g.s0, g.c, g.on == 2, hr,
+                                   mafat_raw_blk_stride(hr - MAFAT_BLK_ROWS + 1, g.raw_e), lane);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
@@ -1536,6 +1567,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int yy = pf / rc.pitch;
                     Y = rc.y0 + yy;
                     Xb = rc.x0 + (pf - yy * rc.pitch);
+                } else if (rc.nby > 0) {
+                    // per-block halos: the item's block b is block flat_by + b of its task in
+                    // column-major order
+                    const int lin = rc.flat_by + b;
+                    const int bxx = lin / rc.nby;
+                    Y = rc.y0 + (lin - bxx * rc.nby) * MAFAT_BLK_ROWS + r;
+                    Xb = X + bxx * MAFAT_BLK_COLS;
                 }
                 const bool valid = (Y < rc.ylim) && (Xb < rc.xlim);
                 // a pooled stage's conv region starts on even rows and columns and has even

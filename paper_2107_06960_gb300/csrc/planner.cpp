@@ -422,11 +422,13 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             s.in_mode = MAFAT_IN_PLANAR;
             s.raw_e = 0;
             s.pix_pair = 0;
+            s.blk_halo = 0;
             if (l == 0 && cfg.dtype == 0) {
                 if (L.c_in < 8 && ((int64_t)L.w_in * L.c_in) % 8 == 0) {
                     s.in_mode = MAFAT_IN_GATHER;
                     // up to 7 leading elements of alignment; pixel pairs read one pixel more
                     s.pix_pair = (L.c_in <= 4 && L.k == 3) ? 1 : 0;
+                    s.blk_halo = 1;
                     s.raw_e = (L.c_in * (s.cols_box + s.pix_pair) + 7 + 7) / 8 * 8;
                 } else if (L.c_in != 8) {
                     t.in_convert = 1;
@@ -434,12 +436,15 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
             }
             // input octets per A chunk: the largest that fits the A stage with mb blocks
             for (;;) {
-                s.rows_box = s.flat ? mafat_flat_rows(s.mb, s.cols_box, L.k) : MAFAT_BLK_ROWS * s.mb + L.k - 1;
+                s.rows_box = s.flat       ? mafat_flat_rows(s.mb, s.cols_box, L.k)
+                             : s.blk_halo ? (MAFAT_BLK_ROWS + L.k - 1) * s.mb
+                                          : MAFAT_BLK_ROWS * s.mb + L.k - 1;
                 const int row_bytes = s.cols_box * 16 * s.rows_box;
                 if (s.in_mode == MAFAT_IN_GATHER) {
-                    // the expanded halo plus the raw rows it is built from share the stage
+                    // the expanded halos plus the raw rows they are built from share the stage
                     s.chunk8 = 1;
-                    if (mafat_raw_offset(s.rows_box, s.cols_box) + s.rows_box * s.raw_e * 2 <= MAFAT_A_STAGE_BYTES ||
+                    if (mafat_raw_offset(s.rows_box, s.cols_box) + s.mb * mafat_raw_blk_stride(L.k, s.raw_e) <=
+                            MAFAT_A_STAGE_BYTES ||
                         s.mb == 1)
                         break;
                     s.mb /= 2;
@@ -764,7 +769,8 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
                             tk.out_y0 = orr.y0;
                             tk.out_x0 = orr.x0;
                         }
-                        tk.n_items = ceil_div(tk.nby, st.mb) * tk.nbx * st.n_nblk;
+                        tk.n_items = (st.blk_halo ? ceil_div(tk.nby * tk.nbx, st.mb) : ceil_div(tk.nby, st.mb) * tk.nbx) *
+                                     st.n_nblk;
                         TaskDep d;
                         int qi = (int)(q - w0);
                         if (s == t.stage_first[g]) {
@@ -899,11 +905,16 @@ std::string build_plan(const Net& net, const PlanConfig& cfg, PlanTables& t, boo
         // channel-block major: consecutive items share a resident weight set; a task's block
         // rows are split evenly over ceil(nby / mb) items (9 rows at mb = 8 give 5 + 4, not
         // 8 + 1, whose 1-block item would pay a whole item's fixed cost for little work)
-        const int n_rows = ceil_div(tk.nby, st.mb);
+        // Per-block-halo stages pack the task's blocks, in column-major order, evenly into
+        // ceil(blocks / mb) items whatever the block columns (`by` = first block, `bx` = 0).
+        const int n_blocks = tk.nby * tk.nbx;
+        const int n_rows = st.blk_halo ? ceil_div(n_blocks, st.mb) : ceil_div(tk.nby, st.mb);
+        const int n_cols = st.blk_halo ? 1 : tk.nbx;
+        const int n_span = st.blk_halo ? n_blocks : tk.nby;
         for (int nb = 0; nb < st.n_nblk; ++nb)
             for (int ri = 0; ri < n_rows; ++ri)
-                for (int bx = 0; bx < tk.nbx; ++bx) {
-                    const int by = ri * tk.nby / n_rows, by_end = (ri + 1) * tk.nby / n_rows;
+                for (int bx = 0; bx < n_cols; ++bx) {
+                    const int by = ri * n_span / n_rows, by_end = (ri + 1) * n_span / n_rows;
                     MafatItemDev it{};
                     it.task = ti;
                     it.stage = (int16_t)tk.stage;
@@ -990,8 +1001,11 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         if ((s.cols_box * 16) % 16 != 0) return "TMA inner box not a multiple of 16 bytes";
         if (s.n_blk % 16 != 0 || s.n_blk < 16 || s.n_blk > MAFAT_MAX_NBLK) return "bad MMA N";
         if (s.mb < 1 || s.mb * s.n_blk > 256) return "blocks of an item exceed one TMEM accumulator buffer";
-        if (s.rows_box != (s.flat ? mafat_flat_rows(s.mb, s.cols_box, s.k) : MAFAT_BLK_ROWS * s.mb + s.k - 1))
+        if (s.rows_box != (s.flat       ? mafat_flat_rows(s.mb, s.cols_box, s.k)
+                           : s.blk_halo ? (MAFAT_BLK_ROWS + s.k - 1) * s.mb
+                                        : MAFAT_BLK_ROWS * s.mb + s.k - 1))
             return "A box rows do not cover the item";
+        if (s.blk_halo && (s.in_mode != MAFAT_IN_GATHER || s.flat)) return "per-block halos on a stage that is not gathered";
         if (s.flat) {
             if (s.pool || s.chain || s.chained || s.paired || s.cin8 < 2 || s.in_mode != MAFAT_IN_PLANAR)
                 return "flat blocks on a pooled, chained, paired-tap or gathered stage";
@@ -1034,7 +1048,9 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
                 return "raw row does not hold the halo's elements";
             if (s.pix_pair && (L.c_in > 4 || s.k != 3 || s.n_bsteps != 3 || s.cols_box != MAFAT_BLK_COLS + 2))
                 return "pixel pairs on a stage that is not a 3x3 convolution of at most 4 gathered channels";
-            if (mafat_raw_offset(s.rows_box, s.cols_box) + (int64_t)s.rows_box * s.raw_e * 2 > MAFAT_A_STAGE_BYTES)
+            if (!s.blk_halo) return "a gathered stage without per-block halos";
+            if (mafat_raw_offset(s.rows_box, s.cols_box) + (int64_t)s.mb * mafat_raw_blk_stride(s.k, s.raw_e) >
+                MAFAT_A_STAGE_BYTES)
                 return "raw rows exceed their A stage";
         }
     }
@@ -1095,9 +1111,16 @@ std::string validate_plan(const Net& net, const PlanTables& t) {
         const MafatItemDev& it = t.items[i];
         const MafatTaskDev& k = t.tasks[it.task];
         const MafatStageDev& s = t.stages[k.stage];
-        if (it.by >= k.nby || it.bx >= k.nbx || it.nb >= s.n_nblk || it.by < 0 || it.bx < 0 || it.nb < 0)
-            return "item block out of range";
-        if (it.nbk < 1 || it.nbk > s.mb || it.by + it.nbk > k.nby) return "item block count out of range";
+        if (s.blk_halo) {
+            // a run of the task's blocks in column-major order
+            if ((int64_t)k.nby * k.nbx > 32767 || it.bx != 0 || it.by < 0 || it.nb < 0 || it.nb >= s.n_nblk ||
+                it.nbk < 1 || it.nbk > s.mb || it.by + it.nbk > k.nby * k.nbx)
+                return "per-block-halo item out of range";
+        } else {
+            if (it.by >= k.nby || it.bx >= k.nbx || it.nb >= s.n_nblk || it.by < 0 || it.bx < 0 || it.nb < 0)
+                return "item block out of range";
+            if (it.nbk < 1 || it.nbk > s.mb || it.by + it.nbk > k.nby) return "item block count out of range";
+        }
         if (s.flat) {
             // every pixel the item's MMAs read (its blocks' 128 pixels at every tap offset) lies
             // inside the A box that starts at the row of its first pixel

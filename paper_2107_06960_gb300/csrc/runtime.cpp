@@ -123,7 +123,7 @@ bool encode_planar_map(CUtensorMap* m, const void* base, int w, int h, int c8, i
 
 // 3-D tiled map over a narrow NHWC bf16 input (c < 8 channels) seen as rows of raw
 // elements [frames][h][w*c]: dim0 = w*c elements, dim1 = h, dim2 = frames.  Box = raw_e
-// elements (from a 16-byte aligned element) x rows_box rows x 1 frame; elements outside
+// elements (from a 16-byte aligned element) x one block's halo rows x 1 frame; elements outside
 // the image read as zero (the convolution's zero padding, left and right included).
 bool encode_raw_rows_map(CUtensorMap* m, const void* base, int w, int h, int c, int frames, int raw_e,
                          int rows_box, std::string* err) {
@@ -238,7 +238,7 @@ mafat_status launch(mafat_plan_s* p, const void* input, void* output, cudaStream
             bool ok;
             if (s0.in_mode == MAFAT_IN_GATHER)
                 ok = encode_raw_rows_map(&p->in_map, in_dev, L0.w_in, L0.h_in, L0.c_in, p->t.cfg.batch, s0.raw_e,
-                                         s0.rows_box, &err);
+                                         MAFAT_BLK_ROWS + s0.k - 1, &err);  // one block's halo rows
             else  // octet-planar: an 8-channel NHWC input is one octet plane, or the converted copy
                 ok = encode_planar_map(&p->in_map, in_dev, L0.w_in, L0.h_in, p->t.in_c8, p->t.cfg.batch,
                                        p->t.in_cols_box, p->t.in_rows_box, p->t.in_chunk8, &err);
