@@ -599,6 +599,71 @@ __device__ __forceinline__ void epi_chunk(uint32_t taddr, const float* sc, const
     }
 }
 
+// Sixteen TMEM lanes from `taddr` x 32 columns in the 16x256b shape (then wait): lane l of the
+// warp gets, for column group g = 0..3, v[4g + e] = column 8g + 2 (l % 4) + (e & 1) of TMEM lane
+// l / 4 (e < 2) or l / 4 + 8 (e >= 2) counted from taddr's lane (pinned on GB300 by a probe that
+// wrote lane << 8 | column into every cell).
+__device__ __forceinline__ void tmem_ld16x256_x4(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x256b.x4.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+// Epilogue of one block x 32 accumulator columns (channels ch0 .. ch0 + 31) with the fused 2x2
+// max-pool, read in the 16x256b shape so that both rows of a pool window sit in one lane: the
+// warp's quarter holds conv rows 4 wq .. 4 wq + 3 of the block (TMEM lane = 8 row + column), and
+// its two loads (lanes +0 and +16) give lane l the pixels (2h, l / 4) and (2h + 1, l / 4) of
+// load h, channels 8g + 2 (l % 4) + {0, 1}.  Folded BN, leaky ReLU and bf16 rounding as in
+// epi_chunk, the vertical max in the lane, then one exchange with lane l ^ 4 (the next column):
+// a lane of an even column keeps pooled row 0 of its quarter, one of an odd column row 1.  Each
+// lane then stores 4 bytes (two channels) of each of its pooled pixel's four octets.
+struct EpiPoolDst {
+    __nv_bfloat16* out;
+    uint32_t pix, plane;  // element offset of the pooled pixel (NHWC: of its channel 0); octet plane
+    int nhwc, cout;
+    bool store;
+};
+__device__ __forceinline__ void epi_pool32(uint32_t taddr, const float* sc, const float* bi, int ch0,
+                                           const EpiPoolDst& d, int lane) {
+    uint32_t raw0[16], raw1[16];
+    tmem_ld16x256_x4(taddr, raw0);
+    tmem_ld16x256_x4(taddr + (16u << 16), raw1);
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    const int q2 = 2 * (lane & 3);
+    uint32_t pv0[4], pv1[4];  // per column group: bf16x2 of channels 8g + q2, + 1 after the vertical max
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        const float2 s = *reinterpret_cast<const float2*>(sc + 8 * g + q2);  // shared memory
+        const float2 c = *reinterpret_cast<const float2*>(bi + 8 * g + q2);
+        float a0, a1, b0, b1;
+        bn_leaky2(s.x, s.y, raw0[4 * g], raw0[4 * g + 1], c.x, c.y, a0, a1);
+        bn_leaky2(s.x, s.y, raw0[4 * g + 2], raw0[4 * g + 3], c.x, c.y, b0, b1);
+        pv0[g] = max_bf16x2(pack_bf16x2(a0, a1), pack_bf16x2(b0, b1));
+        bn_leaky2(s.x, s.y, raw1[4 * g], raw1[4 * g + 1], c.x, c.y, a0, a1);
+        bn_leaky2(s.x, s.y, raw1[4 * g + 2], raw1[4 * g + 3], c.x, c.y, b0, b1);
+        pv1[g] = max_bf16x2(pack_bf16x2(a0, a1), pack_bf16x2(b0, b1));
+    }
+    const bool odd = ((lane >> 2) & 1) != 0;
+    uint32_t res[4];
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        const uint32_t got = __shfl_xor_sync(0xffffffffu, odd ? pv0[g] : pv1[g], 4);
+        res[g] = max_bf16x2(odd ? pv1[g] : pv0[g], got);
+    }
+    if (!d.store) return;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        const int ch = ch0 + 8 * g;
+        if (ch >= d.cout) break;  // channels past cout belong to the zero-padded MMA N
+        __nv_bfloat16* p = d.out + (d.nhwc ? d.pix + (uint32_t)(ch + q2) : (uint32_t)(ch >> 3) * d.plane + d.pix + q2);
+        *reinterpret_cast<uint32_t*>(p) = res[g];
+    }
+}
+
 // Weight-buffer bookkeeping.  The producer and the MMA issuer each keep a copy and
 // apply the same transitions to the same item sequence, so they agree without
 // talking on which of the two buffers holds which weights.  A set that fits one
@@ -1545,7 +1610,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 sc += rc.n_mid;
                 bi += rc.n_mid;
             }
-            const int X = rc.x0 + cc;
             const bool pool = (rc.flags & 1) != 0, nhwc = (rc.flags & 2) != 0;
             // Work split between the warpgroups in units of one block x 32 output columns
             // (16 when N is an odd multiple of 16), dealt round-robin.
@@ -1559,7 +1623,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (b >= rc.nbk) break;
                 const int q = qi * uw;
-                int Y = rc.y0 + b * MAFAT_BLK_ROWS + r, Xb = X;
+                const uint32_t taddr = acc_lanes + col0 + (uint32_t)(b * rc.n_blk + q);
+                // conv position of the block's top-left pixel
+                int yb = rc.y0 + b * MAFAT_BLK_ROWS, xb = rc.x0;
+                if (rc.nby > 0) {
+                    // per-block halos: the item's block b is block flat_by + b of its task in
+                    // column-major order
+                    const int lin = rc.flat_by + b;
+                    const int bxx = lin / rc.nby;
+                    yb = rc.y0 + (lin - bxx * rc.nby) * MAFAT_BLK_ROWS;
+                    xb = rc.x0 + bxx * MAFAT_BLK_COLS;
+                }
+                if (pool && uw == 32) {
+                    // the window of this lane's pooled pixel (epi_pool32): rows 4 wq + 2 (c & 1) + {0, 1},
+                    // columns (c & ~1) + {0, 1} of the block, c = lane / 4
+                    const int c = lane >> 2;
+                    const int Yw = yb + wq * 4 + 2 * (c & 1), Xw = xb + (c & ~1);
+                    const uint32_t pix = (uint32_t)(((Yw >> 1) - rc.out_y0) * rc.out_w + ((Xw >> 1) - rc.out_x0));
+                    EpiPoolDst pd;
+                    pd.out = rc.out;
+                    pd.nhwc = nhwc;
+                    pd.pix = nhwc ? pix * (uint32_t)rc.cout : pix * 8u;
+                    pd.plane = (uint32_t)(rc.out_h * rc.out_w * 8);
+                    pd.cout = rc.cout;
+                    pd.store = (Yw < rc.ylim) && (Xw < rc.xlim);
+                    epi_pool32(taddr, sc + q, bi + q, rc.ch_base + q, pd, lane);
+                    continue;
+                }
+                int Y = yb + r, Xb = xb + cc;
                 if (rc.pitch > 0) {
                     // flat stage (never pooled): pixel 128 (flat_by + b) + 32 wq + lane of the
                     // region read row after row, rc.pitch pixels a row
@@ -1567,13 +1658,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int yy = pf / rc.pitch;
                     Y = rc.y0 + yy;
                     Xb = rc.x0 + (pf - yy * rc.pitch);
-                } else if (rc.nby > 0) {
-                    // per-block halos: the item's block b is block flat_by + b of its task in
-                    // column-major order
-                    const int lin = rc.flat_by + b;
-                    const int bxx = lin / rc.nby;
-                    Y = rc.y0 + (lin - bxx * rc.nby) * MAFAT_BLK_ROWS + r;
-                    Xb = X + bxx * MAFAT_BLK_COLS;
                 }
                 const bool valid = (Y < rc.ylim) && (Xb < rc.xlim);
                 // a pooled stage's conv region starts on even rows and columns and has even
@@ -1592,7 +1676,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 dst.cout = rc.cout;
                 dst.store = valid;
                 dst.pool = pool;
-                const uint32_t taddr = acc_lanes + col0 + (uint32_t)(b * rc.n_blk + q);
                 if (uw == 32)
                     epi_chunk<32>(taddr, sc + q, bi + q, rc.ch_base + q, dst, lane);
                 else
