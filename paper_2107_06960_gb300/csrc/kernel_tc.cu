@@ -889,6 +889,7 @@ __device__ __forceinline__ void mma_item(MmaState& s, MmaJob& j) {
 __device__ __noinline__ void gather_generic(const uint8_t* raw_b, uint8_t* stage, int rows, int cols, int raw_e,
                                             int s0, int c, bool pp, int hr, int blk_stride, int lane) {
     uint4* dst = reinterpret_cast<uint4*>(stage);
+    if (cols <= 0) return;  // only a record read after a pipeline wait ran out can hold this
     int r = 0, x = lane;
     while (x >= cols) {
         x -= cols;
@@ -1614,7 +1615,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Work split between the warpgroups in units of one block x 32 output columns
             // (16 when N is an odd multiple of 16), dealt round-robin.
             const int uw = (rc.n_blk & 31) == 0 ? 32 : 16;
-            const int upb = uw == 32 ? rc.n_blk >> 5 : rc.n_blk >> 4;  // units per block
+            // units per block (at least 1: only a record read after a pipeline wait ran out
+            // can hold a smaller N, and the unit walk below must end)
+            const int upb = max(1, uw == 32 ? rc.n_blk >> 5 : rc.n_blk >> 4);
             // unit u = b * upb + qi, from u = h in steps of kEpiGroups (no division per unit)
             for (int b = 0, qi = h;; qi += kEpiGroups) {
                 while (qi >= upb) {
