@@ -182,6 +182,26 @@ def test_first_layer_k_steps(mf, c, k_issued):
     assert st32["executed_flops"] == st["executed_flops"]
 
 
+def test_gathered_first_layer_packs_blocks_across_columns(mf):
+    # The first layer read from the RGB image keeps one halo per block, so an item's blocks
+    # are any run of its task's blocks in column-major order: a 144x1216 map on one tile is
+    # 9 block rows x 152 block columns = 1368 blocks, enough for 8 blocks per item on 152
+    # CTAs: 171 items of 8 (stacked per block column it takes 2 items per column, 304).  A
+    # first layer of 8 channels is read as an octet plane and keeps stacked blocks.
+    conv = [("conv", 3, 1, 1, 32)]
+    for c, items in ((3, 171), (8, 304)):
+        net = mf.Net(conv, 144, 1216, c)
+        net.set_params(synth.make_params(conv, c, 1, "bf16"))
+        st = mf.Plan(net, None, [(1, 1)], dry_run=True).stats()
+        assert st["n_items"] == items, (c, st["n_items"])
+        assert st["issued_flops"] == 2 * 1368 * 128 * 32 * (48 if c == 3 else 80)
+    # with the pool fused the blocks and items are the same
+    pooled = [("conv", 3, 1, 1, 32), ("max", 2, 2, 0, 0)]
+    net = mf.Net(pooled, 144, 1216, 3)
+    net.set_params(synth.make_params(pooled, 3, 1, "bf16"))
+    assert mf.Plan(net, None, [(1, 1)], dry_run=True).stats()["n_items"] == 171
+
+
 def test_plan_validation_errors(mf):
     layers = synth.YOLO16
     net = _net(mf, layers, 64)
