@@ -463,7 +463,7 @@ struct __align__(16) MmaRec {
 // What the MMA issuer needs of a chain item's chained 1x1 (N, input chunks, K steps per blob,
 // swizzled blobs, blobs per piece, pieces, TMEM columns of its A operand and accumulator,
 // blob elements, scale / bias offset).  Read from the queue slot only on the chain path.
-struct ChainRec {
+struct __align__(8) ChainRec {
     int16_t n2, nch2, kst2, swz2, bpp2, np2, a_col, out_col;
     int32_t blob2, sb2;
 };
@@ -472,7 +472,7 @@ struct ChainRec {
 // queue slot by the producer (which has the work tables in registers anyway), so that
 // none of them reads a work table from global memory on its critical path.
 // What the gather warp needs of an item that reads raw NHWC rows (MAFAT_IN_GATHER).
-struct GatherRec {
+struct __align__(8) GatherRec {
     int16_t on;              // 1: this item's A halo is built from raw rows by the gather warp,
                              // one pixel per 16-byte slot; 2: two pixels per slot (pixel pairs)
     int16_t c;               // channels of the input (1..7)
@@ -480,7 +480,7 @@ struct GatherRec {
     int16_t s0;              // element of the first halo pixel's channel 0 within a raw row
 };
 
-struct EpiRec {
+struct __align__(16) EpiRec {  // 16-byte aligned: written and read with 16-byte accesses
     __nv_bfloat16* out;      // output buffer of the task (frame and tile offset applied)
     int32_t x0, xlim;        // conv column of the item's block column; end of the task's columns
     int32_t y0, ylim;        // conv row of the item's first block row; end of the task's rows
@@ -1119,9 +1119,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait(bar(kBarQEmpty + qs), ((q_cnt / kQDepth) & 1u) ^ 1u, p.ctr, pipe_limit, broken, 64);
                 q_items[qs] = ticket;
                 if (ticket >= 0) {
-                    EpiRec& rc = recs[qs].epi;
+                    // the records are built in registers and stored whole (a few wide stores rather
+                    // than one per field, on this single thread while the tensor core keeps the
+                    // shared memory busy)
+                    EpiRec rc{};
                     MmaRec& rm = recs[qs].mma;
-                    GatherRec& rg = recs[qs].gather;
+                    GatherRec rg{};
                     rc.out = (__nv_bfloat16*)(tk.out_kind == MAFAT_BUF_USER_OUT ? p.user_out
                                               : tk.out_kind == MAFAT_BUF_CUT    ? p.cut
                                                                                 : p.scratch) +
@@ -1163,7 +1166,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rc.n_mid = (int16_t)st.n_blk;
                     rc.chain = (int16_t)chain;
                     if (chain) {
-                        ChainRec& rh = recs[qs].chain;
+                        ChainRec rh{};
                         rh.n2 = (int16_t)st.c2_n_blk;
                         rh.nch2 = (int16_t)st.c2_n_chunks;
                         rh.kst2 = (int16_t)st.c2_kst;
@@ -1174,6 +1177,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         rh.out_col = (int16_t)st.chain_out_col;
                         rh.blob2 = st.c2_blob_elems;
                         rh.sb2 = st.c2_sb_off;
+                        recs[qs].chain = rh;
                         rc.a_col = (int16_t)st.chain_a_col;
                         rc.out_col = (int16_t)st.chain_out_col;
                     }
@@ -1185,6 +1189,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         rg.raw_e = (int16_t)st.raw_e;
                         rg.s0 = (int16_t)(e_start - (e_start & ~7));
                     }
+                    recs[qs].epi = rc;
+                    recs[qs].gather = rg;
                 }
                 mbar_arrive(bar(kBarQFull + qs));  // release: the record is visible to the consumers
                 ++q_cnt;
