@@ -113,6 +113,9 @@ def test_fp32_full_size(mf, name):
     (1, 16, 3, True, 20, 24, (2, 2)),     # 1 channel
     (7, 16, 3, False, 17, 16, (1, 1)),    # 7 channels
     (8, 32, 3, True, 20, 22, (2, 2)),     # 8 channels: the NHWC input is one octet plane
+    (32, 24, 3, True, 34, 30, (2, 2)),    # pooled 32-column unit with its last octet past cout
+    (64, 40, 3, True, 26, 42, (1, 2)),    # pooled, N = 48: 16-column units
+    (64, 96, 1, True, 32, 16, (2, 1)),    # pooled 1x1, three 32-column units per block
 ])
 def test_bf16_single_layer(mf, cin, cout, k, pool, h, w, grid):
     layers = [("conv", k, 1, (k - 1) // 2, cout)] + ([("max", 2, 2, 0, 0)] if pool else [])
